@@ -1,0 +1,379 @@
+"""Benchmark of one AdaPLD draft-construction step (lexical anchoring ->
+semantic fallback -> rerank + draft tree) over B sequences on GB300.
+
+Default workload: the largest-context shape (B=8, L=131072, d=8192, 80%
+forced lexical misses, n_max=5, k=32, W=4, D=16, tau=0.1), synthetic and
+seeded, resident in HBM (17.2 GB, far above the 129 MB L2, so no flush is
+needed between steps).  Prints one JSON line.
+
+  python bench.py [--gpus N --steps K --warmup W] [--impl native|reference]
+
+Under torchrun each rank runs its own batch (weak scaling, no collective on
+the data path); rank 0 prints the line with the max-over-ranks time.
+``--impl reference`` times the CPU oracle instead (rank 0 only), on a bounded
+sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "draft-construction steps/sec (B seqs, device-timed) and achieved HBM GB/s vs peak"
+UNIT = "steps/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--config", type=int, default=5)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# --------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed
+    region (read-only queries)."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.idx)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, ValueError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------- oracle timing
+class OracleSample:
+    """A bounded sample of the workload for timing the CPU oracle: one forced
+    lexical miss and one lexical-hit sequence, truncated to ``rows`` positions
+    and generated on the host.  The oracle's cost is linear in the positions,
+    so a full step is extrapolated as n_miss * t_miss * (L-1)/(rows-1) +
+    n_hit * t_hit * L/rows."""
+
+    def __init__(self, cfg_id: int, seed: int, rows: int):
+        from paper_2606_05742_gb300 import synth
+        c = synth.CONFIGS[cfg_id]
+        self.L, B = c["L"], c["B"]
+        self.rows = min(rows, self.L)
+        self.w = synth.make_workload(cfg_id, B=2, L=self.rows, nohit=0.5, seed=seed + 1000)
+        self.miss = int(self.w.forced[0])
+        self.hit = 1 - self.miss
+        self.n_miss = int(synth.forced_set(cfg_id, B, c["nohit"], seed).size)
+        self.n_hit = B - self.n_miss
+        self.desc = (f"oracle (1 thread) on 1 forced-miss + 1 lexical-hit sequence of config "
+                     f"{cfg_id} truncated to {self.rows} positions (d={c['d']}), extrapolated "
+                     f"linearly to {self.n_miss} misses + {self.n_hit} hits of length {self.L}")
+
+    def rate(self) -> float:
+        import oracle
+        w = self.w
+        t = {}
+        for b in (self.miss, self.hit):
+            s = time.perf_counter()
+            oracle.step(w.tokens[b:b + 1], w.lengths[b:b + 1], w.reps[b:b + 1],
+                        w.query[b:b + 1], w.n_max, w.k, w.W, w.D, w.succ_len, w.tau)
+            t[b] = time.perf_counter() - s
+        est = (self.n_miss * t[self.miss] * (self.L - 1) / (self.rows - 1)
+               + self.n_hit * t[self.hit] * self.L / self.rows)
+        return 1.0 / est
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    sample = OracleSample(args.config, args.seed, rows=4096)
+    for _ in range(args.warmup):
+        sample.rate()
+    vals = []
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        vals.append(sample.rate())
+        if time.perf_counter() - t0 > 150:
+            break
+    desc = sample.desc
+    value = statistics.median(vals)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": len(vals), "warmup": args.warmup,
+        "ms_per_step": 1000.0 / value, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(args.config),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(cfg_id):
+    from paper_2606_05742_gb300 import synth
+    c = synth.CONFIGS[cfg_id]
+    return {"workload": f"config{cfg_id}: {synth.describe(cfg_id)} tau={synth.TAU}",
+            "B": c["B"], "L": c["L"], "d": c["d"], "global_batch": c["B"],
+            "l2": "inputs larger than L2 (no flush needed)"}
+
+
+# ---------------------------------------------------------- native arm
+def algorithmic_bytes(w, g, lengths, tokens):
+    """Bytes the step must move at minimum (no re-reads), per kernel."""
+    d, k = w.d, w.k
+    hk = g["hit_kind"]
+    active = hk != 1
+    lex_bytes = int(4 * lengths.sum())
+    sem_rows = int(sum(lengths[b] - 1 for b in range(w.B) if active[b] and lengths[b] >= 2))
+    n_active = int(active.sum())
+    sem_bytes = sem_rows * d * 2 + n_active * d * 2 + 4 * w.B
+    # tree kernel: rerank rows + query for lexical hits, successor scan + rows
+    gathered = 0
+    succ_scan = 0
+    for b in range(w.B):
+        L = int(lengths[b])
+        if hk[b] == 1:
+            gathered += int(g["n_cand"][b]) + 1
+        elif hk[b] == 2:
+            n = int(g["n_nodes"][b])
+            par = g["parents"][b, :n]
+            heads = [i for i in range(1, n) if par[i] == 0]
+            succ_scan += 4 * (L - 1)
+            gathered += 1
+            for h in heads:
+                t = int(g["draft_tokens"][b, h])
+                gathered += min(k, int((tokens[b, : L - 1] == t).sum()))
+    N = g["draft_tokens"].shape[1]
+    out_bytes = w.B * (N * 12 + N * N + k * 8 + 32)
+    tree_bytes = gathered * d * 2 + succ_scan + out_bytes
+    return {"lexical": lex_bytes, "semantic": sem_bytes, "tree": tree_bytes,
+            "step": lex_bytes + sem_bytes + tree_bytes}
+
+
+def run_native(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_05742_gb300 import native, synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    cfg = args.config
+    w = synth.make_workload(cfg, device=str(dev), seed=args.seed + rank)
+    p = native.make_params(w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, 0)
+    eng = native.Engine(w.B, w.ld, w.d, p, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(max(3, args.warmup)):
+        eng.run(w.tokens, w.lengths, w.reps, w.query)
+    torch.cuda.synchronize(dev)
+    if native.read_device_status(eng.ws) != 0:
+        raise RuntimeError("device status raised during warm-up")
+    g = eng.out.to_host()
+    lengths = w.lengths.cpu().numpy()
+    tokens = w.tokens.cpu().numpy()
+    nbytes = algorithmic_bytes(w, g, lengths, tokens)
+
+    # timed region: K steps, CUDA events on the launching stream
+    K = args.steps
+    ev_sem = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+    ev_all = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(K)]
+    for pair in ev_all + ev_sem:        # torch creates CUDA events lazily, on first record
+        for e in pair:
+            e.record(stream)
+    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize(dev)
+    if clocks:
+        clocks.start()
+        time.sleep(0.3)
+    start.record(stream)
+    for i in range(K):
+        # lexical_begin/lexical_end slots carry the per-step bracket, the
+        # semantic pair brackets the semantic kernel alone
+        native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws,
+                    events=native.StepEvents(ev_all[i][0].cuda_event, None,
+                                             ev_sem[i][0].cuda_event, ev_sem[i][1].cuda_event,
+                                             None, ev_all[i][1].cuda_event))
+    end.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier()
+    clk = clocks.stop() if clocks else None
+    total_ms = start.elapsed_time(end)
+    if native.read_device_status(eng.ws) != 0:
+        raise RuntimeError("device status raised during the timed region")
+    sem_ms = [a.elapsed_time(b) for a, b in ev_sem]
+    step_ms = [a.elapsed_time(b) for a, b in ev_all]
+    t = torch.tensor([total_ms], device=dev)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms = float(t.item())
+    ms_per_step = total_ms / K
+    value = world * K / (total_ms / 1000.0)
+
+    # end-to-end through the public API from pinned host buffers
+    e2e = None
+    if not args.no_e2e:
+        tok_h = w.tokens.cpu().pin_memory()
+        len_h = w.lengths.cpu().pin_memory()
+        reps_h = torch.empty(w.reps.shape, dtype=w.reps.dtype, pin_memory=True)
+        reps_h.copy_(w.reps)
+        q_h = w.query.cpu().pin_memory()
+        dev_in = (torch.empty_like(w.tokens), torch.empty_like(w.lengths),
+                  torch.empty_like(w.reps), torch.empty_like(w.query))
+        host_out = [torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+                    for x in eng.out.tensors()]
+        eng.run_from_host(tok_h, len_h, reps_h, q_h, dev_in, host_out)
+        torch.cuda.synchronize(dev)
+        KE = args.e2e_steps
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        barrier()
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for _ in range(KE):
+            h2d, d2h = eng.run_from_host(tok_h, len_h, reps_h, q_h, dev_in, host_out)
+        e1.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier()
+        te = torch.tensor([e0.elapsed_time(e1)], device=dev)
+        if world > 1:
+            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        e2e = {"value": world * KE / (float(te.item()) / 1000.0), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+        del reps_h, dev_in
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    peak, peak_kind = peaks()
+    sem_avg_ms = sum(sem_ms) / len(sem_ms)
+    achieved = nbytes["semantic"] / (sem_avg_ms / 1000.0) / 1e9
+    step_gbs = nbytes["step"] / (ms_per_step / 1000.0) / 1e9
+    cpu = None
+    if not args.no_cpu_baseline:
+        sample = OracleSample(cfg, args.seed, rows=16384)
+        v = statistics.median([sample.rate() for _ in range(3)])
+        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample.desc}
+    hk = g["hit_kind"]
+    conf = workload_config(cfg)
+    conf.update({"parallelism": f"replicas x{world} (batch per GPU)",
+                 "outcomes": {"lexical": int((hk == 1).sum()), "semantic": int((hk == 2).sum()),
+                              "none": int((hk == 0).sum())},
+                 "accumulate": "fp32"})
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
+        "warmup": max(3, args.warmup), "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": conf,
+        "roofline": {"bound": "hbm", "kernel": "semantic_kernel",
+                     "achieved": achieved, "peak": peak, "peak_kind": peak_kind,
+                     "unit": "GB/s", "frac": achieved / peak, "traffic": None,
+                     "algorithmic_bytes": nbytes["semantic"], "avg_launch_ms": sem_avg_ms},
+        "step_hbm": {"achieved": step_gbs, "frac": step_gbs / peak,
+                     "algorithmic_bytes": nbytes["step"],
+                     "median_step_ms": statistics.median(step_ms)},
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 3 * K,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_native(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,287 @@
+/*
+ * adapld.h - C ABI of the GB300 (sm_103a) AdaPLD draft-construction library.
+ *
+ * One call of adapld_step() performs, for B independent sequences, the
+ * per-decoding-step draft construction of AdaPLD (arXiv 2606.05742):
+ *
+ *   1. lexical anchoring (Sec. 3.3, Eq. 3), generalised from the last token to
+ *      the longest suffix n-gram of length <= n_max;
+ *   2. semantic fallback retrieval for sequences without a lexical hit
+ *      (Sec. 3.3, Eq. 4-5): cosine of the query against every cached
+ *      per-position representation, threshold tau, top-k;
+ *   3. hidden-state rerank (Sec. 3.4, Eq. 6-7) and branched reuse construction
+ *      (Sec. 3.5, Eq. 8-15; Algorithm 1): main span copy, branch tokens,
+ *      successor tokens, emitted as a flat draft tree for tree attention
+ *      (Sec. 3.6).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - All array arguments are DEVICE pointers owned by the caller.  The library
+ *    never allocates or frees memory and keeps no state between calls; all
+ *    temporary storage is the caller's workspace (see
+ *    adapld_workspace_bytes()).
+ *  - Work is enqueued asynchronously on `stream`; outputs are valid once the
+ *    stream has been synchronised.  No entry point synchronises the host
+ *    except adapld_read_device_status().  Calls on different streams are
+ *    independent provided they use different workspaces and outputs.
+ *  - Sequence b (0 <= b < B) of the token history is tokens[b*ld .. b*ld+len_b)
+ *    with len_b = lengths[b]; the query anchor is tokens[b*ld + len_b - 1].
+ *  - Representations are bf16, passed as uint16_t bit patterns.  Row j of
+ *    sequence b is reps[(b*ld + j)*d .. +d): the representation that belongs
+ *    to candidate position j, i.e. the prefix state h_{j-1} of Eq. 6 in the
+ *    paper's 1-indexed notation (or the token embedding of Eq. 4 if the
+ *    caller stores those).  query[b*d .. +d) is the current state
+ *    h_{|M|-1}.  Row j*+1 is the successor reference h_{j*} of Eq. 13.
+ *  - Positions are 0-indexed; candidates are positions j in [0, len_b-2].
+ *  - Rankings use one total order: higher cosine first, equal cosines broken
+ *    towards the more recent (larger) position.
+ *  - Return value: ADAPLD_OK (0) or a negative ADAPLD_ERR_* code.  Argument
+ *    errors are detected on the host before anything is enqueued.  Problems
+ *    that depend on device data (a length outside [1, ld]) are reported per
+ *    sequence in the status output instead, never by a device trap.
+ */
+#ifndef ADAPLD_H
+#define ADAPLD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t / CUstream; 0 is the legacy default stream. */
+typedef struct CUstream_st *adapld_stream_t;
+
+/* ---- status codes --------------------------------------------------------- */
+#define ADAPLD_OK 0
+#define ADAPLD_ERR_NULL (-1)          /* a required pointer is NULL            */
+#define ADAPLD_ERR_BATCH (-2)         /* B < 1                                 */
+#define ADAPLD_ERR_NMAX (-3)          /* n_max outside [1, 8]                  */
+#define ADAPLD_ERR_K (-4)             /* k outside [1, 32]                     */
+#define ADAPLD_ERR_WIDTH (-5)         /* branch_width outside [0, 64]          */
+#define ADAPLD_ERR_DRAFT_LEN (-6)     /* draft_len outside [1, 256]            */
+#define ADAPLD_ERR_DIM (-7)           /* d outside [8, 16384] or d % 8 != 0    */
+#define ADAPLD_ERR_ALIGN (-8)         /* reps or query not 16-byte aligned     */
+#define ADAPLD_ERR_WORKSPACE (-9)     /* workspace NULL or too small           */
+#define ADAPLD_ERR_LD (-10)           /* ld < 1                                */
+#define ADAPLD_ERR_TOO_LARGE (-11)    /* B*ld >= 2^31 or tree > 1024 nodes     */
+#define ADAPLD_ERR_SUCC_LEN (-12)     /* succ_len outside [1, 16]              */
+#define ADAPLD_ERR_TOPK_TABLE (-13)   /* next_topk given with Kn < 1           */
+#define ADAPLD_ERR_TAU (-14)          /* tau is NaN                            */
+#define ADAPLD_ERR_CUDA (-20)         /* a CUDA runtime call failed            */
+
+/* ---- retrieval outcome per sequence (Eq. 5, Algorithm 1) ------------------- */
+#define ADAPLD_HIT_NONE 0 /* nothing retrieved: the caller takes an AR step   */
+#define ADAPLD_HIT_LEX 1  /* lexical (strict) hit                             */
+#define ADAPLD_HIT_SEM 2  /* semantic fallback hit                            */
+
+/* ---- per-sequence status bits (adapld_step_out.status) --------------------- */
+#define ADAPLD_SEQ_BAD_LENGTH 1 /* len_b outside [1, ld]: hit NONE, 0 nodes    */
+#define ADAPLD_SEQ_BAD_CANDIDATE 2 /* adapld_build_draft_tree() was given a
+                                      candidate outside [0, len_b-2]: the
+                                      sequence is treated as retrieving nothing */
+
+/* ---- device status bits (adapld_read_device_status) ------------------------ */
+#define ADAPLD_DEV_TIMEOUT 1  /* a bounded wait in a kernel expired; that
+                                 call's outputs are not valid                  */
+#define ADAPLD_DEV_INTERNAL 2 /* an internal index check failed (a bug)       */
+
+/* ---- flags (adapld_params.flags) ------------------------------------------ */
+#define ADAPLD_NO_LEX_RERANK 1u  /* lexical anchor = most recent match; no
+                                    Eq. 6 gathers; lexical scores are NaN    */
+#define ADAPLD_SUCC_ON_STRICT 2u /* successor drafting on lexical hits too
+                                    (the prose of Sec. 3.5; Algorithm 1 runs it
+                                    on semantic hits only, the default)       */
+#define ADAPLD_NO_SEMANTIC 4u    /* lexical-only retrieval (Table 4 ablation) */
+#define ADAPLD_NO_BRANCH 8u      /* no branch or successor paths (Table 4)    */
+#define ADAPLD_NO_SUCC 16u       /* no successor drafting (Table 4)           */
+
+/*
+ * Draft-construction hyper-parameters (Algorithm 1 inputs).
+ *   n_max        longest suffix n-gram tried by lexical anchoring, [1, 8]
+ *   k            candidates kept by retrieval (and successor candidates per
+ *                branch), [1, 32]
+ *   branch_width W: branch tokens before Eq. 11's removal, [0, 64]
+ *                (the paper's K; 8 in its experiments)
+ *   draft_len    D: maximum main-copy length l_m of Eq. 8, [1, 256]
+ *   succ_len     tokens appended per branch by successor drafting, [1, 16]
+ *                (the paper appends one, Eq. 15)
+ *   tau          semantic threshold of Eq. 4 (0.1 in the paper); -INFINITY
+ *                keeps every row (pure top-k)
+ *   flags        ADAPLD_* switches above
+ */
+typedef struct adapld_params {
+    int32_t n_max;
+    int32_t k;
+    int32_t branch_width;
+    int32_t draft_len;
+    int32_t succ_len;
+    float tau;
+    uint32_t flags;
+} adapld_params;
+
+/*
+ * Draft-tree outputs (Sec. 3.6; the flat layout is this library's reading, the
+ * paper prints none).  N = adapld_tree_nodes(params) slots per sequence:
+ * node 0 is the anchor token (parent -1, position len-1), then the main chain
+ * (lexical hits), then per branch its token (parent 0) followed by its
+ * successor tokens, each the child of the previous.  Parents precede
+ * children; position id = len-1+depth; mask[i][j] = 1 iff node j is node i
+ * or one of its ancestors.  Unused slots hold token/parent/position -1 and
+ * mask 0.  A NONE outcome yields the root alone (n_nodes 1); an invalid
+ * length yields n_nodes 0.
+ *   anchor       [B]        j* (Eq. 7), -1 when nothing was retrieved
+ *   draft_tokens [B][N]     int32
+ *   parents      [B][N]     int32
+ *   positions    [B][N]     int32
+ *   mask         [B][N][N]  uint8
+ *   n_nodes      [B]        int32
+ *   stats        [4] int32 or NULL: lexical hits, semantic hits, empty
+ *                retrievals (Eq. 17-18 counts) and branches extended by a
+ *                successor.  Overwritten by adapld_step(); accumulated (not
+ *                cleared) by adapld_build_draft_tree().
+ */
+typedef struct adapld_tree_out {
+    int32_t *anchor;
+    int32_t *draft_tokens;
+    int32_t *parents;
+    int32_t *positions;
+    uint8_t *mask;
+    int32_t *n_nodes;
+    int32_t *stats;
+} adapld_tree_out;
+
+/*
+ * All outputs of adapld_step().  Every pointer except status and stats is
+ * required.
+ *   hit_kind [B]     ADAPLD_HIT_*
+ *   match_n  [B]     length of the matched suffix n-gram (0 unless lexical)
+ *   cand     [B][k]  ranked candidates: for a lexical hit reranked by Eq. 6
+ *                    (recency order with ADAPLD_NO_LEX_RERANK), for a semantic
+ *                    hit by Eq. 4; cand[b][0] = j*.  Padding -1.
+ *   score    [B][k]  float cosines of cand (padding 0; NaN for lexical
+ *                    candidates under ADAPLD_NO_LEX_RERANK)
+ *   n_cand   [B]     number of valid entries in cand
+ *   status   [B]     ADAPLD_SEQ_* bits, or NULL
+ *   tree             draft-tree outputs (see adapld_tree_out)
+ */
+typedef struct adapld_step_out {
+    int32_t *hit_kind;
+    int32_t *match_n;
+    int32_t *cand;
+    float *score;
+    int32_t *n_cand;
+    int32_t *status;
+    adapld_tree_out tree;
+} adapld_step_out;
+
+/* Optional CUDA events recorded around each kernel of adapld_step_ex(), for
+ * timing a single stage inside a step.  Any member may be NULL.  The events
+ * are cudaEvent_t handles, passed as void*. */
+typedef struct adapld_step_events {
+    void *lexical_begin, *lexical_end;
+    void *semantic_begin, *semantic_end;
+    void *tree_begin, *tree_end;
+} adapld_step_events;
+
+/* Node slots of one draft tree: 1 + draft_len + branch_width*(1+succ_len). */
+int32_t adapld_tree_nodes(const adapld_params *p);
+
+/* Workspace bytes needed by any entry point for B sequences of capacity ld and
+ * dimension d under parameters p (0 if the arguments are invalid).  The
+ * workspace is device memory, 256-byte aligned, with no initialisation
+ * required; one workspace may be reused by consecutive calls on one stream. */
+size_t adapld_workspace_bytes(int32_t B, int64_t ld, int32_t d, const adapld_params *p);
+
+/* Human-readable text for a status code (static storage). */
+const char *adapld_status_string(int code);
+
+/*
+ * Lexical anchoring (Sec. 3.3, Eq. 3; generalised to the longest suffix).
+ * For each sequence: n* = the largest n <= min(n_max, len-1) such that the
+ * last n tokens also occur ending at some j <= len-2; the k most recent such
+ * j are written to cand[b][0..n_cand) in descending order, match_n[b] = n*,
+ * hit_kind[b] = ADAPLD_HIT_LEX.  Without a match: match_n 0, n_cand 0,
+ * hit_kind ADAPLD_HIT_NONE.  cand padding is -1.  A length outside [1, ld]
+ * is treated as no match.
+ *   tokens [B][ld] int32, lengths [B] int32; outputs as in adapld_step_out.
+ */
+int adapld_lexical_match(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                         int32_t B, int32_t n_max, int32_t k, int32_t *hit_kind,
+                         int32_t *match_n, int32_t *cand, int32_t *n_cand, void *ws,
+                         size_t ws_bytes, adapld_stream_t stream);
+
+/*
+ * Semantic fallback retrieval (Sec. 3.3, Eq. 4-5), capped at k.
+ * For every selected sequence (active == NULL selects all; otherwise those
+ * with active[b] != 0) with a valid length: score(j) = cos(R_b[j], q_b) for
+ * every j in [0, len-2], computed from bf16 inputs with fp32 accumulation;
+ * rows with score >= tau are kept and the best min(k, count) are written to
+ * cand/score in ranking order, n_cand[b] = count.  Padding: cand -1, score 0.
+ * Rows of unselected sequences are left untouched.  A selected sequence with
+ * an invalid length gets n_cand 0.
+ *   reps  [B][ld][d] bf16 bits, 16-byte aligned, d % 8 == 0
+ *   query [B][d]     bf16 bits, 16-byte aligned
+ *   active [B] uint8 or NULL
+ */
+int adapld_semantic_topk(const uint16_t *reps, int64_t ld, int32_t d, const uint16_t *query,
+                         const int32_t *lengths, const uint8_t *active, int32_t B, int32_t k,
+                         float tau, int32_t *cand, float *score, int32_t *n_cand, void *ws,
+                         size_t ws_bytes, adapld_stream_t stream);
+
+/*
+ * Rerank and draft-tree construction (Sec. 3.4-3.6, Eq. 6-15, Algorithm 1)
+ * from retrieval results already in hit_kind / cand / score / n_cand (as
+ * written by the two retrieval entry points).  For a lexical hit the
+ * candidates are reranked by Eq. 6 in place (cand and score are rewritten in
+ * ranking order; score NaN under ADAPLD_NO_LEX_RERANK); for a semantic hit the
+ * Eq. 4 order is kept.  j* = cand[b][0].
+ * Branch tokens: if next_topk is non-NULL ([B][ld][Kn] int32, the caller's
+ * cached top-Kn next-token ids of the target model at every position, Eq.
+ * 10), the first W non-negative ids of row j*; otherwise the first W
+ * distinct tokens following the ranked candidates, tokens[c+1] (a model-free
+ * reading of the anchor-conditioned next-token distribution).  On a lexical
+ * hit the main path's first token is then removed (Eq. 11).
+ * Successor drafting (Eq. 13-15) runs for semantic hits (and for lexical
+ * ones under ADAPLD_SUCC_ON_STRICT): for branch token b, among the k most
+ * recent positions t <= len-2 holding b, pick the one maximising
+ * cos(R[t], R[j*+1]) and append tokens[t+1 .. t+succ_len] (clipped at
+ * len-1).
+ * status [B] may be NULL.
+ */
+int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                            const uint16_t *reps, int32_t d, const uint16_t *query, int32_t B,
+                            const int32_t *hit_kind, int32_t *cand, float *score,
+                            const int32_t *n_cand, const int32_t *next_topk, int32_t Kn,
+                            const adapld_params *p, const adapld_tree_out *out, int32_t *status,
+                            void *ws, size_t ws_bytes, adapld_stream_t stream);
+
+/*
+ * One full draft-construction step for B sequences: lexical anchoring, the
+ * semantic fallback for the sequences without a lexical hit (unless
+ * ADAPLD_NO_SEMANTIC), then rerank and draft-tree construction, enqueued as
+ * three kernels with no host synchronisation.  Arguments as above;
+ * next_topk may be NULL (then Kn is ignored).
+ */
+int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const uint16_t *reps,
+                int32_t d, const uint16_t *query, const int32_t *next_topk, int32_t Kn, int32_t B,
+                const adapld_params *p, const adapld_step_out *out, void *ws, size_t ws_bytes,
+                adapld_stream_t stream);
+
+/* adapld_step() that also records the given CUDA events around its kernels. */
+int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                   const uint16_t *reps, int32_t d, const uint16_t *query,
+                   const int32_t *next_topk, int32_t Kn, int32_t B, const adapld_params *p,
+                   const adapld_step_out *out, void *ws, size_t ws_bytes,
+                   const adapld_step_events *events, adapld_stream_t stream);
+
+/* Synchronises `stream` and returns in *status the ADAPLD_DEV_* bits raised by
+ * the most recent call that used workspace `ws` (0 = none). */
+int adapld_read_device_status(const void *ws, int32_t *status, adapld_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ADAPLD_H */

@@ -1,0 +1,217 @@
+// C ABI of the library (include/adapld.h): argument validation, workspace
+// layout and stream-ordered kernel launches.  No entry point allocates memory
+// or synchronises the host (except adapld_read_device_status).
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+
+#include "common.cuh"
+
+using namespace adapld;
+
+namespace {
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+int check_params(const adapld_params *p) {
+    if (!p) return ADAPLD_ERR_NULL;
+    if (p->n_max < 1 || p->n_max > 8) return ADAPLD_ERR_NMAX;
+    if (p->k < 1 || p->k > kMaxK) return ADAPLD_ERR_K;
+    if (p->branch_width < 0 || p->branch_width > kMaxW) return ADAPLD_ERR_WIDTH;
+    if (p->draft_len < 1 || p->draft_len > 256) return ADAPLD_ERR_DRAFT_LEN;
+    if (p->succ_len < 1 || p->succ_len > 16) return ADAPLD_ERR_SUCC_LEN;
+    if (std::isnan(p->tau)) return ADAPLD_ERR_TAU;
+    if (adapld_tree_nodes(p) > kMaxNodes) return ADAPLD_ERR_TOO_LARGE;
+    return ADAPLD_OK;
+}
+
+int check_shape(int32_t B, int64_t ld) {
+    if (B < 1) return ADAPLD_ERR_BATCH;
+    if (ld < 1) return ADAPLD_ERR_LD;
+    if ((int64_t)B * ld >= ((int64_t)1 << 31)) return ADAPLD_ERR_TOO_LARGE;
+    return ADAPLD_OK;
+}
+
+int check_dim(int32_t d) {
+    if (d < 8 || d > 16384 || (d % 8) != 0) return ADAPLD_ERR_DIM;
+    return ADAPLD_OK;
+}
+
+int check_ws(void *ws, size_t ws_bytes, int32_t B, int64_t ld, int32_t W) {
+    if (!ws) return ADAPLD_ERR_WORKSPACE;
+    if (!aligned16(ws)) return ADAPLD_ERR_ALIGN;
+    if (ws_bytes < layout_workspace(nullptr, B, ld, W).total_bytes) return ADAPLD_ERR_WORKSPACE;
+    return ADAPLD_OK;
+}
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA; }
+
+int record(void *ev, cudaStream_t s) {
+    if (!ev) return ADAPLD_OK;
+    return cuda_status(cudaEventRecord((cudaEvent_t)ev, s));
+}
+
+#define ADAPLD_TRY(x)                   \
+    do {                                \
+        int rc_ = (x);                  \
+        if (rc_ != ADAPLD_OK) return rc_; \
+    } while (0)
+
+}  // namespace
+
+extern "C" {
+
+int32_t adapld_tree_nodes(const adapld_params *p) {
+    if (!p) return 0;
+    return 1 + p->draft_len + p->branch_width * (1 + p->succ_len);
+}
+
+size_t adapld_workspace_bytes(int32_t B, int64_t ld, int32_t d, const adapld_params *p) {
+    if (check_shape(B, ld) != ADAPLD_OK || check_dim(d) != ADAPLD_OK) return 0;
+    const int32_t W = p ? p->branch_width : 1;
+    return layout_workspace(nullptr, B, ld, W).total_bytes;
+}
+
+const char *adapld_status_string(int code) {
+    switch (code) {
+        case ADAPLD_OK: return "ok";
+        case ADAPLD_ERR_NULL: return "a required pointer is NULL";
+        case ADAPLD_ERR_BATCH: return "batch size B must be >= 1";
+        case ADAPLD_ERR_NMAX: return "n_max must be in [1, 8]";
+        case ADAPLD_ERR_K: return "k must be in [1, 32]";
+        case ADAPLD_ERR_WIDTH: return "branch_width must be in [0, 64]";
+        case ADAPLD_ERR_DRAFT_LEN: return "draft_len must be in [1, 256]";
+        case ADAPLD_ERR_DIM: return "d must be a multiple of 8 in [8, 16384]";
+        case ADAPLD_ERR_ALIGN: return "reps, query and workspace must be 16-byte aligned";
+        case ADAPLD_ERR_WORKSPACE: return "workspace missing or smaller than adapld_workspace_bytes()";
+        case ADAPLD_ERR_LD: return "ld must be >= 1";
+        case ADAPLD_ERR_TOO_LARGE: return "B*ld must be < 2^31 and the tree at most 1024 nodes";
+        case ADAPLD_ERR_SUCC_LEN: return "succ_len must be in [1, 16]";
+        case ADAPLD_ERR_TOPK_TABLE: return "next_topk needs Kn in [1, 64]";
+        case ADAPLD_ERR_TAU: return "tau must not be NaN";
+        case ADAPLD_ERR_CUDA: return "a CUDA runtime call failed";
+        default: return "unknown status";
+    }
+}
+
+int adapld_lexical_match(const int32_t *tokens, int64_t ld, const int32_t *lengths, int32_t B,
+                         int32_t n_max, int32_t k, int32_t *hit_kind, int32_t *match_n,
+                         int32_t *cand, int32_t *n_cand, void *ws, size_t ws_bytes,
+                         adapld_stream_t stream) {
+    if (!tokens || !lengths || !hit_kind || !match_n || !cand || !n_cand) return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_shape(B, ld));
+    if (n_max < 1 || n_max > 8) return ADAPLD_ERR_NMAX;
+    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
+    ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
+    cudaStream_t s = (cudaStream_t)stream;
+    Workspace w = layout_workspace(ws, B, ld, 1);
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    LexLaunch a{tokens, ld, lengths, B, n_max, k, hit_kind, match_n, cand, n_cand,
+                nullptr, nullptr, nullptr, false};
+    return cuda_status(launch_lexical(a, w, s));
+}
+
+int adapld_semantic_topk(const uint16_t *reps, int64_t ld, int32_t d, const uint16_t *query,
+                         const int32_t *lengths, const uint8_t *active, int32_t B, int32_t k,
+                         float tau, int32_t *cand, float *score, int32_t *n_cand, void *ws,
+                         size_t ws_bytes, adapld_stream_t stream) {
+    if (!reps || !query || !lengths || !cand || !score || !n_cand) return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_dim(d));
+    if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
+    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
+    if (std::isnan(tau)) return ADAPLD_ERR_TAU;
+    ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
+    cudaStream_t s = (cudaStream_t)stream;
+    Workspace w = layout_workspace(ws, B, ld, 1);
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    SemLaunch a{reps, ld, d, query, lengths, active, B, k, tau, cand, score, n_cand,
+                nullptr, false};
+    return cuda_status(launch_semantic(a, w, s));
+}
+
+int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                            const uint16_t *reps, int32_t d, const uint16_t *query, int32_t B,
+                            const int32_t *hit_kind, int32_t *cand, float *score,
+                            const int32_t *n_cand, const int32_t *next_topk, int32_t Kn,
+                            const adapld_params *p, const adapld_tree_out *out, int32_t *status,
+                            void *ws, size_t ws_bytes, adapld_stream_t stream) {
+    if (!tokens || !lengths || !reps || !query || !hit_kind || !cand || !score || !n_cand || !out)
+        return ADAPLD_ERR_NULL;
+    if (!out->anchor || !out->draft_tokens || !out->parents || !out->positions || !out->mask ||
+        !out->n_nodes)
+        return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_params(p));
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_dim(d));
+    if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
+    if (next_topk && (Kn < 1 || Kn > kMaxW)) return ADAPLD_ERR_TOPK_TABLE;
+    ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, p->branch_width));
+    cudaStream_t s = (cudaStream_t)stream;
+    Workspace w = layout_workspace(ws, B, ld, p->branch_width);
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    TreeLaunch a{tokens, ld, lengths, reps, d, query, B, hit_kind, cand, score, n_cand,
+                 next_topk, next_topk ? Kn : 0, *p, *out, status};
+    return cuda_status(launch_tree(a, w, s));
+}
+
+int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                   const uint16_t *reps, int32_t d, const uint16_t *query,
+                   const int32_t *next_topk, int32_t Kn, int32_t B, const adapld_params *p,
+                   const adapld_step_out *out, void *ws, size_t ws_bytes,
+                   const adapld_step_events *ev, adapld_stream_t stream) {
+    if (!tokens || !lengths || !reps || !query || !out) return ADAPLD_ERR_NULL;
+    if (!out->hit_kind || !out->match_n || !out->cand || !out->score || !out->n_cand)
+        return ADAPLD_ERR_NULL;
+    const adapld_tree_out &to = out->tree;
+    if (!to.anchor || !to.draft_tokens || !to.parents || !to.positions || !to.mask || !to.n_nodes)
+        return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_params(p));
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_dim(d));
+    if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
+    if (next_topk && (Kn < 1 || Kn > kMaxW)) return ADAPLD_ERR_TOPK_TABLE;
+    ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, p->branch_width));
+    cudaStream_t s = (cudaStream_t)stream;
+    Workspace w = layout_workspace(ws, B, ld, p->branch_width);
+    const bool semantic = !(p->flags & ADAPLD_NO_SEMANTIC);
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+
+    ADAPLD_TRY(record(ev ? ev->lexical_begin : nullptr, s));
+    LexLaunch la{tokens, ld, lengths, B, p->n_max, p->k, out->hit_kind, out->match_n, out->cand,
+                 out->n_cand, out->score, out->status, to.stats, semantic};
+    ADAPLD_TRY(cuda_status(launch_lexical(la, w, s)));
+    ADAPLD_TRY(record(ev ? ev->lexical_end : nullptr, s));
+
+    if (semantic) {
+        ADAPLD_TRY(record(ev ? ev->semantic_begin : nullptr, s));
+        SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
+                     out->n_cand, out->hit_kind, true};
+        ADAPLD_TRY(cuda_status(launch_semantic(sa, w, s)));
+        ADAPLD_TRY(record(ev ? ev->semantic_end : nullptr, s));
+    }
+
+    ADAPLD_TRY(record(ev ? ev->tree_begin : nullptr, s));
+    TreeLaunch ta{tokens, ld, lengths, reps, d, query, B, out->hit_kind, out->cand, out->score,
+                  out->n_cand, next_topk, next_topk ? Kn : 0, *p, to, out->status};
+    ADAPLD_TRY(cuda_status(launch_tree(ta, w, s)));
+    return record(ev ? ev->tree_end : nullptr, s);
+}
+
+int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const uint16_t *reps,
+                int32_t d, const uint16_t *query, const int32_t *next_topk, int32_t Kn, int32_t B,
+                const adapld_params *p, const adapld_step_out *out, void *ws, size_t ws_bytes,
+                adapld_stream_t stream) {
+    return adapld_step_ex(tokens, ld, lengths, reps, d, query, next_topk, Kn, B, p, out, ws,
+                          ws_bytes, nullptr, stream);
+}
+
+int adapld_read_device_status(const void *ws, int32_t *status, adapld_stream_t stream) {
+    if (!ws || !status) return ADAPLD_ERR_NULL;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaMemcpyAsync(status, ws, sizeof(int32_t), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return ADAPLD_ERR_CUDA;
+    return cuda_status(cudaStreamSynchronize(s));
+}
+
+}  // extern "C"

@@ -1,0 +1,298 @@
+// Shared device helpers and the workspace layout of the AdaPLD sm_103a library.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "adapld.h"
+
+namespace adapld {
+
+// ---- limits and tiling ------------------------------------------------------
+constexpr int kMaxK = 32;          // candidates per list (one per warp lane)
+constexpr int kMaxW = 64;          // branch width
+constexpr int kMaxNodes = 1024;    // draft-tree node slots
+constexpr int kChunk1 = 4096;      // lexical scan: positions per CTA
+constexpr int kThreads1 = 256;
+constexpr int kSlice4 = 8192;      // successor scan: positions per CTA
+constexpr int kThreads4 = 512;
+constexpr int kMaxGrid2 = 1024;    // semantic kernel: CTAs at most
+constexpr int kConsumers2 = 256;   // semantic kernel: consumer threads (8 warps)
+constexpr int kMaxStages2 = 8;
+constexpr int kSlotInts = 68;      // partial top-k slot: count, 32 ids, 32 scores (+pad)
+constexpr int kPart1Ints = 2 + kMaxK;
+constexpr int kPart4Ints = 1 + kMaxK;
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded waits: 2 s
+
+// ---- workspace --------------------------------------------------------------
+// Counters (zeroed by every call) come first, then scratch that every call
+// fully rewrites before reading.
+struct Workspace {
+    int32_t *dev_status;     // [1]  ADAPLD_DEV_* bits
+    int32_t *global_ticket;  // [1]  lexical kernel: CTAs done with their sequence
+    int32_t *ticket1;        // [B]  lexical kernel: chunks done per sequence
+    int32_t *done2;          // [B]  semantic kernel: CTAs done per sequence
+    int32_t *ticket4;        // [B]  tree kernel: slices done per sequence
+    int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
+    int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
+    int32_t *slots2;         // [B + kMaxGrid2][kSlotInts] partial top-k lists
+    int32_t *part4;          // [B][S4][W][kPart4Ints] per-slice successor lists
+    size_t counters_bytes;
+    size_t total_bytes;
+    int C1, S4, W;
+};
+
+__host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+__host__ __device__ inline int chunks_of(int64_t n, int64_t per) {
+    return (int)((n < 1 ? 1 : n + per - 1) / per);
+}
+
+// Lays the workspace out at `base` (NULL: sizing only).
+inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) {
+    Workspace w{};
+    w.C1 = chunks_of(ld - 1, kChunk1);
+    w.S4 = chunks_of(ld - 1, kSlice4);
+    w.W = W < 1 ? 1 : W;
+    char *p = (char *)base;
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        char *r = p ? p + off : nullptr;
+        off = align_up(off + bytes, 256);
+        return r;
+    };
+    w.dev_status = (int32_t *)take(sizeof(int32_t) * (2 + 3 * (size_t)B));
+    if (p) {
+        w.global_ticket = w.dev_status + 1;
+        w.ticket1 = w.dev_status + 2;
+        w.done2 = w.ticket1 + B;
+        w.ticket4 = w.done2 + B;
+    }
+    w.counters_bytes = sizeof(int32_t) * (2 + 3 * (size_t)B);
+    w.part1 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1 * kPart1Ints);
+    w.plan = (int64_t *)take(sizeof(int64_t) * ((size_t)B + 1));
+    w.slots2 = (int32_t *)take(sizeof(int32_t) * ((size_t)B + kMaxGrid2) * kSlotInts);
+    w.part4 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.S4 * w.W * kPart4Ints);
+    w.total_bytes = off;
+    return w;
+}
+
+// ---- device helpers ------------------------------------------------------------
+#ifdef __CUDACC__
+
+__device__ __forceinline__ uint64_t global_ns() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+// The ranking order used everywhere: higher score first, ties to the larger
+// (more recent) position.
+__device__ __forceinline__ bool better(float sa, int ja, float sb, int jb) {
+    return sa > sb || (sa == sb && ja > jb);
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+                 : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Waits for the phase of `bar` with the given parity to complete; gives up
+// after kWaitLimitNs and returns false.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    uint64_t t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > kWaitLimitNs) return false;
+    }
+    return true;
+}
+
+// One bulk (non-tensor) TMA copy global -> shared, completing on `bar`.
+// Both addresses 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes,
+                                         uint64_t *bar, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1], %2, [%3], %4;" ::"r"(smem_u32(dst)),
+        "l"(src), "r"(bytes), "r"(smem_u32(bar)), "l"(policy)
+        : "memory");
+}
+
+__device__ __forceinline__ uint64_t l2_evict_first_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ void named_bar_sync(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void named_bar_arrive(int id, int count) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ uint4 ldg_nc_v4(const void *p) {
+    uint4 r;
+    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+                 : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ float bf16lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+// Cosine from fp32 accumulators, zero when either norm is zero.
+__device__ __forceinline__ float cosine_from(float dot, float ss, float qss) {
+    return (ss > 0.f && qss > 0.f) ? dot / (sqrtf(ss) * sqrtf(qss)) : 0.f;
+}
+
+// Warp-resident top-k list: lane i < n holds the i-th best (s, j).
+struct WarpTopK {
+    float s;
+    int j;
+    int n;  // warp-uniform count
+
+    __device__ __forceinline__ void reset() {
+        s = -INFINITY;
+        j = -1;
+        n = 0;
+    }
+
+    // Inserts the candidates held by the lanes with `want` set.  All 32 lanes
+    // must call.  k <= 32.
+    __device__ __forceinline__ void insert(bool want, float cs, int cj, int k) {
+        const int lane = threadIdx.x & 31;
+        float ks = __shfl_sync(0xffffffffu, s, k - 1);
+        int kj = __shfl_sync(0xffffffffu, j, k - 1);
+        unsigned m = __ballot_sync(0xffffffffu, want && (n < k || better(cs, cj, ks, kj)));
+        while (m) {
+            int src = __ffs(m) - 1;
+            m &= m - 1;
+            float xs = __shfl_sync(0xffffffffu, cs, src);
+            int xj = __shfl_sync(0xffffffffu, cj, src);
+            if (n == k && !better(xs, xj, ks, kj)) continue;
+            int pos = __popc(__ballot_sync(0xffffffffu, lane < n && better(s, j, xs, xj)));
+            float us = __shfl_up_sync(0xffffffffu, s, 1);
+            int uj = __shfl_up_sync(0xffffffffu, j, 1);
+            if (lane > pos) {
+                s = us;
+                j = uj;
+            } else if (lane == pos) {
+                s = xs;
+                j = xj;
+            }
+            n = n < k ? n + 1 : k;
+            ks = __shfl_sync(0xffffffffu, s, k - 1);
+            kj = __shfl_sync(0xffffffffu, j, k - 1);
+        }
+    }
+};
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ int warp_max_i(int v) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) v = max(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+#endif  // __CUDACC__
+
+// ---- host-side launchers (one per kernel) ---------------------------------------
+struct LexLaunch {
+    const int32_t *tokens;
+    int64_t ld;
+    const int32_t *lengths;
+    int32_t B, n_max, k;
+    int32_t *hit_kind, *match_n, *cand, *n_cand;
+    float *score;            // optional: zeroed for every sequence
+    int32_t *status;         // optional
+    int32_t *stats;          // optional: zeroed
+    bool build_plan;         // also build the semantic plan (step path)
+};
+cudaError_t launch_lexical(const LexLaunch &a, const Workspace &ws, cudaStream_t s);
+
+// Semantic work plan for the standalone semantic entry point (one CTA):
+// ws.plan[b] = rows of earlier selected sequences (selection: active == NULL
+// means all, else active[b] != 0; a sequence needs a valid length); selected
+// sequences get default outputs (no candidates).
+cudaError_t launch_plan(const int32_t *lengths, int64_t ld, int32_t B, const uint8_t *active,
+                        int32_t k, int32_t *cand, float *score, int32_t *n_cand,
+                        const Workspace &ws, cudaStream_t s);
+
+struct SemLaunch {
+    const uint16_t *reps;
+    int64_t ld;
+    int32_t d;
+    const uint16_t *query;
+    const int32_t *lengths;
+    const uint8_t *active;   // standalone path (plan built by a separate kernel)
+    int32_t B, k;
+    float tau;
+    int32_t *cand;
+    float *score;
+    int32_t *n_cand;
+    int32_t *hit_kind;       // step path: set SEM / NONE at the final merge
+    bool plan_ready;         // step path: the lexical kernel built the plan
+};
+cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_t s);
+
+struct TreeLaunch {
+    const int32_t *tokens;
+    int64_t ld;
+    const int32_t *lengths;
+    const uint16_t *reps;
+    int32_t d;
+    const uint16_t *query;
+    int32_t B;
+    const int32_t *hit_kind;
+    int32_t *cand;
+    float *score;
+    const int32_t *n_cand;
+    const int32_t *next_topk;
+    int32_t Kn;
+    adapld_params p;
+    adapld_tree_out out;
+    int32_t *status;
+};
+cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s);
+
+}  // namespace adapld

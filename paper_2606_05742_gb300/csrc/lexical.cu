@@ -1,0 +1,242 @@
+// Lexical anchoring (Sec. 3.3, Eq. 3, generalised to the longest suffix
+// n-gram) and the semantic work plan.
+//
+// Grid (C1 chunks, B sequences), 256 threads.  A CTA stages one chunk of
+// 4096 candidate positions (plus an n_max-1 token halo) in shared memory,
+// computes for each position j the length m(j) of the backward match
+// M[j-i] == M[len-1-i], i < m(j) <= min(n_max, len-1), reduces the chunk
+// maximum and collects the k most recent positions reaching it with warp
+// ballots.  The last CTA of a sequence (atomic ticket) merges the chunk
+// results: n* = max m, candidates = the k most recent positions with
+// m(j) = n*.  On the step path the last sequence to finish also writes the
+// prefix sums of the semantic fallback's rows (the plan), so the semantic
+// kernel can balance rows over the whole GPU without a host round trip.
+#include "common.cuh"
+
+namespace adapld {
+
+namespace {
+
+struct LexArgs {
+    LexLaunch p;
+    Workspace ws;
+};
+
+// Block-wide exclusive scan of one int64 per thread (256 threads).
+__device__ int64_t block_exclusive_scan(int64_t v, int64_t *total, int64_t *scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int64_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int64_t u = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += u;
+    }
+    if (lane == 31) scratch[warp] = incl;
+    __syncthreads();
+    int64_t before = 0, all = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+        if (w < warp) before += scratch[w];
+        all += scratch[w];
+    }
+    __syncthreads();
+    *total = all;
+    return before + incl - v;
+}
+
+// One CTA builds plan[0..B] (see launch_plan in common.cuh).
+__device__ void build_plan_cta(const int32_t *lengths, int64_t ld, int32_t B,
+                               const int32_t *hit_kind, const uint8_t *active, int64_t *plan,
+                               bool init_out, int32_t k, int32_t *cand, float *score,
+                               int32_t *n_cand) {
+    __shared__ int64_t scratch[32];
+    int64_t carry = 0;
+    for (int base = 0; base < B; base += blockDim.x) {
+        const int b = base + threadIdx.x;
+        int64_t rows = 0;
+        if (b < B) {
+            const int len = lengths[b];
+            const bool valid = len >= 1 && (int64_t)len <= ld;
+            bool sel;
+            if (hit_kind)
+                sel = __ldcg(hit_kind + b) != ADAPLD_HIT_LEX;
+            else
+                sel = active ? active[b] != 0 : true;
+            if (sel && valid) rows = len - 1;
+            if (sel && init_out) {
+                n_cand[b] = 0;
+                for (int i = 0; i < k; ++i) {
+                    cand[(int64_t)b * k + i] = -1;
+                    score[(int64_t)b * k + i] = 0.f;
+                }
+            }
+        }
+        int64_t total;
+        const int64_t ex = block_exclusive_scan(rows, &total, scratch);
+        if (b < B) plan[b] = carry + ex;
+        carry += total;
+    }
+    if (threadIdx.x == 0) plan[B] = carry;
+}
+
+__global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
+    const LexLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int tok[kChunk1 + 8];
+    __shared__ int suf[8];
+    __shared__ int wval[kThreads1 / 32];
+    __shared__ int list[kMaxK];
+    __shared__ int flag;
+
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int b = blockIdx.y, c = blockIdx.x;
+    const int len = a.lengths[b];
+    const bool valid = len >= 1 && (int64_t)len <= a.ld;
+    const int nj = valid ? len - 1 : 0;               // candidates j in [0, len-2]
+    const int top = valid ? min(a.n_max, len - 1) : 0;
+    const int j0 = c * kChunk1;
+    const int j1 = min(j0 + kChunk1, nj);
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+
+    if (a.stats && b == 0 && c == 0 && t < 4) a.stats[t] = 0;
+
+    int cmax = 0, cnt = 0;
+    if (j0 < j1 && top > 0) {
+        const int h = top - 1;  // halo before the chunk
+        for (int i = t; i < j1 - j0 + h; i += kThreads1) {
+            const int p = j0 - h + i;
+            tok[i] = p >= 0 ? M[p] : 0;
+        }
+        if (t < top) suf[t] = M[len - 1 - t];
+        __syncthreads();
+        int m[kChunk1 / kThreads1];
+        int mymax = 0;
+#pragma unroll
+        for (int e = 0; e < kChunk1 / kThreads1; ++e) {
+            const int p = j0 + e * kThreads1 + t;
+            int mm = 0;
+            if (p < j1) {
+                while (mm < top && p - mm >= 0 && tok[p - mm - j0 + h] == suf[mm]) ++mm;
+            }
+            m[e] = mm;
+            mymax = max(mymax, mm);
+        }
+        mymax = warp_max_i(mymax);
+        if (lane == 0) wval[warp] = mymax;
+        __syncthreads();
+        for (int w = 0; w < kThreads1 / 32; ++w) cmax = max(cmax, wval[w]);
+        __syncthreads();
+        if (cmax > 0) {
+            // most recent first: position blocks from the top, within a block
+            // higher warps and then higher lanes first
+#pragma unroll
+            for (int e = kChunk1 / kThreads1 - 1; e >= 0; --e) {
+                const int p = j0 + e * kThreads1 + t;
+                const bool hit = p < j1 && m[e] == cmax;
+                const unsigned bal = __ballot_sync(0xffffffffu, hit);
+                if (lane == 0) wval[warp] = __popc(bal);
+                __syncthreads();
+                int above = 0, all = 0;
+                for (int w = 0; w < kThreads1 / 32; ++w) {
+                    if (w > warp) above += wval[w];
+                    all += wval[w];
+                }
+                const unsigned higher = lane == 31 ? 0u : (bal & (0xffffffffu << (lane + 1)));
+                const int rank = cnt + above + __popc(higher);
+                if (hit && rank < a.k) list[rank] = p;
+                cnt += all;
+                __syncthreads();
+                if (cnt >= a.k) break;
+            }
+            cnt = min(cnt, a.k);
+        }
+    }
+
+    int32_t *part = ws.part1 + ((int64_t)b * ws.C1 + c) * kPart1Ints;
+    __syncthreads();
+    if (t == 0) {
+        part[0] = cmax;
+        part[1] = cnt;
+    }
+    if (t < cnt) part[2 + t] = list[t];
+    __threadfence();
+    __syncthreads();
+    if (t == 0) flag = atomicAdd(ws.ticket1 + b, 1) == (int)gridDim.x - 1;
+    __syncthreads();
+    if (!flag) return;
+    __threadfence();
+
+    // ---- last chunk of sequence b: merge ------------------------------------
+    if (warp == 0) {
+        int best = 0;
+        for (int cc = lane; cc < (int)gridDim.x; cc += 32)
+            best = max(best, __ldcg(ws.part1 + ((int64_t)b * ws.C1 + cc) * kPart1Ints));
+        best = warp_max_i(best);
+        int total = 0;
+        int32_t *cb = a.cand + (int64_t)b * a.k;
+        if (best > 0) {
+            for (int cc = (int)gridDim.x - 1; cc >= 0 && total < a.k; --cc) {
+                const int32_t *pp = ws.part1 + ((int64_t)b * ws.C1 + cc) * kPart1Ints;
+                if (__ldcg(pp) != best) continue;
+                const int n = __ldcg(pp + 1);
+                const int take = min(n, a.k - total);
+                if (lane < take) cb[total + lane] = __ldcg(pp + 2 + lane);
+                total += take;
+            }
+        }
+        if (lane >= total && lane < a.k) cb[lane] = -1;
+        if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
+        if (lane == 0) {
+            a.match_n[b] = best;
+            a.n_cand[b] = total;
+            a.hit_kind[b] = best > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
+            if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
+        }
+    }
+    if (!a.build_plan) return;
+
+    // ---- last sequence overall: semantic plan ---------------------------------
+    __threadfence();
+    __syncthreads();
+    if (t == 0) flag = atomicAdd(ws.global_ticket, 1) == a.B - 1;
+    __syncthreads();
+    if (!flag) return;
+    __threadfence();
+    build_plan_cta(a.lengths, a.ld, a.B, a.hit_kind, nullptr, ws.plan, false, a.k, nullptr,
+                   nullptr, nullptr);
+}
+
+struct PlanArgs {
+    const int32_t *lengths;
+    int64_t ld;
+    int32_t B;
+    const uint8_t *active;
+    int32_t k;
+    int32_t *cand;
+    float *score;
+    int32_t *n_cand;
+    int64_t *plan;
+};
+
+__global__ void __launch_bounds__(kThreads1) plan_kernel(PlanArgs a) {
+    build_plan_cta(a.lengths, a.ld, a.B, nullptr, a.active, a.plan, true, a.k, a.cand, a.score,
+                   a.n_cand);
+}
+
+}  // namespace
+
+cudaError_t launch_lexical(const LexLaunch &a, const Workspace &ws, cudaStream_t s) {
+    LexArgs args{a, ws};
+    dim3 grid(ws.C1, a.B);
+    lexical_kernel<<<grid, kThreads1, 0, s>>>(args);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_plan(const int32_t *lengths, int64_t ld, int32_t B, const uint8_t *active,
+                        int32_t k, int32_t *cand, float *score, int32_t *n_cand,
+                        const Workspace &ws, cudaStream_t s) {
+    PlanArgs a{lengths, ld, B, active, k, cand, score, n_cand, ws.plan};
+    plan_kernel<<<1, kThreads1, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace adapld

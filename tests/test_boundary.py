@@ -1,0 +1,150 @@
+"""The C-ABI boundary without a GPU: the library builds, loads and exports every
+function declared in include/adapld.h, and argument errors are reported with
+the documented codes before anything is enqueued (every call here fails
+validation, so no CUDA work is attempted)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2606_05742_gb300 import build, native
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "adapld.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return native.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^[A-Za-z_][\w\s\*]*?\b(adapld_\w+)\s*\(", src, flags=re.M)))
+
+
+def test_header_declares_expected_entry_points():
+    decl = declared_functions()
+    for name in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
+                 "adapld_step"):
+        assert name in decl
+    assert sorted(native.EXPORTED) == decl
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_status_strings(lib):
+    for code in (0, -1, -2, -3, -4, -5, -6, -7, -8, -9, -10, -11, -12, -13, -14, -20):
+        s = native.status_string(code)
+        assert s and s != "unknown status"
+    assert native.status_string(-999) == "unknown status"
+
+
+def test_tree_nodes_and_workspace(lib):
+    p = native.make_params(5, 32, 4, 16, 1)
+    assert native.tree_nodes(p) == 1 + 16 + 4 * 2
+    assert native.workspace_bytes(8, 131072, 8192, p) > 0
+    assert native.workspace_bytes(0, 10, 8, p) == 0          # bad B
+    assert native.workspace_bytes(1, 10, 12, p) == 0         # d % 8 != 0
+    assert native.workspace_bytes(1, 10, 16392, p) == 0      # d too large
+    assert native.workspace_bytes(1, 1 << 31, 8, p) == 0     # B*ld too large
+    assert native.workspace_bytes(1, 0, 8, p) == 0           # bad ld
+
+
+FAKE = 1 << 20  # a 16-byte aligned non-null address; never dereferenced here
+
+
+def _step(lib, **kw):
+    a = dict(tokens=FAKE, ld=64, lengths=FAKE, reps=FAKE, d=16, query=FAKE, next_topk=None, Kn=0,
+             B=2, p=native.make_params(3, 8, 2, 8), ws=FAKE, ws_bytes=1 << 30)
+    a.update(kw)
+    so = native.StepOut(FAKE, FAKE, FAKE, FAKE, FAKE, None,
+                        native.TreeOut(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None))
+    if "out" in kw:
+        so = kw["out"]
+    return lib.adapld_step(a["tokens"], a["ld"], a["lengths"], a["reps"], a["d"], a["query"],
+                           a["next_topk"], a["Kn"], a["B"], ctypes.byref(a["p"]),
+                           ctypes.byref(so), a["ws"], a["ws_bytes"], None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(tokens=None), -1),
+    (dict(reps=None), -1),
+    (dict(B=0), -2),
+    (dict(p=native.make_params(0, 8, 2, 8)), -3),
+    (dict(p=native.make_params(9, 8, 2, 8)), -3),
+    (dict(p=native.make_params(3, 0, 2, 8)), -4),
+    (dict(p=native.make_params(3, 33, 2, 8)), -4),
+    (dict(p=native.make_params(3, 8, -1, 8)), -5),
+    (dict(p=native.make_params(3, 8, 65, 8)), -5),
+    (dict(p=native.make_params(3, 8, 2, 0)), -6),
+    (dict(p=native.make_params(3, 8, 2, 257)), -6),
+    (dict(d=12), -7),
+    (dict(d=0), -7),
+    (dict(reps=FAKE + 4), -8),
+    (dict(query=FAKE + 8), -8),
+    (dict(ws=None), -9),
+    (dict(ws_bytes=16), -9),
+    (dict(ld=0), -10),
+    (dict(ld=1 << 31), -11),
+    (dict(p=native.make_params(3, 8, 64, 256, 16)), -11),
+    (dict(p=native.make_params(3, 8, 2, 8, 0)), -12),
+    (dict(p=native.make_params(3, 8, 2, 8, 17)), -12),
+    (dict(next_topk=FAKE, Kn=0), -13),
+    (dict(next_topk=FAKE, Kn=65), -13),
+    (dict(p=native.make_params(3, 8, 2, 8, 1, float("nan"))), -14),
+])
+def test_step_argument_errors(lib, kw, code):
+    assert _step(lib, **kw) == code
+
+
+def test_step_null_outputs(lib):
+    so = native.StepOut(FAKE, FAKE, None, FAKE, FAKE, None,
+                        native.TreeOut(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None))
+    assert _step(lib, out=so) == -1
+    so = native.StepOut(FAKE, FAKE, FAKE, FAKE, FAKE, None,
+                        native.TreeOut(FAKE, FAKE, FAKE, FAKE, None, FAKE, None))
+    assert _step(lib, out=so) == -1
+
+
+def test_entry_point_argument_errors(lib):
+    L = lib
+    assert L.adapld_lexical_match(FAKE, 64, FAKE, 0, 3, 8, FAKE, FAKE, FAKE, FAKE, FAKE,
+                                  1 << 30, None) == -2
+    assert L.adapld_lexical_match(FAKE, 64, FAKE, 2, 9, 8, FAKE, FAKE, FAKE, FAKE, FAKE,
+                                  1 << 30, None) == -3
+    assert L.adapld_lexical_match(FAKE, 64, FAKE, 2, 3, 8, None, FAKE, FAKE, FAKE, FAKE,
+                                  1 << 30, None) == -1
+    assert L.adapld_lexical_match(FAKE, 64, FAKE, 2, 3, 8, FAKE, FAKE, FAKE, FAKE, FAKE,
+                                  8, None) == -9
+    assert L.adapld_semantic_topk(FAKE, 64, 16, FAKE, FAKE, None, 2, 40, 0.1, FAKE, FAKE, FAKE,
+                                  FAKE, 1 << 30, None) == -4
+    assert L.adapld_semantic_topk(FAKE + 2, 64, 16, FAKE, FAKE, None, 2, 8, 0.1, FAKE, FAKE,
+                                  FAKE, FAKE, 1 << 30, None) == -8
+    assert L.adapld_semantic_topk(FAKE, 64, 20, FAKE, FAKE, None, 2, 8, 0.1, FAKE, FAKE, FAKE,
+                                  FAKE, 1 << 30, None) == -7
+    to = native.TreeOut(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None)
+    p = native.make_params(3, 8, 2, 8)
+    assert L.adapld_build_draft_tree(FAKE, 64, FAKE, FAKE, 16, FAKE, 2, FAKE, FAKE, FAKE, FAKE,
+                                     None, 0, ctypes.byref(p), None, None, FAKE, 1 << 30,
+                                     None) == -1
+    bad = native.make_params(3, 8, 2, 8, 1)
+    bad.k = 0
+    assert L.adapld_build_draft_tree(FAKE, 64, FAKE, FAKE, 16, FAKE, 2, FAKE, FAKE, FAKE, FAKE,
+                                     None, 0, ctypes.byref(bad), ctypes.byref(to), None, FAKE,
+                                     1 << 30, None) == -4
+    v = ctypes.c_int32(0)
+    assert L.adapld_read_device_status(None, ctypes.byref(v), None) == -1
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(native, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(native, "_lib", None)
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        native.load()

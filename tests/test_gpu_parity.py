@@ -1,0 +1,340 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
+same seeded inputs.  Integer outputs bit-exact, scores within 1e-2, cosine
+decisions tie-tolerant within the fp32 error bound (see tests/parity.py)."""
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2606_05742_gb300 import build, native, synth
+from tests import parity
+from tests.conftest import load_golden
+
+pytestmark = pytest.mark.gpu
+NEG_INF = float("-inf")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    build.build()
+    native.load()
+
+
+def to_dev(w):
+    """numpy workload -> torch CUDA tensors (tokens, lengths, reps, query)."""
+    tok = torch.from_numpy(np.ascontiguousarray(w.tokens)).cuda()
+    ln = torch.from_numpy(np.ascontiguousarray(w.lengths)).cuda()
+    reps = torch.from_numpy(np.ascontiguousarray(w.reps).view(np.int16)).cuda().view(torch.bfloat16)
+    q = torch.from_numpy(np.ascontiguousarray(w.query).view(np.int16)).cuda().view(torch.bfloat16)
+    return tok, ln, reps, q
+
+
+def P_of(w, tau=None, flags=0, **over):
+    P = dict(n_max=w.n_max, k=w.k, W=w.W, D=w.D, succ_len=w.succ_len,
+             tau=w.tau if tau is None else tau, flags=flags)
+    P.update(over)
+    return P
+
+
+def params(P):
+    return native.make_params(P["n_max"], P["k"], P["W"], P["D"], P["succ_len"], P["tau"],
+                              P["flags"])
+
+
+def run_step(w, P, next_topk=None):
+    tok, ln, reps, q = to_dev(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    nt = torch.from_numpy(next_topk).cuda() if next_topk is not None else None
+    eng.run(tok, ln, reps, q, next_topk=nt)
+    torch.cuda.synchronize()
+    assert native.read_device_status(eng.ws) == 0
+    return eng.out.to_host()
+
+
+def succ_extensions(g, b):
+    n = int(g["n_nodes"][b])
+    par = g["parents"][b, :n]
+    heads = [i for i in range(1, n) if par[i] == 0]
+    if g["hit_kind"][b] == oracle.LEX:
+        heads = [i for i in heads if i != 1]
+    return sum(1 for h in heads if (par == h).any())
+
+
+def check_all(w, g, P, next_topk=None, full_eps=True, seqs=None):
+    rep = parity.Report()
+    seqs = range(w.B) if seqs is None else seqs
+    for b in seqs:
+        parity.compare_sequence(b, w.tokens[b], int(w.lengths[b]), w.ld, w.reps[b], w.query[b],
+                                g, P, rep, None if next_topk is None else next_topk[b],
+                                full_eps)
+    hk = g["hit_kind"]
+    exp_stats = [int((hk == 1).sum()), int((hk == 2).sum()), int(w.B - (hk == 1).sum() - (hk == 2).sum()),
+                 sum(succ_extensions(g, b) for b in range(w.B))]
+    assert g["stats"].tolist() == exp_stats
+    print(rep)
+    return rep
+
+
+def bf16_rows(rows, d):
+    out = np.zeros((len(rows), d), np.float32)
+    for i, r in enumerate(rows):
+        out[i, : len(r)] = r
+    return synth.f32_to_bf16_bits(out)
+
+
+def single(tokens, R, q, n_max, k, W, D, succ_len=1, tau=0.1):
+    L, d = R.shape
+    return synth.Workload(0, 1, L, d, n_max, k, W, D, succ_len, tau,
+                          np.asarray(tokens, np.int32)[None], np.array([L], np.int32), R[None],
+                          q[None], np.array([], int))
+
+
+# ---------------------------------------------------------------- golden cases
+def test_worked_example_lexical():
+    g0 = load_golden("worked_example_lexical.txt")
+    M = [int(x) for x in g0["tokens"]]
+    L, d = len(M), 8
+    row = synth.f32_to_bf16_bits(np.random.default_rng(0).standard_normal(d).astype(np.float32))
+    R = np.tile(row, (L, 1))
+    w = single(M, R, R[L - 1], 2, 8, 2, 8)
+    g = run_step(w, P_of(w))
+    n = int(g["n_nodes"][0])
+    assert g["hit_kind"][0] == 1 and g["match_n"][0] == 2
+    assert g["cand"][0, : g["n_cand"][0]].tolist() == [int(x) for x in g0["cand"]]
+    assert g["draft_tokens"][0, :n].tolist() == [int(x) for x in g0["tree_tokens"]]
+    assert g["parents"][0, :n].tolist() == [int(x) for x in g0["tree_parents"]]
+    assert g["positions"][0, :n].tolist() == [int(x) for x in g0["tree_positions"]]
+    for i in range(n):
+        assert np.flatnonzero(g["mask"][0, i]).tolist() == [int(x) for x in g0[f"mask_row{i}"]]
+    check_all(w, g, P_of(w))
+
+
+def test_worked_example_semantic():
+    g0 = load_golden("worked_example_semantic.txt")
+    M = [int(x) for x in g0["tokens"]]
+    L = len(M)
+    R = bf16_rows([[float(x) for x in g0[f"row{i}"]] for i in range(L)], 8)
+    q = bf16_rows([[float(x) for x in g0["query"]]], 8)[0]
+    w = single(M, R, q, 3, 3, 2, 4)
+    g = run_step(w, P_of(w))
+    n = int(g["n_nodes"][0])
+    assert g["hit_kind"][0] == 2
+    assert g["cand"][0, :3].tolist() == [int(x) for x in g0["cand"]]
+    np.testing.assert_allclose(g["score"][0, :3], [float(x) for x in g0["score"]], atol=1e-6)
+    assert g["draft_tokens"][0, :n].tolist() == [int(x) for x in g0["tree_tokens"]]
+    assert g["parents"][0, :n].tolist() == [int(x) for x in g0["tree_parents"]]
+    assert g["positions"][0, :n].tolist() == [int(x) for x in g0["tree_positions"]]
+    assert g["stats"].tolist() == [0, 1, 0, 2]
+    check_all(w, g, P_of(w))
+
+
+# ------------------------------------------------------ seeded small workloads
+SMALL = [  # (cfg, B, L, d, seed)
+    (1, 1, 700, 64, 0), (1, 3, 2048, 256, 1), (2, 8, 1500, 128, 0), (2, 6, 3000, 520, 2),
+    (3, 6, 2500, 640, 0), (4, 24, 600, 96, 0), (4, 40, 300, 8, 3), (5, 4, 4000, 256, 0),
+]
+
+
+@pytest.mark.parametrize("cfg,B,L,d,seed", SMALL)
+def test_small_workloads(cfg, B, L, d, seed):
+    rng = np.random.default_rng(seed)
+    lengths = rng.integers(max(2, L // 3), L + 1, size=B).astype(np.int32)
+    lengths[0] = L
+    w = synth.make_workload(cfg, B=B, L=L, d=d, ld=L + 5, lengths=lengths, seed=seed)
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P), P)
+
+
+@pytest.mark.parametrize("d", [8, 136, 2048, 2056, 4096, 4104, 5120, 6144, 6152, 8192, 8200,
+                               12288, 12296, 16384])
+def test_every_dimension_variant(d):
+    L = 96 if d > 4096 else 300
+    w = synth.make_workload(3, B=4, L=L, d=d, nohit=0.75, seed=d)
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P), P)
+
+
+def test_rows_spread_over_all_ctas():
+    """Far more rows than CTAs: every CTA range straddles sequence boundaries."""
+    w = synth.make_workload(2, B=5, L=30011, d=64, nohit=1.0, seed=5,
+                            lengths=[30011, 17, 29000, 1, 12345])
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau, k=32)
+        check_all(w, run_step(w, P), P)
+
+
+def test_fewer_rows_than_ctas():
+    w = synth.make_workload(2, B=3, L=9, d=16, nohit=1.0, seed=6, lengths=[9, 4, 2])
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P), P)
+
+
+def test_exact_ties_break_to_recent():
+    """Identical rows give identical fp32 scores: order must be by position."""
+    L, d = 400, 64
+    M = np.arange(L, dtype=np.int32) % 97
+    M[-1] = 1000                              # no lexical hit
+    rng = np.random.default_rng(3)
+    R = synth.f32_to_bf16_bits(rng.standard_normal((L, d)).astype(np.float32))
+    R[5:: 7] = R[0]
+    q = R[0].copy()
+    w = single(M, R, q, 3, 32, 3, 6)
+    P = P_of(w, tau=NEG_INF)
+    g = run_step(w, P)
+    tied = sorted([j for j in range(L - 1) if (R[j] == R[0]).all()], reverse=True)[:32]
+    assert g["cand"][0].tolist() == tied
+    check_all(w, g, P)
+
+
+@pytest.mark.parametrize("lengths", [[0, 1, 2, 3, 50, 51], [1, 1, 1, 1, 1, 1], [2, 2, 3, 3, 4, 4]])
+@pytest.mark.parametrize("n_max,k,W", [(8, 1, 0), (1, 3, 3), (4, 32, 64)])
+def test_edge_lengths(lengths, n_max, k, W):
+    w = synth.make_workload(4, B=6, L=50, d=16, ld=50, seed=9, nohit=0.5,
+                            lengths=[min(x, 50) for x in lengths])
+    w.lengths = np.asarray(lengths, np.int32)   # 51 > ld: invalid on purpose
+    P = P_of(w, n_max=n_max, k=k, W=W, tau=NEG_INF)
+    check_all(w, run_step(w, P), P)
+
+
+@pytest.mark.parametrize("flags", [oracle.NO_LEX_RERANK, oracle.SUCC_ON_STRICT, oracle.NO_SEMANTIC,
+                                   oracle.NO_BRANCH, oracle.NO_SUCC,
+                                   oracle.NO_LEX_RERANK | oracle.NO_BRANCH | oracle.NO_SEMANTIC])
+def test_ablation_flags(flags):
+    w = synth.make_workload(2, B=12, L=2000, d=128, nohit=0.5, seed=11)
+    P = P_of(w, flags=flags)
+    check_all(w, run_step(w, P), P)
+
+
+@pytest.mark.parametrize("succ_len", [2, 5])
+def test_longer_successors(succ_len):
+    w = synth.make_workload(2, B=8, L=1200, d=64, nohit=0.75, seed=12)
+    P = P_of(w, succ_len=succ_len, flags=oracle.SUCC_ON_STRICT)
+    check_all(w, run_step(w, P), P)
+
+
+def test_next_token_table():
+    w = synth.make_workload(2, B=6, L=400, d=64, nohit=0.5, seed=13)
+    tk = synth.make_next_topk(w.tokens, w.lengths, 32000, 6)
+    P = P_of(w)
+    check_all(w, run_step(w, P, next_topk=tk), P, next_topk=tk)
+
+
+def test_standalone_entry_points():
+    """lexical -> semantic (selected sequences) -> tree, as three calls."""
+    w = synth.make_workload(2, B=10, L=900, d=128, nohit=0.5, seed=14)
+    P = P_of(w)
+    tok, ln, reps, q = to_dev(w)
+    p = params(P)
+    out = native.Outputs.allocate(w.B, p)
+    ws = native.allocate_workspace(w.B, w.ld, w.d, p)
+    native.lexical_match(tok, ln, w.n_max, w.k, out.hit_kind, out.match_n, out.cand, out.n_cand, ws)
+    torch.cuda.synchronize()
+    hk = out.hit_kind.cpu().numpy()
+    for b in range(w.B):
+        n, c = oracle.lexical(w.tokens[b], w.n_max, w.k)
+        assert hk[b] == (1 if n else 0)
+        assert out.cand[b, : out.n_cand[b]].tolist() == c
+    active = (out.hit_kind != 1).to(torch.uint8)
+    native.semantic_topk(reps, q, ln, w.k, w.tau, out.cand, out.score, out.n_cand, ws,
+                         active=active)
+    torch.cuda.synchronize()
+    nc = out.n_cand.cpu().numpy()
+    out.hit_kind.copy_(torch.where(out.hit_kind == 1, out.hit_kind,
+                                   torch.where(out.n_cand > 0, 2, 0).to(torch.int32)))
+    out.status.zero_()
+    out.stats.zero_()
+    native.build_draft_tree(tok, ln, reps, q, out.hit_kind, out.cand, out.score, out.n_cand, p,
+                            out, ws)
+    torch.cuda.synchronize()
+    g = out.to_host()
+    g["match_n"] = np.array([oracle.lexical(w.tokens[b], w.n_max, w.k)[0] for b in range(w.B)])
+    assert (nc[hk == 1] >= 1).all()
+    check_all(w, g, P)
+    # the fallback alone over every sequence, pure top-k
+    cand = torch.empty((w.B, w.k), dtype=torch.int32, device="cuda")
+    score = torch.empty((w.B, w.k), dtype=torch.float32, device="cuda")
+    n_c = torch.empty(w.B, dtype=torch.int32, device="cuda")
+    native.semantic_topk(reps, q, ln, w.k, NEG_INF, cand, score, n_c, ws)
+    torch.cuda.synchronize()
+    rep = parity.Report()
+    for b in range(w.B):
+        L = int(w.lengths[b])
+        s_all = oracle.scores_all(w.reps[b], w.query[b], L)
+        eps = parity.eps_rows(w.reps[b][: L - 1], w.query[b], w.d)
+        parity.check_semantic_list(cand[b].cpu().numpy(), score[b].cpu().numpy(), int(n_c[b]),
+                                   s_all, eps, w.k, NEG_INF, rep)
+
+
+def test_repeated_calls_reuse_workspace():
+    w = synth.make_workload(4, B=16, L=700, d=64, seed=15)
+    P = P_of(w)
+    tok, ln, reps, q = to_dev(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    eng.ws.fill_(0xA5)                      # garbage workspace: every call must reset it
+    first = None
+    for _ in range(3):
+        eng.run(tok, ln, reps, q)
+        torch.cuda.synchronize()
+        g = eng.out.to_host()
+        if first is None:
+            first = g
+        for key in first:
+            assert np.array_equal(first[key], g[key], equal_nan=True), key
+    check_all(w, first, P)
+
+
+# ----------------------------------------------------- full-size workloads
+@pytest.mark.parametrize("cfg", [1, 2, 3, 4, 5])
+def test_full_size_config(cfg):
+    """The five workload shapes at full size, launched as the benchmark does;
+    the oracle checks a sample of sequences (every forced miss up to 3, and
+    lexical hits), every sequence gets the lexical and structural checks."""
+    w = synth.make_workload(cfg, device="cuda")
+    P = P_of(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    eng.run(w.tokens, w.lengths, w.reps, w.query)
+    torch.cuda.synchronize()
+    assert native.read_device_status(eng.ws) == 0
+    g = eng.out.to_host()
+    tokens = w.tokens.cpu().numpy()
+    lengths = w.lengths.cpu().numpy()
+    for b in range(w.B):
+        n, c = oracle.lexical(tokens[b], w.n_max, w.k)
+        assert g["match_n"][b] == n
+        if n:
+            assert g["hit_kind"][b] == 1
+            assert sorted(g["cand"][b, : g["n_cand"][b]].tolist(), reverse=True) == c
+        else:
+            assert g["hit_kind"][b] in (0, 2)
+    forced = [int(b) for b in w.forced][:3]
+    others = [b for b in range(w.B) if b not in w.forced][:2]
+    sample = forced + others
+    host = {}
+    for b in sample:
+        host[b] = (w.reps[b].view(torch.int16).cpu().numpy().view(np.uint16),
+                   w.query[b].view(torch.int16).cpu().numpy().view(np.uint16))
+    hw = synth.Workload(cfg, w.B, w.ld, w.d, w.n_max, w.k, w.W, w.D, w.succ_len, w.tau,
+                        tokens, lengths, None, None, w.forced)
+    rep = parity.Report()
+
+    def one(b):
+        R, q = host[b]
+        parity.compare_sequence(b, tokens[b], int(lengths[b]), w.ld, R, q, g, P, rep,
+                                full_eps=False)
+
+    with ThreadPoolExecutor(max_workers=min(8, len(sample))) as ex:
+        list(ex.map(one, sample))
+    print(f"config {cfg}: sample {sample}: {rep}")
+    # planted near-duplicates are found for every forced miss
+    for b in forced:
+        assert g["hit_kind"][b] == 2
+        got = set(g["cand"][b, : g["n_cand"][b]].tolist())
+        assert set(w.planted[b][: w.k]) <= got or len(got) == w.k
+    del hw
