@@ -69,6 +69,8 @@ typedef struct CUstream_st *adapld_stream_t;
 #define ADAPLD_ERR_SUCC_LEN (-12)     /* succ_len outside [1, 16]              */
 #define ADAPLD_ERR_TOPK_TABLE (-13)   /* next_topk given with Kn < 1           */
 #define ADAPLD_ERR_TAU (-14)          /* tau is NaN                            */
+#define ADAPLD_ERR_STATIC_LIMIT (-15) /* B > ADAPLD_STATIC_MAX_B for the
+                                         workspace-free entry point           */
 #define ADAPLD_ERR_CUDA (-20)         /* a CUDA runtime call failed            */
 
 /* ---- retrieval outcome per sequence (Eq. 5, Algorithm 1) ------------------- */
@@ -275,6 +277,39 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                    const int32_t *next_topk, int32_t Kn, int32_t B, const adapld_params *p,
                    const adapld_step_out *out, void *ws, size_t ws_bytes,
                    const adapld_step_events *events, adapld_stream_t stream);
+
+/*
+ * adapld_semantic_topk_static(): adapld_semantic_topk() for callers that cannot
+ * provide any device memory beyond their inputs and outputs.  The paper has no
+ * counterpart; this exists for deployment.  Typical such callers are host
+ * libraries embedded in a serving process whose GPU memory is wholly owned by
+ * another allocator (a cudaMalloc there would escape that allocator's budget
+ * and implicitly synchronise the device), or integrations whose calling
+ * convention has no place for a workspace buffer.
+ *
+ * Arguments, results and errors are those of adapld_semantic_topk() without
+ * ws / ws_bytes.  The entry point allocates nothing: its scratch is one
+ * file-scope device array of ADAPLD_STATIC_SCRATCH_BYTES (1 MiB), which every
+ * GPU that loads the library reserves until the process exits.
+ *   - B may be at most ADAPLD_STATIC_MAX_B (1024); larger batches return
+ *     ADAPLD_ERR_STATIC_LIMIT without enqueuing anything.
+ *   - The first call on each device looks up the array's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture.
+ *   - All calls on a device share the one array and it keeps the previous
+ *     call's contents (each call clears what must start at zero), so calls
+ *     that overlap on the GPU -- on different streams, or from different host
+ *     threads -- race and must not be issued.  Serialise them.
+ *   - The device status word of this variant is internal (not readable with
+ *     adapld_read_device_status()).
+ */
+#define ADAPLD_STATIC_SCRATCH_BYTES (1u << 20)
+#define ADAPLD_STATIC_MAX_B 1024
+int adapld_semantic_topk_static(const uint16_t *reps, int64_t ld, int32_t d,
+                                const uint16_t *query, const int32_t *lengths,
+                                const uint8_t *active, int32_t B, int32_t k, float tau,
+                                int32_t *cand, float *score, int32_t *n_cand,
+                                adapld_stream_t stream);
 
 /* Synchronises `stream` and returns in *status the ADAPLD_DEV_* bits raised by
  * the most recent call that used workspace `ws` (0 = none). */

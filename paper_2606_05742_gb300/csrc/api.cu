@@ -89,6 +89,7 @@ const char *adapld_status_string(int code) {
         case ADAPLD_ERR_SUCC_LEN: return "succ_len must be in [1, 16]";
         case ADAPLD_ERR_TOPK_TABLE: return "next_topk needs Kn in [1, 64]";
         case ADAPLD_ERR_TAU: return "tau must not be NaN";
+        case ADAPLD_ERR_STATIC_LIMIT: return "B exceeds ADAPLD_STATIC_MAX_B (1024) for the workspace-free entry point";
         case ADAPLD_ERR_CUDA: return "a CUDA runtime call failed";
         default: return "unknown status";
     }

@@ -33,7 +33,10 @@ EXPORTED = [
     "adapld_tree_nodes", "adapld_workspace_bytes", "adapld_status_string",
     "adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
     "adapld_step", "adapld_step_ex", "adapld_read_device_status",
+    "adapld_semantic_topk_static",
 ]
+STATIC_MAX_B = 1024
+ERR_STATIC_LIMIT = -15
 
 
 class AdapldError(RuntimeError):
@@ -102,8 +105,11 @@ def load() -> ctypes.CDLL:
         lib.adapld_step.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P]
         lib.adapld_step_ex.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P, P]
         lib.adapld_read_device_status.argtypes = [P, P, P]
+        lib.adapld_semantic_topk_static.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P,
+                                                    P, P]
         for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
-                  "adapld_step", "adapld_step_ex", "adapld_read_device_status"):
+                  "adapld_step", "adapld_step_ex", "adapld_read_device_status",
+                  "adapld_semantic_topk_static"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -153,6 +159,18 @@ def semantic_topk(reps, query, lengths, k: int, tau: float, cand, score, n_cand,
                                      _ptr(n_cand), _ptr(ws), ws.numel() * ws.element_size(),
                                      _stream(stream))
     _check(rc, "adapld_semantic_topk")
+
+
+def semantic_topk_static(reps, query, lengths, k: int, tau: float, cand, score, n_cand,
+                         active=None, stream=None) -> None:
+    """adapld_semantic_topk_static: the semantic fallback for callers that
+    cannot supply a workspace (scratch in the library's own device array;
+    B <= 1024; calls must not overlap on the GPU)."""
+    B, ld, d = reps.shape
+    rc = load().adapld_semantic_topk_static(_ptr(reps), ld, d, _ptr(query), _ptr(lengths),
+                                            _ptr(active), B, k, tau, _ptr(cand), _ptr(score),
+                                            _ptr(n_cand), _stream(stream))
+    _check(rc, "adapld_semantic_topk_static")
 
 
 def _tree_out(anchor, draft_tokens, parents, positions, mask, n_nodes, stats=None) -> TreeOut:
