@@ -41,6 +41,8 @@ def parse():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--config", type=int, default=5)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--batch", type=int, default=None,
+                    help="override B (profiling of small cases; not the headline workload)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -237,7 +239,7 @@ def run_native(args):
             dist.barrier()
 
     cfg = args.config
-    w = synth.make_workload(cfg, device=str(dev), seed=args.seed + rank)
+    w = synth.make_workload(cfg, device=str(dev), seed=args.seed + rank, B=args.batch)
     p = native.make_params(w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, 0)
     eng = native.Engine(w.B, w.ld, w.d, p, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -252,14 +254,14 @@ def run_native(args):
     tokens = w.tokens.cpu().numpy()
     nbytes = algorithmic_bytes(w, g, lengths, tokens)
 
-    # timed region: K steps, CUDA events on the launching stream
+    # Timed region A (the headline): K steps back to back, CUDA events only at
+    # the two ends, so consecutive kernels keep their programmatic-launch
+    # overlap.  Timed region B: K more steps with events around each kernel,
+    # for the per-kernel durations (the roofline) and the stage breakdown.
     K = args.steps
-    ev_sem = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(K)]
-    ev_all = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in range(K)]
-    for pair in ev_all + ev_sem:        # torch creates CUDA events lazily, on first record
-        for e in pair:
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(K)]
+    for row in ev:                       # torch creates CUDA events lazily, on first record
+        for e in row:
             e.record(stream)
     clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
     start = torch.cuda.Event(enable_timing=True)
@@ -271,21 +273,27 @@ def run_native(args):
         time.sleep(0.3)
     start.record(stream)
     for i in range(K):
-        # lexical_begin/lexical_end slots carry the per-step bracket, the
-        # semantic pair brackets the semantic kernel alone
-        native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws,
-                    events=native.StepEvents(ev_all[i][0].cuda_event, None,
-                                             ev_sem[i][0].cuda_event, ev_sem[i][1].cuda_event,
-                                             None, ev_all[i][1].cuda_event))
+        native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws)
     end.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
-    clk = clocks.stop() if clocks else None
     total_ms = start.elapsed_time(end)
+    startb = torch.cuda.Event(enable_timing=True)
+    endb = torch.cuda.Event(enable_timing=True)
+    startb.record(stream)
+    for i in range(K):
+        native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws,
+                    events=native.StepEvents(*[e.cuda_event for e in ev[i]]))
+    endb.record(stream)
+    torch.cuda.synchronize(dev)
+    barrier()
+    clk = clocks.stop() if clocks else None
+    total_b_ms = startb.elapsed_time(endb)
     if native.read_device_status(eng.ws) != 0:
         raise RuntimeError("device status raised during the timed region")
-    sem_ms = [a.elapsed_time(b) for a, b in ev_sem]
-    step_ms = [a.elapsed_time(b) for a, b in ev_all]
+    stage = {name: [r[2 * i].elapsed_time(r[2 * i + 1]) for r in ev]
+             for i, name in enumerate(("lexical", "semantic", "tree"))}
+    sem_ms = stage["semantic"]
     t = torch.tensor([total_ms], device=dev)
     if world > 1:
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -341,6 +349,9 @@ def run_native(args):
         cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample.desc}
     hk = g["hit_kind"]
     conf = workload_config(cfg)
+    if args.batch is not None:
+        conf["workload"] += f" (resized: B={w.B})"
+        conf["B"] = conf["global_batch"] = w.B
     conf.update({"parallelism": f"replicas x{world} (batch per GPU)",
                  "outcomes": {"lexical": int((hk == 1).sum()), "semantic": int((hk == 2).sum()),
                               "none": int((hk == 0).sum())},
@@ -355,11 +366,12 @@ def run_native(args):
                      "unit": "GB/s", "frac": achieved / peak, "traffic": None,
                      "algorithmic_bytes": nbytes["semantic"], "avg_launch_ms": sem_avg_ms},
         "step_hbm": {"achieved": step_gbs, "frac": step_gbs / peak,
-                     "algorithmic_bytes": nbytes["step"],
-                     "median_step_ms": statistics.median(step_ms)},
+                     "algorithmic_bytes": nbytes["step"]},
+        "stage_ms": {name: sum(v) / len(v) for name, v in stage.items()},
+        "ms_per_step_with_stage_events": total_b_ms / K,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 3 * K,
+        "gpu_launches": 4 * K,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

@@ -32,11 +32,17 @@ struct Workspace {
     int32_t *global_ticket;  // [1]  lexical kernel: CTAs done with their sequence
     int32_t *ticket1;        // [B]  lexical kernel: chunks done per sequence
     int32_t *done2;          // [B]  semantic kernel: CTAs done per sequence
-    int32_t *ticket4;        // [B]  tree kernel: slices done per sequence
+    int32_t *ticket4;        // [B]  successor scan: slices done per sequence
+    int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
     int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
     int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
     int32_t *slots2;         // [B + kMaxGrid2][kSlotInts] partial top-k lists
     int32_t *part4;          // [B][S4][W][kPart4Ints] per-slice successor lists
+    int32_t *succ;           // [B][W][kMaxK] merged successor candidates
+    int32_t *succ_n;         // [B][W] their counts
+    int32_t *rr_cand;        // [B][kMaxK] reranked lexical candidates (successor scan)
+    float *rr_score;         // [B][kMaxK] their scores
+    float *score5;           // [B][W*kMaxK] scores computed by the tree kernel
     size_t counters_bytes;
     size_t total_bytes;
     int C1, S4, W;
@@ -61,24 +67,39 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         off = align_up(off + bytes, 256);
         return r;
     };
-    w.dev_status = (int32_t *)take(sizeof(int32_t) * (2 + 3 * (size_t)B));
+    w.dev_status = (int32_t *)take(sizeof(int32_t) * (2 + 4 * (size_t)B));
     if (p) {
         w.global_ticket = w.dev_status + 1;
         w.ticket1 = w.dev_status + 2;
         w.done2 = w.ticket1 + B;
         w.ticket4 = w.done2 + B;
+        w.ticket5 = w.ticket4 + B;
     }
-    w.counters_bytes = sizeof(int32_t) * (2 + 3 * (size_t)B);
+    w.counters_bytes = sizeof(int32_t) * (2 + 4 * (size_t)B);
     w.part1 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1 * kPart1Ints);
     w.plan = (int64_t *)take(sizeof(int64_t) * ((size_t)B + 1));
     w.slots2 = (int32_t *)take(sizeof(int32_t) * ((size_t)B + kMaxGrid2) * kSlotInts);
     w.part4 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.S4 * w.W * kPart4Ints);
+    w.succ = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.W * kMaxK);
+    w.succ_n = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.W);
+    w.rr_cand = (int32_t *)take(sizeof(int32_t) * (size_t)B * kMaxK);
+    w.rr_score = (float *)take(sizeof(float) * (size_t)B * kMaxK);
+    w.score5 = (float *)take(sizeof(float) * (size_t)B * w.W * kMaxK);
     w.total_bytes = off;
     return w;
 }
 
 // ---- device helpers ------------------------------------------------------------
 #ifdef __CUDACC__
+
+// Programmatic dependent launch: wait until the previous kernel in the stream
+// has completed and its writes are visible (a no-op when this kernel was not
+// launched as a dependent), then allow the next kernel to begin launching.
+// Calling the two in this order keeps completion transitive along the chain.
+__device__ __forceinline__ void pdl_wait_then_release() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 __device__ __forceinline__ uint64_t global_ns() {
     uint64_t t;
@@ -222,6 +243,44 @@ struct WarpTopK {
     }
 };
 
+// Concatenates per-part lists, highest part first, into out[0..k) with one
+// warp: count_of(p) gives part p's list length, entry_of(p, i) its i-th
+// entry.  Every lane loads one part's count and fills one output slot per
+// group of 32 parts, so the merge costs a few memory round trips, not one per
+// part.  All 32 lanes must call; returns the number written (<= k).
+template <class CountF, class EntryF>
+__device__ __forceinline__ int warp_merge_desc(int nparts, int k, CountF count_of, EntryF entry_of,
+                                               int32_t *out) {
+    const int lane = threadIdx.x & 31;
+    int total = 0;
+    for (int base = 0; base < nparts && total < k; base += 32) {
+        const int part = nparts - 1 - (base + lane);
+        const int n = base + lane < nparts ? count_of(part) : 0;
+        int incl = n;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += u;
+        }
+        const int excl = incl - n;
+        const int group = __shfl_sync(0xffffffffu, incl, 31);
+        // output slot `lane` of this group comes from the last part whose
+        // range starts at or before it
+        int src = 0;
+#pragma unroll
+        for (int m = 0; m < 32; ++m) {
+            const int e = __shfl_sync(0xffffffffu, excl, m);
+            const int nn = __shfl_sync(0xffffffffu, n, m);
+            if (nn > 0 && e <= lane) src = m;
+        }
+        const int e_src = __shfl_sync(0xffffffffu, excl, src);
+        if (lane < group && total + lane < k)
+            out[total + lane] = entry_of(nparts - 1 - (base + src), lane - e_src);
+        total = min(k, total + group);
+    }
+    return total;
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -237,6 +296,25 @@ __device__ __forceinline__ int warp_max_i(int v) {
 #endif  // __CUDACC__
 
 // ---- host-side launchers (one per kernel) ---------------------------------------
+// Launches `kern` as a programmatic dependent of the previous kernel in the
+// stream (it must call pdl_wait_then_release before reading that kernel's
+// outputs).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_dependent(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                             cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 struct LexLaunch {
     const int32_t *tokens;
     int64_t ld;

@@ -87,6 +87,7 @@ __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
     __shared__ int list[kMaxK];
     __shared__ int flag;
 
+    pdl_wait_then_release();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int b = blockIdx.y, c = blockIdx.x;
     const int len = a.lengths[b];
@@ -167,21 +168,21 @@ __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
 
     // ---- last chunk of sequence b: merge ------------------------------------
     if (warp == 0) {
+        const int nchunks = (int)gridDim.x;
+        const int32_t *pb = ws.part1 + (int64_t)b * ws.C1 * kPart1Ints;
         int best = 0;
-        for (int cc = lane; cc < (int)gridDim.x; cc += 32)
-            best = max(best, __ldcg(ws.part1 + ((int64_t)b * ws.C1 + cc) * kPart1Ints));
+        for (int cc = lane; cc < nchunks; cc += 32) best = max(best, __ldcg(pb + cc * kPart1Ints));
         best = warp_max_i(best);
-        int total = 0;
         int32_t *cb = a.cand + (int64_t)b * a.k;
+        int total = 0;
         if (best > 0) {
-            for (int cc = (int)gridDim.x - 1; cc >= 0 && total < a.k; --cc) {
-                const int32_t *pp = ws.part1 + ((int64_t)b * ws.C1 + cc) * kPart1Ints;
-                if (__ldcg(pp) != best) continue;
-                const int n = __ldcg(pp + 1);
-                const int take = min(n, a.k - total);
-                if (lane < take) cb[total + lane] = __ldcg(pp + 2 + lane);
-                total += take;
-            }
+            total = warp_merge_desc(
+                nchunks, a.k,
+                [&](int cc) {
+                    const int32_t *pp = pb + cc * kPart1Ints;
+                    return __ldcg(pp) == best ? __ldcg(pp + 1) : 0;
+                },
+                [&](int cc, int i) { return __ldcg(pb + cc * kPart1Ints + 2 + i); }, cb);
         }
         if (lane >= total && lane < a.k) cb[lane] = -1;
         if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;

@@ -25,13 +25,15 @@
 //  * Every mbarrier wait is bounded; on expiry the CTA raises
 //    ADAPLD_DEV_TIMEOUT, stops issuing copies, drains the copies in flight and
 //    exits without publishing.
+#include <cstdio>
+#include <cstdlib>
+
 #include "common.cuh"
 
 namespace adapld {
 
 namespace {
 
-constexpr int kRingBytes = 192 * 1024;
 constexpr int kProducerWarp = kConsumers2 / 32;  // warp 8
 constexpr int kBarQ = 15;                        // named barrier for |q|^2
 
@@ -89,20 +91,53 @@ __device__ __forceinline__ int seq_of(const int64_t *plan, int B, int64_t g) {
     return lo;
 }
 
+// Two fp32 values in one 64-bit register, for the packed f32x2 FMA.
+__device__ __forceinline__ uint64_t bf16x2_to_f32x2(uint32_t w) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(w << 16), "r"(w & 0xffff0000u));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+
+__device__ __forceinline__ float sum_f32x2(uint64_t v) {
+    float lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+    return lo + hi;
+}
+
+// c += a * b on both halves (two fp32 FMAs, round to nearest).
+__device__ __forceinline__ void fma2(uint64_t &c, uint64_t a, uint64_t b) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(c) : "l"(a), "l"(b));
+}
+
+// Variants whose per-thread state (query slice plus one stage of loads) is
+// large get the register budget of one CTA per SM.
 template <int MAXC, int SR>
-__global__ void __launch_bounds__(kConsumers2 + 32, 1) semantic_kernel(SemArgs args) {
+constexpr int semantic_min_blocks() {
+    return MAXC * (SR * 4 + 8) > 72 ? 1 : 2;
+}
+
+template <int MAXC, int SR>
+__global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, SR>()))
+    semantic_kernel(SemArgs args) {
     const SemLaunch &a = args.p;
     const Workspace &ws = args.ws;
     extern __shared__ __align__(128) uint8_t smem[];
     const int NS = args.nstages;
     const int stage_bytes = args.stage_bytes;
     uint8_t *ring = smem;
-    float *red = (float *)(smem + (size_t)NS * stage_bytes);  // [kMaxStages2][32][8]
-    float *qred = red + kMaxStages2 * 32 * 8;                  // [2][8]
-    uint64_t *full = (uint64_t *)(qred + 16);                  // [kMaxStages2]
-    uint64_t *empty = full + kMaxStages2;                      // [kMaxStages2]
+    float *red = (float *)(smem + (size_t)NS * stage_bytes);  // [NS][32][8]
+    float *qred = red + NS * 32 * 8;                           // [2][8]
+    uint64_t *full = (uint64_t *)(qred + 16);                  // [NS]
+    uint64_t *empty = full + kMaxStages2;                      // [NS]
     volatile int *abort_flag = (volatile int *)(empty + kMaxStages2);
 
+    pdl_wait_then_release();  // the plan and the lexical outcomes come from the previous kernel
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int grid = gridDim.x, c = blockIdx.x;
     const int B = a.B, d = a.d, k = a.k;
@@ -175,7 +210,11 @@ __global__ void __launch_bounds__(kConsumers2 + 32, 1) semantic_kernel(SemArgs a
     }
 
     // ------------------------------------------------------------ consumers
-    float qf[MAXC][8];
+    // column slice of this thread: 16-byte chunks t + 256*cc, cc < MAXC
+    bool colok[MAXC];
+#pragma unroll
+    for (int cc = 0; cc < MAXC; ++cc) colok[cc] = (t + kConsumers2 * cc) * 8 < d;
+    uint64_t q2[MAXC][4];
     WarpTopK tk;
     tk.reset();
     bool aborted = false;
@@ -190,27 +229,20 @@ __global__ void __launch_bounds__(kConsumers2 + 32, 1) semantic_kernel(SemArgs a
         const int jbeg = (int)(g - plan[b]);
         const int jend = (int)(seg_end - plan[b]);
 
-        // query slice of this sequence and |q|^2
+        // query slice of this sequence (registers) and |q|^2
         float qpart = 0.f;
         const uint16_t *q = a.query + (int64_t)b * d;
 #pragma unroll
         for (int cc = 0; cc < MAXC; ++cc) {
-            const int col8 = t + kConsumers2 * cc;
-            if (col8 * 8 < d) {
-                const uint4 w = ldg_nc_v4(q + col8 * 8);
-                qf[cc][0] = bf16lo(w.x);
-                qf[cc][1] = bf16hi(w.x);
-                qf[cc][2] = bf16lo(w.y);
-                qf[cc][3] = bf16hi(w.y);
-                qf[cc][4] = bf16lo(w.z);
-                qf[cc][5] = bf16hi(w.z);
-                qf[cc][6] = bf16lo(w.w);
-                qf[cc][7] = bf16hi(w.w);
+            const uint4 w = colok[cc] ? ldg_nc_v4(q + (t + kConsumers2 * cc) * 8)
+                                      : make_uint4(0, 0, 0, 0);
+            const uint32_t ws4[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-                for (int e = 0; e < 8; ++e) qpart = fmaf(qf[cc][e], qf[cc][e], qpart);
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) qf[cc][e] = 0.f;
+            for (int e = 0; e < 4; ++e) {
+                const float lo = bf16lo(ws4[e]), hi = bf16hi(ws4[e]);
+                q2[cc][e] = f32x2(lo, hi);
+                qpart = fmaf(lo, lo, qpart);
+                qpart = fmaf(hi, hi, qpart);
             }
         }
         qpart = warp_sum(qpart);
@@ -230,47 +262,33 @@ __global__ void __launch_bounds__(kConsumers2 + 32, 1) semantic_kernel(SemArgs a
                 *abort_flag = 1;
                 atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
             }
-            if (*abort_flag) aborted = true;
-
+            // all shared loads of this stage first, then the packed FMAs
+            const uint8_t *st = ring + (size_t)s * stage_bytes + (size_t)t * 16;
+            uint4 wv[SR][MAXC];
+#pragma unroll
+            for (int r = 0; r < SR; ++r)
+#pragma unroll
+                for (int cc = 0; cc < MAXC; ++cc)
+                    wv[r][cc] = (r < nrows && colok[cc])
+                                    ? *(const uint4 *)(st + (size_t)r * row_bytes +
+                                                       (size_t)cc * kConsumers2 * 16)
+                                    : make_uint4(0, 0, 0, 0);
             float acc[2 * SR];
 #pragma unroll
-            for (int i = 0; i < 2 * SR; ++i) acc[i] = 0.f;
-            const uint8_t *st = ring + (size_t)s * stage_bytes;
-#pragma unroll
             for (int r = 0; r < SR; ++r) {
-                if (r < nrows) {
+                uint64_t dacc[2] = {0ull, 0ull}, sacc[2] = {0ull, 0ull};
 #pragma unroll
-                    for (int cc = 0; cc < MAXC; ++cc) {
-                        const int col8 = t + kConsumers2 * cc;
-                        if (col8 * 8 < d) {
-                            const uint4 w =
-                                *(const uint4 *)(st + (size_t)r * row_bytes + (size_t)col8 * 16);
-                            const float x0 = bf16lo(w.x), x1 = bf16hi(w.x);
-                            const float x2 = bf16lo(w.y), x3 = bf16hi(w.y);
-                            const float x4 = bf16lo(w.z), x5 = bf16hi(w.z);
-                            const float x6 = bf16lo(w.w), x7 = bf16hi(w.w);
-                            float dt = acc[2 * r], ss = acc[2 * r + 1];
-                            dt = fmaf(x0, qf[cc][0], dt);
-                            dt = fmaf(x1, qf[cc][1], dt);
-                            dt = fmaf(x2, qf[cc][2], dt);
-                            dt = fmaf(x3, qf[cc][3], dt);
-                            dt = fmaf(x4, qf[cc][4], dt);
-                            dt = fmaf(x5, qf[cc][5], dt);
-                            dt = fmaf(x6, qf[cc][6], dt);
-                            dt = fmaf(x7, qf[cc][7], dt);
-                            ss = fmaf(x0, x0, ss);
-                            ss = fmaf(x1, x1, ss);
-                            ss = fmaf(x2, x2, ss);
-                            ss = fmaf(x3, x3, ss);
-                            ss = fmaf(x4, x4, ss);
-                            ss = fmaf(x5, x5, ss);
-                            ss = fmaf(x6, x6, ss);
-                            ss = fmaf(x7, x7, ss);
-                            acc[2 * r] = dt;
-                            acc[2 * r + 1] = ss;
-                        }
+                for (int cc = 0; cc < MAXC; ++cc) {
+                    const uint32_t w4[4] = {wv[r][cc].x, wv[r][cc].y, wv[r][cc].z, wv[r][cc].w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const uint64_t x = bf16x2_to_f32x2(w4[e]);
+                        fma2(dacc[e & 1], x, q2[cc][e]);
+                        fma2(sacc[e & 1], x, x);
                     }
                 }
+                acc[2 * r] = sum_f32x2(dacc[0]) + sum_f32x2(dacc[1]);
+                acc[2 * r + 1] = sum_f32x2(sacc[0]) + sum_f32x2(sacc[1]);
             }
             ReduceScatter<2 * SR, 16>::run(acc, lane);
             constexpr int GRP = 32 / (2 * SR);
@@ -299,7 +317,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, 1) semantic_kernel(SemArgs a
         }
 
         // ---- end of this CTA's segment of sequence b: publish, maybe merge
-        if (warp == 0 && !aborted) {
+        if (warp == 0 && !aborted && !*abort_flag) {
             const int slot = b + c;
             int32_t *sp = ws.slots2 + (int64_t)slot * kSlotInts;
             if (lane == 0) sp[0] = tk.n;
@@ -350,31 +368,72 @@ __global__ void __launch_bounds__(kConsumers2 + 32, 1) semantic_kernel(SemArgs a
     }
 }
 
+// Shared memory per CTA: the ring, the per-stage reduction buffers, |q|^2
+// partials, the barriers and the abort flag.
+inline size_t semantic_smem(int ns, int stage) {
+    return (size_t)ns * stage + (size_t)ns * 32 * 8 * 4 + 16 * 4 + 2 * kMaxStages2 * 8 + 16;
+}
+
 template <int MAXC, int SR>
-cudaError_t launch_variant(const SemArgs &args0, int grid, cudaStream_t s) {
+cudaError_t launch_variant(const SemArgs &args0, int sms, int ctas_per_sm, cudaStream_t s) {
     SemArgs args = args0;
+    auto kern = semantic_kernel<MAXC, SR>;
     const int stage = (int)align_up((size_t)SR * args.p.d * 2, 128);
-    int ns = kRingBytes / stage;
-    ns = ns > kMaxStages2 ? kMaxStages2 : (ns < 2 ? 2 : ns);
+    // shared memory budget per CTA for the requested CTAs per SM
+    const size_t per_sm = 227 * 1024;
+    int cps = ctas_per_sm < 1 ? 1 : ctas_per_sm;
+    int ns = 0;
+    for (; cps >= 1; --cps) {
+        const size_t budget = (per_sm - (size_t)(cps - 1) * 1024) / cps;
+        ns = 0;
+        while (ns < kMaxStages2 && semantic_smem(ns + 1, stage) <= budget) ++ns;
+        if (ns >= 2) break;
+    }
+    if (cps < 1 || ns < 2) return cudaErrorInvalidConfiguration;
     args.nstages = ns;
     args.stage_bytes = stage;
-    const size_t smem = (size_t)ns * stage + kMaxStages2 * 32 * 8 * 4 + 16 * 4 +
-                        2 * kMaxStages2 * 8 + 16;
-    auto kern = semantic_kernel<MAXC, SR>;
+    const size_t smem = semantic_smem(ns, stage);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kConsumers2 + 32, smem, s>>>(args);
-    return cudaGetLastError();
+    int fit = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&fit, kern, kConsumers2 + 32, smem);
+    if (e != cudaSuccess) return e;
+    if (fit < 1) return cudaErrorInvalidConfiguration;
+    if (cps > fit) cps = fit;
+    int grid = sms * cps;
+    if (grid > kMaxGrid2) grid = kMaxGrid2;
+    return launch_dependent(kern, dim3(grid), dim3(kConsumers2 + 32), smem, s, args);
+}
+
+// Launch shape: CTAs per SM and rows per stage.  The defaults per dimension
+// range come from a sweep on GB300 (more resident consumer warps hide the
+// shared-load and FMA latencies; the ring per SM stays ~192 KB):
+//   d <= 4096: 3 CTAs/SM x 4 rows, d <= 6144: 2 x 4, d <= 8192: 3 x 2.
+// ADAPLD_SEMANTIC_TUNING="<ctas_per_sm>,<rows_per_stage>" overrides them, for
+// tuning sweeps (0 keeps the default).
+struct SemTuning {
+    int ctas_per_sm = 0;
+    int rows = 0;
+};
+
+SemTuning semantic_tuning() {
+    SemTuning t;
+    if (const char *e = std::getenv("ADAPLD_SEMANTIC_TUNING")) {
+        int a = 0, b = 0;
+        if (std::sscanf(e, "%d,%d", &a, &b) >= 1 && a >= 1 && a <= 4) t.ctas_per_sm = a;
+        if (b == 1 || b == 2 || b == 4 || b == 8 || b == 16) t.rows = b;
+    }
+    return t;
 }
 
 }  // namespace
 
-int semantic_grid() {
+int semantic_sms() {
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    return sms < kMaxGrid2 ? sms : kMaxGrid2;
+    return sms;
 }
 
 cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_t s) {
@@ -383,16 +442,39 @@ cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_
                                     a.n_cand, ws, s);
         if (e != cudaSuccess) return e;
     }
-    const int grid = semantic_grid();
-    if (grid <= 0) return cudaErrorInvalidDevice;
+    const int sms = semantic_sms();
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    const SemTuning tun = semantic_tuning();
     SemArgs args{a, ws, 0, 0};
-    const int d = a.d;
-    if (d <= 2048) return launch_variant<1, 16>(args, grid, s);
-    if (d <= 4096) return launch_variant<2, 4>(args, grid, s);
-    if (d <= 6144) return launch_variant<3, 4>(args, grid, s);
-    if (d <= 8192) return launch_variant<4, 2>(args, grid, s);
-    if (d <= 12288) return launch_variant<6, 2>(args, grid, s);
-    return launch_variant<8, 1>(args, grid, s);
+    const int d = a.d, R = tun.rows;
+#define ADAPLD_SEM(MAXC, SR, CPS) \
+    return launch_variant<MAXC, SR>(args, sms, tun.ctas_per_sm ? tun.ctas_per_sm : CPS, s)
+    if (d <= 2048) {
+        if (R == 4) ADAPLD_SEM(1, 4, 3);
+        if (R == 8) ADAPLD_SEM(1, 8, 3);
+        ADAPLD_SEM(1, 16, 3);
+    }
+    if (d <= 4096) {
+        if (R == 2) ADAPLD_SEM(2, 2, 3);
+        if (R == 8) ADAPLD_SEM(2, 8, 3);
+        ADAPLD_SEM(2, 4, 3);
+    }
+    if (d <= 6144) {
+        if (R == 2) ADAPLD_SEM(3, 2, 2);
+        ADAPLD_SEM(3, 4, 2);
+    }
+    if (d <= 8192) {
+        if (R == 1) ADAPLD_SEM(4, 1, 3);
+        if (R == 4) ADAPLD_SEM(4, 4, 3);
+        ADAPLD_SEM(4, 2, 3);
+    }
+    if (d <= 12288) {
+        if (R == 2) ADAPLD_SEM(6, 2, 2);
+        ADAPLD_SEM(6, 1, 2);
+    }
+    if (R == 2) ADAPLD_SEM(8, 2, 2);
+    ADAPLD_SEM(8, 1, 2);
+#undef ADAPLD_SEM
 }
 
 }  // namespace adapld

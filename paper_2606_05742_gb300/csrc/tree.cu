@@ -1,49 +1,90 @@
-// Rerank and draft-tree construction (Sec. 3.4-3.6, Eq. 6-15, Algorithm 1).
+// Rerank and draft-tree construction (Sec. 3.4-3.6, Eq. 6-15, Algorithm 1),
+// as two kernels so that every gathered representation row is read by its
+// own warp somewhere on the GPU instead of queueing behind one CTA.
 //
-// Grid (S4 slices, B sequences), 512 threads.
-//  1. Every participating CTA of a sequence rebuilds the anchor and branch set:
-//     lexical hits are reranked by Eq. 6 (one warp per candidate row, the
-//     query in shared memory as fp32), semantic hits keep their Eq. 4 order;
-//     j* = the first candidate; branch tokens come from the caller's cached
-//     next-token table row at j* or, without one, are the first W distinct
-//     continuation tokens of the ranked candidates; Eq. 11 removes the main
-//     path's first token on a lexical hit.
-//  2. When successor drafting applies (Algorithm 1: semantic hits; or every
-//     hit under ADAPLD_SUCC_ON_STRICT) the token history is cut into slices
-//     of 8192 positions, one CTA each; a warp per branch token scans its slice
-//     backwards with ballots and keeps the k most recent occurrences.  The
-//     last slice CTA (atomic ticket) merges them, scores every occurrence t by
-//     cos(R[t], R[j*+1]) (Eq. 13) and keeps the argmax (Eq. 14).
-//  3. The finishing CTA lays out the tree (root, main chain, branch paths with
-//     their successors) and writes tokens, parents, position ids and the
-//     ancestor mask.  Without successor drafting only slice 0 does any work.
+// succ_scan_kernel, grid (S4 slices, B), 512 threads -- only for sequences
+// that draft successors (Algorithm 1: semantic hits; every hit under
+// ADAPLD_SUCC_ON_STRICT).  Each CTA rebuilds the anchor and the branch set
+// (lexical hits are reranked here in that mode), then scans its slice of
+// 8192 positions for the branch tokens, a warp per branch, backwards with
+// ballots, keeping the k most recent occurrences.  The last slice CTA
+// (atomic ticket) merges the slices, most recent first, into the successor
+// candidate lists.
+//
+// tree_kernel, grid (R5, B), 512 threads.  Every sequence has a list of rows
+// to score: the lexical candidates against the query (Eq. 6), or every
+// successor candidate against R[j*+1] (Eq. 13).  CTA r scores rows
+// [16r, 16r+16), one warp per row, both operands streamed from global memory
+// with eight 16-byte loads per lane in flight.  The last CTA of the sequence
+// then ranks the lexical candidates (Eq. 7), picks each branch's successor
+// (Eq. 14), lays out the tree (root, main chain, branch paths with their
+// successors) and writes tokens, parents, position ids and the ancestor mask.
 #include "common.cuh"
 
 namespace adapld {
 
 namespace {
 
+constexpr int kRowsPerCta5 = kThreads4 / 32;  // one warp per scored row
+
 struct TreeArgs {
     TreeLaunch p;
     Workspace ws;
+    int rows_ctas;  // gridDim.x of tree_kernel
 };
 
-// <row, ref> and |row|^2 of one bf16 row against an fp32 vector in shared
-// memory; one warp, 8 independent 16-byte loads per lane in flight.
+// cos(row, ref) of two bf16 rows in global memory (one warp).  The norm of
+// ref is recomputed by every warp in the same order, so it is bit-identical.
+__device__ __forceinline__ float warp_cosine(const uint16_t *row, const uint16_t *ref, int d) {
+    const int lane = threadIdx.x & 31;
+    const int nch = d >> 3;
+    float dot = 0.f, sx = 0.f, sy = 0.f;
+    for (int base = 0; base < nch; base += 32 * 8) {
+        uint4 wx[8], wy[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int ch = base + u * 32 + lane;
+            wx[u] = ch < nch ? ldg_nc_v4(row + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
+            wy[u] = ch < nch ? ldg_nc_v4(ref + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const uint32_t xs[4] = {wx[u].x, wx[u].y, wx[u].z, wx[u].w};
+            const uint32_t ys[4] = {wy[u].x, wy[u].y, wy[u].z, wy[u].w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float x0 = bf16lo(xs[e]), x1 = bf16hi(xs[e]);
+                const float y0 = bf16lo(ys[e]), y1 = bf16hi(ys[e]);
+                dot = fmaf(x0, y0, dot);
+                dot = fmaf(x1, y1, dot);
+                sx = fmaf(x0, x0, sx);
+                sx = fmaf(x1, x1, sx);
+                sy = fmaf(y0, y0, sy);
+                sy = fmaf(y1, y1, sy);
+            }
+        }
+    }
+    return cosine_from(warp_sum(dot), warp_sum(sx), warp_sum(sy));
+}
+
+// <row, ref> and |row|^2 of one bf16 row in global memory against an fp32
+// vector in shared memory (one warp, 16 independent 16-byte loads per lane
+// in flight).
 __device__ __forceinline__ void warp_row_dot(const uint16_t *row, const float *ref, int d,
                                              float &dot_out, float &ss_out) {
+    constexpr int U = 16;
     const int lane = threadIdx.x & 31;
     const int nch = d >> 3;
     float dot = 0.f, ss = 0.f;
-    for (int base = 0; base < nch; base += 32 * 8) {
-        uint4 w[8];
+    for (int base = 0; base < nch; base += 32 * U) {
+        uint4 w[U];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < U; ++u) {
             const int ch = base + u * 32 + lane;
             w[u] = ch < nch ? ldg_nc_v4(row + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
+        for (int u = 0; u < U; ++u) {
             const int ch = base + u * 32 + lane;
             if (ch < nch) {
                 const float4 r0 = *(const float4 *)(ref + ch * 8);
@@ -82,8 +123,8 @@ __device__ float block_load_vec(const uint16_t *v, float *dst, int d, float *scr
     float part = 0.f;
     for (int ch = threadIdx.x; ch < (d >> 3); ch += blockDim.x) {
         const uint4 w = ldg_nc_v4(v + (size_t)ch * 8);
-        float x[8] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y),
-                      bf16lo(w.z), bf16hi(w.z), bf16lo(w.w), bf16hi(w.w)};
+        const float x[8] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y),
+                            bf16lo(w.z), bf16hi(w.z), bf16lo(w.w), bf16hi(w.w)};
 #pragma unroll
         for (int e = 0; e < 8; ++e) {
             dst[ch * 8 + e] = x[e];
@@ -99,179 +140,300 @@ __device__ float block_load_vec(const uint16_t *v, float *dst, int d, float *scr
     return tot;
 }
 
-__global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
+// Per-sequence facts every kernel of the tree stage derives the same way.
+struct SeqView {
+    int len;
+    bool valid, cand_ok, lex, sem, branch_on, need_succ;
+    int nc;
+};
+
+// Block-wide (every thread must call, before any early exit).
+__device__ __forceinline__ SeqView view_of(const TreeLaunch &a, int b) {
+    SeqView v;
+    const int k = a.p.k, W = a.p.branch_width, t = threadIdx.x;
+    const uint32_t flags = a.p.flags;
+    v.len = a.lengths[b];
+    v.valid = v.len >= 1 && (int64_t)v.len <= a.ld;
+    // candidates come from the caller on the standalone path: check the range
+    const int nc0 = v.valid ? min(a.n_cand[b], k) : 0;
+    bool ok = true;
+    if (t < nc0) {
+        const int c = a.cand[(int64_t)b * k + t];
+        ok = c >= 0 && c <= v.len - 2;
+    }
+    v.cand_ok = __syncthreads_and(ok) != 0;
+    const int hk = (v.valid && v.cand_ok) ? a.hit_kind[b] : ADAPLD_HIT_NONE;
+    v.nc = v.cand_ok ? max(nc0, 0) : 0;
+    v.lex = hk == ADAPLD_HIT_LEX && v.nc > 0;
+    v.sem = hk == ADAPLD_HIT_SEM && v.nc > 0;
+    v.branch_on = !(flags & ADAPLD_NO_BRANCH) && W > 0 && (v.lex || v.sem);
+    v.need_succ = v.branch_on && !(flags & ADAPLD_NO_SUCC) &&
+                  (v.sem || (v.lex && (flags & ADAPLD_SUCC_ON_STRICT)));
+    return v;
+}
+
+// Branch set (Eq. 10-11) into s_br, count returned; s_cand holds the ranked
+// candidates (s_cand[0] = j*).  Block-wide: every thread must call.
+__device__ __forceinline__ int branch_set(const TreeLaunch &a, int b, const SeqView &v,
+                                          const int *s_cand,
+                          int *s_next, int *s_br, int *s_misc) {
+    const int t = threadIdx.x, W = a.p.branch_width;
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const int js = s_cand[0];
+    if (a.next_topk) {
+        const int32_t *row = a.next_topk + ((int64_t)b * a.ld + js) * a.Kn;
+        if (t < a.Kn) s_next[t] = row[t];
+    } else if (t < v.nc) {
+        s_next[t] = M[s_cand[t] + 1];
+    }
+    if (t == kThreads4 - 1) s_misc[0] = v.lex ? M[js + 1] : -1;
+    __syncthreads();
+    if (t == 0) {
+        int nb = 0;
+        if (a.next_topk) {
+            for (int r = 0; r < a.Kn && nb < W; ++r)
+                if (s_next[r] >= 0) s_br[nb++] = s_next[r];
+        } else {
+            for (int r = 0; r < v.nc && nb < W; ++r) {
+                const int tkn = s_next[r];
+                bool dup = false;
+                for (int e = 0; e < nb; ++e) dup |= s_br[e] == tkn;
+                if (!dup) s_br[nb++] = tkn;
+            }
+        }
+        if (v.lex) {  // Eq. 11
+            int m = 0;
+            for (int e = 0; e < nb; ++e)
+                if (s_br[e] != s_misc[0]) s_br[m++] = s_br[e];
+            nb = m;
+        }
+        s_misc[1] = nb;
+    }
+    __syncthreads();
+    return s_misc[1];
+}
+
+// Warp 0 sorts n <= 32 (score, position) pairs in place by (score desc,
+// position desc).
+__device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int n) {
+    const int lane = threadIdx.x & 31;
+    const float sc = lane < n ? s_score[lane] : -INFINITY;
+    const int cj = lane < n ? s_cand[lane] : -1;
+    int rank = 0;
+    for (int m = 0; m < n; ++m) {
+        const float os = __shfl_sync(0xffffffffu, sc, m);
+        const int oj = __shfl_sync(0xffffffffu, cj, m);
+        rank += better(os, oj, sc, cj) ? 1 : 0;
+    }
+    __syncwarp();
+    if (lane < n) {
+        s_cand[rank] = cj;
+        s_score[rank] = sc;
+    }
+    __syncwarp();
+}
+
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     const TreeLaunch &a = args.p;
     const Workspace &ws = args.ws;
-    extern __shared__ __align__(16) float dsm[];
-    const int d = a.d, k = a.p.k, W = a.p.branch_width, D = a.p.draft_len;
-    const int succ_len = a.p.succ_len;
-    const uint32_t flags = a.p.flags;
-    float *vec = dsm;                                  // [d]   query, then R[j*+1]
-    int *s_tok = (int *)(vec + d);                     // [kSlice4]
-    int *s_sc = s_tok + kSlice4;                       // [kMaxW * kMaxK]
-    float *s_ss = (float *)(s_sc + kMaxW * kMaxK);     // [kMaxW * kMaxK]
-    int *node_par = (int *)(s_ss + kMaxW * kMaxK);     // [kMaxNodes]
-    int *node_depth = node_par + kMaxNodes;            // [kMaxNodes]
-    int *node_path = node_depth + kMaxNodes;           // [kMaxNodes]
-    int *node_src = node_path + kMaxNodes;             // [kMaxNodes]
+    __shared__ int s_tok[kSlice4];
     __shared__ int s_cand[kMaxK];
     __shared__ float s_score[kMaxK];
     __shared__ int s_next[kMaxW];
     __shared__ int s_br[kMaxW];
-    __shared__ int s_scn[kMaxW];
-    __shared__ int s_succ[kMaxW];
-    __shared__ float scratch[32];
-    __shared__ int s_nb, s_main0, s_flag, s_n, s_ext;
+    __shared__ int s_misc[4];
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int nwarps = kThreads4 / 32;
     const int b = blockIdx.y, sl = blockIdx.x;
-    const int len = a.lengths[b];
-    const bool valid = len >= 1 && (int64_t)len <= a.ld;
-    // candidates come from the caller on the standalone path: check the range
-    bool cand_ok = true;
-    const int nc0 = valid ? min(a.n_cand[b], k) : 0;
-    for (int i = 0; i < nc0; ++i) {
-        const int c = a.cand[(int64_t)b * k + i];
-        cand_ok &= c >= 0 && c <= len - 2;
-    }
-    const int hk = (valid && cand_ok) ? a.hit_kind[b] : ADAPLD_HIT_NONE;
-    const int nc = cand_ok ? nc0 : 0;
-    const bool lex = hk == ADAPLD_HIT_LEX && nc > 0;
-    const bool sem = hk == ADAPLD_HIT_SEM && nc > 0;
-    const bool branch_on = !(flags & ADAPLD_NO_BRANCH) && W > 0 && (lex || sem);
-    const bool need_succ = branch_on && !(flags & ADAPLD_NO_SUCC) &&
-                           (sem || (lex && (flags & ADAPLD_SUCC_ON_STRICT)));
-    if (!need_succ && sl != 0) return;
-
+    const int k = a.p.k, d = a.d;
+    pdl_wait_then_release();
+    const SeqView v = view_of(a, b);
+    if (!v.need_succ) return;
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
 
-    // ---- 1. anchor and branch set ------------------------------------------------
-    if (t < nc) {
+    if (t < v.nc) {
         s_cand[t] = a.cand[(int64_t)b * k + t];
         s_score[t] = a.score[(int64_t)b * k + t];
     }
     __syncthreads();
-    if (lex) {
-        if (!(flags & ADAPLD_NO_LEX_RERANK)) {
-            const float qss = block_load_vec(a.query + (int64_t)b * d, vec, d, scratch);
-            for (int ci = warp; ci < nc; ci += nwarps) {
-                float dot, ss;
-                warp_row_dot(R + (int64_t)s_cand[ci] * d, vec, d, dot, ss);
-                if (lane == 0) s_score[ci] = cosine_from(dot, ss, qss);
+    if (v.lex) {  // successors on a strict hit: rerank first (each slice alike)
+        if (!(a.p.flags & ADAPLD_NO_LEX_RERANK)) {
+            const uint16_t *q = a.query + (int64_t)b * d;
+            for (int ci = warp; ci < v.nc; ci += nwarps) {
+                const float cs = warp_cosine(R + (int64_t)s_cand[ci] * d, q, d);
+                if (lane == 0) s_score[ci] = cs;
             }
             __syncthreads();
-            if (warp == 0) {  // sort by (score desc, position desc)
-                const float sc = lane < nc ? s_score[lane] : -INFINITY;
-                const int cj = lane < nc ? s_cand[lane] : -1;
-                int rank = 0;
-                for (int m = 0; m < nc; ++m) {
-                    const float os = __shfl_sync(0xffffffffu, sc, m);
-                    const int oj = __shfl_sync(0xffffffffu, cj, m);
-                    rank += better(os, oj, sc, cj) ? 1 : 0;
-                }
-                __syncwarp();
-                if (lane < nc) {
-                    s_cand[rank] = cj;
-                    s_score[rank] = sc;
-                }
-            }
-        } else if (t < nc) {
+            if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc);
+        } else if (t < v.nc) {
             s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
         }
         __syncthreads();
     }
-    const int js = (lex || sem) ? s_cand[0] : -1;
-    if (branch_on) {
-        if (a.next_topk) {
-            const int32_t *row = a.next_topk + ((int64_t)b * a.ld + js) * a.Kn;
-            if (t < a.Kn) s_next[t] = row[t];
-        } else if (t < nc) {
-            s_next[t] = M[s_cand[t] + 1];
-        }
-        if (t == kThreads4 - 1) s_main0 = lex ? M[js + 1] : -1;
-        __syncthreads();
-        if (t == 0) {
-            int nb = 0;
-            if (a.next_topk) {
-                for (int r = 0; r < a.Kn && nb < W; ++r)
-                    if (s_next[r] >= 0) s_br[nb++] = s_next[r];
-            } else {
-                for (int r = 0; r < nc && nb < W; ++r) {
-                    const int tkn = s_next[r];
-                    bool dup = false;
-                    for (int e = 0; e < nb; ++e) dup |= s_br[e] == tkn;
-                    if (!dup) s_br[nb++] = tkn;
-                }
+    const int nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc);
+
+    const int p0 = sl * kSlice4;
+    const int p1 = min(p0 + kSlice4, v.len - 1);  // positions t <= len-2
+    for (int i = t; i < p1 - p0; i += kThreads4) s_tok[i] = M[p0 + i];
+    __syncthreads();
+    constexpr int U = 8;  // 32-position groups tested per pass (independent loads)
+    for (int w = warp; w < nb; w += nwarps) {
+        const int bt = s_br[w];
+        int32_t *pp = ws.part4 + (((int64_t)b * ws.S4 + sl) * ws.W + w) * kPart4Ints;
+        int cnt = 0;
+        for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32 * U) {
+            unsigned m[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int p = top - 32 * u - lane;
+                m[u] = __ballot_sync(0xffffffffu, p >= p0 && s_tok[p - p0] == bt);
             }
-            if (lex) {  // Eq. 11
-                int m = 0;
-                for (int e = 0; e < nb; ++e)
-                    if (s_br[e] != s_main0) s_br[m++] = s_br[e];
-                nb = m;
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int p = top - 32 * u - lane;
+                const int rank = cnt + __popc(m[u] & ((1u << lane) - 1u));
+                if (((m[u] >> lane) & 1u) && rank < k) pp[1 + rank] = p;
+                cnt += __popc(m[u]);
             }
-            s_nb = nb;
         }
-    } else if (t == 0) {
-        s_nb = 0;
+        if (lane == 0) pp[0] = min(cnt, k);
+    }
+    __threadfence();
+    __syncthreads();
+    if (t == 0) s_misc[2] = atomicAdd(ws.ticket4 + b, 1) == (int)gridDim.x - 1;
+    __syncthreads();
+    if (!s_misc[2]) return;
+    __threadfence();
+    // last slice: merge, most recent first
+    for (int w = warp; w < nb; w += nwarps) {
+        const int32_t *pw = ws.part4 + ((int64_t)b * ws.S4 * ws.W + w) * kPart4Ints;
+        const int64_t stride = (int64_t)ws.W * kPart4Ints;  // next slice, same branch
+        const int total = warp_merge_desc(
+            (int)gridDim.x, k, [&](int s2) { return __ldcg(pw + s2 * stride); },
+            [&](int s2, int i) { return __ldcg(pw + s2 * stride + 1 + i); },
+            ws.succ + ((int64_t)b * ws.W + w) * kMaxK);
+        if (lane == 0) ws.succ_n[(int64_t)b * ws.W + w] = total;
+    }
+    if (v.lex && t < v.nc) {
+        ws.rr_cand[(int64_t)b * kMaxK + t] = s_cand[t];
+        ws.rr_score[(int64_t)b * kMaxK + t] = s_score[t];
+    }
+}
+
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
+    const TreeLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int s_cand[kMaxK];
+    __shared__ float s_score[kMaxK];
+    __shared__ int s_next[kMaxW];
+    __shared__ int s_br[kMaxW];
+    __shared__ int s_succ[kMaxW];
+    __shared__ int s_misc[4];
+    __shared__ int node_par[kMaxNodes];
+    __shared__ short node_depth[kMaxNodes];
+    __shared__ short node_path[kMaxNodes];
+    __shared__ int node_src[kMaxNodes];
+    __shared__ int s_row[kRowsPerCta5];
+    __shared__ float s_red[32];
+    extern __shared__ __align__(16) float s_ref[];  // [d] reference vector (fp32)
+
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int nwarps = kThreads4 / 32;
+    const int b = blockIdx.y, r5 = blockIdx.x;
+    const int k = a.p.k, d = a.d, W = a.p.branch_width, D = a.p.draft_len;
+    const int succ_len = a.p.succ_len;
+    const uint32_t flags = a.p.flags;
+    pdl_wait_then_release();
+    const SeqView v = view_of(a, b);
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
+
+    // ---- ranked candidates (the successor scan reranked a strict hit already)
+    if (t < v.nc) {
+        if (v.need_succ && v.lex) {
+            s_cand[t] = __ldcg(ws.rr_cand + (int64_t)b * kMaxK + t);
+            s_score[t] = __ldcg(ws.rr_score + (int64_t)b * kMaxK + t);
+        } else {
+            s_cand[t] = a.cand[(int64_t)b * k + t];
+            s_score[t] = a.score[(int64_t)b * k + t];
+        }
     }
     __syncthreads();
-    const int nb = s_nb;
+    // with successors the ranking is final here, so the branch set is known
+    int nb = v.need_succ ? branch_set(a, b, v, s_cand, s_next, s_br, s_misc) : 0;
 
-    // ---- 2. successor candidates over this slice ----------------------------------
-    if (need_succ) {
-        const int p0 = sl * kSlice4;
-        const int p1 = min(p0 + kSlice4, len - 1);  // positions t <= len-2
-        for (int i = t; i < p1 - p0; i += kThreads4) s_tok[i] = M[p0 + i];
-        __syncthreads();
-        for (int w = warp; w < nb; w += nwarps) {
-            const int bt = s_br[w];
-            int32_t *pp = ws.part4 + (((int64_t)b * ws.S4 + sl) * ws.W + w) * kPart4Ints;
-            int cnt = 0;
-            for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32) {
-                const int p = top - lane;
-                const bool hit = p >= p0 && s_tok[p - p0] == bt;
-                const unsigned m = __ballot_sync(0xffffffffu, hit);
-                const int rank = cnt + __popc(m & ((1u << lane) - 1u));
-                if (hit && rank < k) pp[1 + rank] = p;
-                cnt += __popc(m);
+    // the rows this sequence scores, and the CTAs that share them: lexical
+    // candidates against the query, or successor candidate (w, i) at w*k + i
+    const bool rerank = v.lex && !v.need_succ && !(flags & ADAPLD_NO_LEX_RERANK);
+    const int ntasks = v.need_succ ? nb * k : (rerank ? v.nc : 0);
+    const int nctas = max(1, (ntasks + kRowsPerCta5 - 1) / kRowsPerCta5);
+    if (r5 >= nctas) return;
+    const int js0 = (v.lex || v.sem) ? s_cand[0] : -1;
+    float *score5 = ws.score5 + (int64_t)b * ws.W * kMaxK;
+
+    // ---- this CTA's share of the scored rows
+    if (ntasks > 0) {
+        const int task0 = r5 * kRowsPerCta5;
+        if (t < kRowsPerCta5) {  // row of each task of this CTA, -1 if none
+            const int task = task0 + t;
+            int row = -1;
+            if (task < ntasks) {
+                if (v.need_succ) {
+                    const int w = task / k, i = task % k;
+                    const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
+                    const int pos = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i);
+                    row = i < n ? pos : -1;
+                } else {
+                    row = s_cand[task];
+                }
             }
-            if (lane == 0) pp[0] = min(cnt, k);
+            s_row[t] = row;
         }
-        __threadfence();
-        __syncthreads();
-        if (t == 0) s_flag = atomicAdd(ws.ticket4 + b, 1) == (int)gridDim.x - 1;
-        __syncthreads();
-        if (!s_flag) return;
-        __threadfence();
-        // merge the slices, most recent first
-        for (int w = warp; w < nb; w += nwarps) {
-            int total = 0;
-            for (int s2 = (int)gridDim.x - 1; s2 >= 0 && total < k; --s2) {
-                const int32_t *pp = ws.part4 + (((int64_t)b * ws.S4 + s2) * ws.W + w) * kPart4Ints;
-                const int n = __ldcg(pp);
-                const int take = min(n, k - total);
-                if (lane < take) s_sc[w * kMaxK + total + lane] = __ldcg(pp + 1 + lane);
-                total += take;
-            }
-            if (lane == 0) s_scn[w] = total;
-        }
-        __syncthreads();
-        // Eq. 13-14: rerank the occurrences against R[j*+1]
-        const float rss = block_load_vec(R + (int64_t)(js + 1) * d, vec, d, scratch);
-        for (int task = warp; task < nb * kMaxK; task += nwarps) {
-            const int w = task / kMaxK, i = task % kMaxK;
-            if (i >= s_scn[w]) continue;
+        const uint16_t *ref = v.need_succ ? R + (int64_t)(js0 + 1) * d : a.query + (int64_t)b * d;
+        const float rss = block_load_vec(ref, s_ref, d, s_red);  // syncs the block
+        const int row = s_row[warp];
+        if (row >= 0) {
             float dot, ss;
-            warp_row_dot(R + (int64_t)s_sc[w * kMaxK + i] * d, vec, d, dot, ss);
-            if (lane == 0) s_ss[w * kMaxK + i] = cosine_from(dot, ss, rss);
+            warp_row_dot(R + (int64_t)row * d, s_ref, d, dot, ss);
+            if (lane == 0) score5[task0 + warp] = cosine_from(dot, ss, rss);
+        }
+        if (nctas > 1) {
+            __threadfence();
+            __syncthreads();
+            if (t == 0) s_misc[2] = atomicAdd(ws.ticket5 + b, 1) == nctas - 1;
+            __syncthreads();
+            if (!s_misc[2]) return;
+            __threadfence();
+        } else {
+            __syncthreads();
+        }
+    }
+
+    // ---- the last CTA of the sequence: rank, branch, pick successors, emit
+    if (rerank) {
+        if (warp == 0) {
+            if (lane < v.nc) s_score[lane] = __ldcg(score5 + lane);
+            __syncwarp();
+            warp_sort_desc(s_cand, s_score, v.nc);
         }
         __syncthreads();
-        for (int w = warp; w < nb; w += nwarps) {
-            const int n = s_scn[w];
-            float bs = lane < n ? s_ss[w * kMaxK + lane] : -INFINITY;
-            int bj = lane < n ? s_sc[w * kMaxK + lane] : -1;
+    } else if (v.lex && (flags & ADAPLD_NO_LEX_RERANK)) {
+        if (t < v.nc) s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
+        __syncthreads();
+    }
+    const int js = (v.lex || v.sem) ? s_cand[0] : -1;
+    if (v.branch_on && !v.need_succ) nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc);
+    if (v.need_succ) {
+        for (int w = warp; w < nb; w += nwarps) {  // Eq. 14: argmax per branch
+            const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
+            const float *sc = score5 + w * k;
+            const int32_t *ps = ws.succ + ((int64_t)b * ws.W + w) * kMaxK;
+            float bs = lane < n ? __ldcg(sc + lane) : -INFINITY;
+            int bj = lane < n ? __ldcg(ps + lane) : -1;
 #pragma unroll
             for (int o = 16; o; o >>= 1) {
                 const float os = __shfl_xor_sync(0xffffffffu, bs, o);
@@ -286,51 +448,48 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
         __syncthreads();
     }
 
-    // ---- 3. the tree ----------------------------------------------------------------
     const int N = 1 + D + W * (1 + succ_len);
     if (t == 0) {
         int n = 0, ext = 0;
-        if (valid) {
+        if (v.valid) {
             node_par[0] = -1;
             node_depth[0] = 0;
             node_path[0] = 0;
-            node_src[0] = len - 1;
+            node_src[0] = v.len - 1;
             n = 1;
-            if (lex) {
-                const int l = min(D, len - 1 - js);
+            if (v.lex) {
+                const int l = min(D, v.len - 1 - js);
                 for (int i = 0; i < l; ++i, ++n) {
                     node_par[n] = i == 0 ? 0 : n - 1;
-                    node_depth[n] = i + 1;
+                    node_depth[n] = (short)(i + 1);
                     node_path[n] = 1;
                     node_src[n] = js + 1 + i;
                 }
             }
             for (int w = 0; w < nb; ++w) {
-                const int bnode = n;
                 node_par[n] = 0;
                 node_depth[n] = 1;
-                node_path[n] = 2 + w;
+                node_path[n] = (short)(2 + w);
                 node_src[n] = -2 - w;  // the branch token itself
                 ++n;
-                if (need_succ && s_succ[w] >= 0) {
+                if (v.need_succ && s_succ[w] >= 0) {
                     const int tb = s_succ[w];
                     int added = 0;
-                    for (int i = 1; i <= succ_len && tb + i <= len - 1; ++i, ++n, ++added) {
+                    for (int i = 1; i <= succ_len && tb + i <= v.len - 1; ++i, ++n, ++added) {
                         node_par[n] = n - 1;
-                        node_depth[n] = 1 + i;
-                        node_path[n] = 2 + w;
+                        node_depth[n] = (short)(1 + i);
+                        node_path[n] = (short)(2 + w);
                         node_src[n] = tb + i;
                     }
-                    (void)bnode;
                     if (added > 0) ++ext;
                 }
             }
         }
-        s_n = n;
-        s_ext = ext;
+        s_misc[0] = n;
+        s_misc[3] = ext;
     }
     __syncthreads();
-    const int n = s_n;
+    const int n = s_misc[0];
     const int64_t ob = (int64_t)b * N;
     for (int i = t; i < N; i += kThreads4) {
         int tok = -1, par = -1, pos = -1;
@@ -338,7 +497,7 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
             const int src = node_src[i];
             tok = src >= 0 ? M[src] : s_br[-2 - src];
             par = node_par[i];
-            pos = len - 1 + node_depth[i];
+            pos = v.len - 1 + node_depth[i];
         }
         a.out.draft_tokens[ob + i] = tok;
         a.out.parents[ob + i] = par;
@@ -348,42 +507,46 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
     for (int idx = t; idx < N * N; idx += kThreads4) {
         const int i = idx / N, j = idx % N;
         const bool anc = i < n && j < n &&
-                         (j == 0 || (node_path[i] == node_path[j] && j <= i && node_path[i] != 0) ||
-                          j == i);
+                         (j == i || j == 0 ||
+                          (node_path[i] == node_path[j] && j <= i && node_path[i] != 0));
         mk[idx] = anc ? 1 : 0;
     }
-    if (lex && t < k) {
-        a.cand[(int64_t)b * k + t] = t < nc ? s_cand[t] : -1;
-        a.score[(int64_t)b * k + t] = t < nc ? s_score[t] : 0.f;
+    if (v.lex && t < k) {
+        a.cand[(int64_t)b * k + t] = t < v.nc ? s_cand[t] : -1;
+        a.score[(int64_t)b * k + t] = t < v.nc ? s_score[t] : 0.f;
     }
     if (t == 0) {
         a.out.anchor[b] = js;
         a.out.n_nodes[b] = n;
         if (a.out.stats) {
-            atomicAdd(a.out.stats + (lex ? 0 : (sem ? 1 : 2)), 1);
-            if (s_ext) atomicAdd(a.out.stats + 3, s_ext);
+            atomicAdd(a.out.stats + (v.lex ? 0 : (v.sem ? 1 : 2)), 1);
+            if (s_misc[3]) atomicAdd(a.out.stats + 3, s_misc[3]);
         }
         if (a.status)
-            a.status[b] = (valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) | (cand_ok ? 0 : ADAPLD_SEQ_BAD_CANDIDATE);
+            a.status[b] = (v.valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) |
+                          (v.cand_ok ? 0 : ADAPLD_SEQ_BAD_CANDIDATE);
     }
 }
 
 }  // namespace
 
-size_t tree_smem_bytes(int d) {
-    return (size_t)d * 4 + (size_t)kSlice4 * 4 + 2 * (size_t)kMaxW * kMaxK * 4 +
-           4 * (size_t)kMaxNodes * 4;
-}
-
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s) {
-    TreeArgs args{a, ws};
-    const size_t smem = tree_smem_bytes(a.d);
+    const int W = a.p.branch_width, k = a.p.k;
+    const bool succ_possible =
+        W > 0 && !(a.p.flags & (ADAPLD_NO_SUCC | ADAPLD_NO_BRANCH));
+    const int tasks = succ_possible ? (W * k > k ? W * k : k) : k;
+    TreeArgs args{a, ws, (tasks + kRowsPerCta5 - 1) / kRowsPerCta5};
+    if (succ_possible) {
+        cudaError_t e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), 0, s,
+                                         args);
+        if (e != cudaSuccess) return e;
+    }
+    const size_t smem = (size_t)a.d * sizeof(float);
     cudaError_t e = cudaFuncSetAttribute(tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e != cudaSuccess) return e;
-    dim3 grid(ws.S4, a.B);
-    tree_kernel<<<grid, kThreads4, smem, s>>>(args);
-    return cudaGetLastError();
+    return launch_dependent(tree_kernel, dim3(args.rows_ctas, a.B), dim3(kThreads4), smem, s,
+                            args);
 }
 
 }  // namespace adapld

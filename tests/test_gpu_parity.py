@@ -338,3 +338,29 @@ def test_full_size_config(cfg):
         got = set(g["cand"][b, : g["n_cand"][b]].tolist())
         assert set(w.planted[b][: w.k]) <= got or len(got) == w.k
     del hw
+
+
+TUNINGS = {64: ["1,4", "2,8", "3,16"], 4096: ["1,2", "2,4", "3,8"], 5120: ["1,2", "2,4"],
+           8192: ["1,1", "2,2", "3,4"], 12288: ["1,1", "2,2"], 16384: ["1,1", "2,2"]}
+
+
+@pytest.mark.parametrize("d", sorted(TUNINGS))
+def test_semantic_launch_shapes(d, monkeypatch):
+    """Every rows-per-stage variant and CTAs-per-SM choice of the semantic
+    kernel gives a valid ranking (the shape only changes the schedule)."""
+    L = 200 if d > 4096 else 700
+    w = synth.make_workload(5, B=3, L=L, d=d, nohit=1.0, seed=d + 7)
+    for tun in TUNINGS[d]:
+        monkeypatch.setenv("ADAPLD_SEMANTIC_TUNING", tun)
+        for tau in (0.1, NEG_INF):
+            P = P_of(w, tau=tau)
+            check_all(w, run_step(w, P), P)
+
+
+def test_long_history_many_chunks():
+    """More than 32 lexical chunks and successor slices per sequence (merges
+    that need several groups of 32 parts)."""
+    w = synth.make_workload(5, B=2, L=300000, d=8, nohit=0.5, seed=41, V=64)
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P), P)
