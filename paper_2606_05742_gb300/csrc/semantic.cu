@@ -36,6 +36,7 @@ namespace {
 
 constexpr int kProducerWarp = kConsumers2 / 32;  // warp 8
 constexpr int kBarQ = 15;                        // named barrier for |q|^2
+constexpr int kBarMerge = 14;                    // named barrier for the final merge
 
 struct SemArgs {
     SemLaunch p;
@@ -131,8 +132,8 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     const int NS = args.nstages;
     const int stage_bytes = args.stage_bytes;
     uint8_t *ring = smem;
-    float *red = (float *)(smem + (size_t)NS * stage_bytes);  // [NS][32][8]
-    float *qred = red + NS * 32 * 8;                           // [2][8]
+    float *red = (float *)(smem + (size_t)NS * stage_bytes);  // [max(NS,3)][32][8]
+    float *qred = red + (NS > 3 ? NS : 3) * 32 * 8;            // [2][8]
     uint64_t *full = (uint64_t *)(qred + 16);                  // [NS]
     uint64_t *empty = full + kMaxStages2;                      // [NS]
     volatile int *abort_flag = (volatile int *)(empty + kMaxStages2);
@@ -316,66 +317,94 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             ++it;
         }
 
-        // ---- end of this CTA's segment of sequence b: publish, maybe merge
-        if (warp == 0 && !aborted && !*abort_flag) {
-            const int slot = b + c;
-            int32_t *sp = ws.slots2 + (int64_t)slot * kSlotInts;
-            if (lane == 0) sp[0] = tk.n;
-            if (lane < tk.n) {
-                sp[1 + lane] = tk.j;
-                sp[1 + kMaxK + lane] = __float_as_int(tk.s);
-            }
-            __threadfence();
-            __syncwarp();
-            const int cfirst = cta_of(plan[b], G, grid);
-            const int clast = cta_of(plan[b + 1] - 1, G, grid);
-            int expected = clast - cfirst + 1;
-            if (G < grid) {
-                expected = 0;
-                for (int cc = cfirst; cc <= clast; ++cc) expected += cta_nonempty(cc, G, grid);
-            }
+        // ---- end of this CTA's segment of sequence b: publish; the CTA that
+        // publishes last for b merges every partial list, with all 8 warps
+        const int cfirst = cta_of(plan[b], G, grid);
+        const int clast = cta_of(plan[b + 1] - 1, G, grid);
+        volatile int *s_flag = (volatile int *)abort_flag + 1;  // the merge decision
+        if (warp == 0) {
             int last = 0;
-            if (lane == 0) last = atomicAdd(ws.done2 + b, 1) == expected - 1;
-            last = __shfl_sync(0xffffffffu, last, 0);
-            if (last) {
-                __threadfence();
-                WarpTopK m;
-                m.reset();
-                for (int cc = cfirst; cc <= clast; ++cc) {
-                    if (!cta_nonempty(cc, G, grid)) continue;
-                    const int32_t *op = ws.slots2 + (int64_t)(b + cc) * kSlotInts;
-                    const int n = __ldcg(op);
-                    float xs = 0.f;
-                    int xj = -1;
-                    if (lane < n) {
-                        xj = __ldcg(op + 1 + lane);
-                        xs = __int_as_float(__ldcg(op + 1 + kMaxK + lane));
-                    }
-                    m.insert(lane < n, xs, xj, k);
+            if (!aborted && !*abort_flag) {
+                int32_t *sp = ws.slots2 + (int64_t)(b + c) * kSlotInts;
+                if (lane == 0) sp[0] = tk.n;
+                if (lane < tk.n) {
+                    sp[1 + lane] = tk.j;
+                    sp[1 + kMaxK + lane] = __float_as_int(tk.s);
                 }
+                __threadfence();
+                __syncwarp();
+                int expected = clast - cfirst + 1;
+                if (G < grid) {
+                    expected = 0;
+                    for (int cc = cfirst; cc <= clast; ++cc) expected += cta_nonempty(cc, G, grid);
+                }
+                if (lane == 0) last = atomicAdd(ws.done2 + b, 1) == expected - 1;
+                last = __shfl_sync(0xffffffffu, last, 0);
+            }
+            if (lane == 0) *s_flag = last;
+        }
+        named_bar_sync(kBarMerge, kConsumers2);
+        const bool merge = *s_flag != 0;
+        if (merge) {
+            __threadfence();
+            // each warp merges every 8th contributing CTA's list, 4 lists per
+            // round of independent loads
+            WarpTopK m;
+            m.reset();
+            for (int cc0 = cfirst + warp * 4; cc0 <= clast; cc0 += 8 * 4) {
+                int n[4], xj[4];
+                float xs[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    const int cc = cc0 + u;
+                    const bool ok = cc <= clast && cta_nonempty(cc, G, grid);
+                    const int32_t *op = ws.slots2 + (int64_t)(b + (ok ? cc : c)) * kSlotInts;
+                    n[u] = ok ? __ldcg(op) : 0;
+                    xj[u] = ok ? __ldcg(op + 1 + lane) : -1;
+                    xs[u] = ok ? __int_as_float(__ldcg(op + 1 + kMaxK + lane)) : 0.f;
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u) m.insert(lane < n[u], xs[u], xj[u], k);
+            }
+            float *wl_s = red;                          // [8][32] per-warp lists
+            int *wl_j = (int *)(red + 8 * 32);          // [8][32]
+            int *wl_n = (int *)(red + 16 * 32);         // [8]
+            wl_s[warp * 32 + lane] = m.s;
+            wl_j[warp * 32 + lane] = m.j;
+            if (lane == 0) wl_n[warp] = m.n;
+            named_bar_sync(kBarMerge, kConsumers2);
+            if (warp == 0) {
+                WarpTopK f;
+                f.reset();
+                for (int w = 0; w < 8; ++w)
+                    f.insert(lane < wl_n[w], wl_s[w * 32 + lane], wl_j[w * 32 + lane], k);
                 if (lane < k) {
-                    a.cand[(int64_t)b * k + lane] = lane < m.n ? m.j : -1;
-                    a.score[(int64_t)b * k + lane] = lane < m.n ? m.s : 0.f;
+                    a.cand[(int64_t)b * k + lane] = lane < f.n ? f.j : -1;
+                    a.score[(int64_t)b * k + lane] = lane < f.n ? f.s : 0.f;
                 }
                 if (lane == 0) {
-                    a.n_cand[b] = m.n;
-                    if (a.hit_kind) a.hit_kind[b] = m.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
+                    a.n_cand[b] = f.n;
+                    if (a.hit_kind) a.hit_kind[b] = f.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
                 }
             }
+            named_bar_sync(kBarMerge, kConsumers2);  // before red is reused by the next stage
         }
         g = seg_end;
         ++segno;
     }
 }
 
-// Shared memory per CTA: the ring, the per-stage reduction buffers, |q|^2
-// partials, the barriers and the abort flag.
+// Shared memory per CTA: the ring, the per-stage reduction buffers (at least
+// three, which the final merge reuses for the per-warp lists), |q|^2
+// partials, the barriers, the abort flag and the merge decision.
 inline size_t semantic_smem(int ns, int stage) {
-    return (size_t)ns * stage + (size_t)ns * 32 * 8 * 4 + 16 * 4 + 2 * kMaxStages2 * 8 + 16;
+    return (size_t)ns * stage + (size_t)(ns > 3 ? ns : 3) * 32 * 8 * 4 + 16 * 4 +
+           2 * kMaxStages2 * 8 + 16;
 }
 
 template <int MAXC, int SR>
-cudaError_t launch_variant(const SemArgs &args0, int sms, int ctas_per_sm, cudaStream_t s) {
+cudaError_t launch_variant(const SemArgs &args0, int sms, int ctas_per_sm, int stages,
+                           cudaStream_t s) {
     SemArgs args = args0;
     auto kern = semantic_kernel<MAXC, SR>;
     const int stage = (int)align_up((size_t)SR * args.p.d * 2, 128);
@@ -386,7 +415,9 @@ cudaError_t launch_variant(const SemArgs &args0, int sms, int ctas_per_sm, cudaS
     for (; cps >= 1; --cps) {
         const size_t budget = (per_sm - (size_t)(cps - 1) * 1024) / cps;
         ns = 0;
-        while (ns < kMaxStages2 && semantic_smem(ns + 1, stage) <= budget) ++ns;
+        while (ns < kMaxStages2 && (stages <= 0 || ns < stages) &&
+               semantic_smem(ns + 1, stage) <= budget)
+            ++ns;
         if (ns >= 2) break;
     }
     if (cps < 1 || ns < 2) return cudaErrorInvalidConfiguration;
@@ -403,26 +434,32 @@ cudaError_t launch_variant(const SemArgs &args0, int sms, int ctas_per_sm, cudaS
     if (cps > fit) cps = fit;
     int grid = sms * cps;
     if (grid > kMaxGrid2) grid = kMaxGrid2;
+    if (std::getenv("ADAPLD_SEMANTIC_TUNING"))
+        std::fprintf(stderr, "adapld semantic: d=%d rows/stage=%d stages=%d stage_bytes=%d "
+                     "ctas/SM=%d grid=%d smem=%zu\n", args.p.d, SR, ns, stage, cps, grid, smem);
     return launch_dependent(kern, dim3(grid), dim3(kConsumers2 + 32), smem, s, args);
 }
 
-// Launch shape: CTAs per SM and rows per stage.  The defaults per dimension
-// range come from a sweep on GB300 (more resident consumer warps hide the
-// shared-load and FMA latencies; the ring per SM stays ~192 KB):
-//   d <= 4096: 3 CTAs/SM x 4 rows, d <= 6144: 2 x 4, d <= 8192: 3 x 2.
-// ADAPLD_SEMANTIC_TUNING="<ctas_per_sm>,<rows_per_stage>" overrides them, for
-// tuning sweeps (0 keeps the default).
+// Launch shape: CTAs per SM, rows per stage and stages per CTA.  The defaults
+// come from sweeps on GB300: about 128 KB of bulk copies in flight per SM, in
+// 32-64 KB copies, is fastest (deeper rings lose bandwidth, 16 KB copies too),
+// i.e. 2 CTAs/SM with 2 stages of ~32-48 KB for d <= 8192.
+// ADAPLD_SEMANTIC_TUNING="<ctas_per_sm>,<rows_per_stage>[,<stages>]" overrides
+// them for tuning sweeps (0 keeps the default; the launch shape chosen is then
+// printed to stderr).
 struct SemTuning {
     int ctas_per_sm = 0;
     int rows = 0;
+    int stages = 0;
 };
 
 SemTuning semantic_tuning() {
     SemTuning t;
     if (const char *e = std::getenv("ADAPLD_SEMANTIC_TUNING")) {
-        int a = 0, b = 0;
-        if (std::sscanf(e, "%d,%d", &a, &b) >= 1 && a >= 1 && a <= 4) t.ctas_per_sm = a;
+        int a = 0, b = 0, c = 0;
+        if (std::sscanf(e, "%d,%d,%d", &a, &b, &c) >= 1 && a >= 1 && a <= 4) t.ctas_per_sm = a;
         if (b == 1 || b == 2 || b == 4 || b == 8 || b == 16) t.rows = b;
+        if (c >= 2 && c <= kMaxStages2) t.stages = c;
     }
     return t;
 }
@@ -447,33 +484,34 @@ cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_
     const SemTuning tun = semantic_tuning();
     SemArgs args{a, ws, 0, 0};
     const int d = a.d, R = tun.rows;
-#define ADAPLD_SEM(MAXC, SR, CPS) \
-    return launch_variant<MAXC, SR>(args, sms, tun.ctas_per_sm ? tun.ctas_per_sm : CPS, s)
+#define ADAPLD_SEM(MAXC, SR, CPS, NS)                                                       \
+    return launch_variant<MAXC, SR>(args, sms, tun.ctas_per_sm ? tun.ctas_per_sm : CPS,       \
+                                    tun.stages ? tun.stages : NS, s)
     if (d <= 2048) {
-        if (R == 4) ADAPLD_SEM(1, 4, 3);
-        if (R == 8) ADAPLD_SEM(1, 8, 3);
-        ADAPLD_SEM(1, 16, 3);
+        if (R == 4) ADAPLD_SEM(1, 4, 2, 2);
+        if (R == 16) ADAPLD_SEM(1, 16, 2, 2);
+        ADAPLD_SEM(1, 8, 2, 2);
     }
     if (d <= 4096) {
-        if (R == 2) ADAPLD_SEM(2, 2, 3);
-        if (R == 8) ADAPLD_SEM(2, 8, 3);
-        ADAPLD_SEM(2, 4, 3);
+        if (R == 2) ADAPLD_SEM(2, 2, 2, 2);
+        if (R == 8) ADAPLD_SEM(2, 8, 2, 2);
+        ADAPLD_SEM(2, 4, 2, 2);
     }
     if (d <= 6144) {
-        if (R == 2) ADAPLD_SEM(3, 2, 2);
-        ADAPLD_SEM(3, 4, 2);
+        if (R == 2) ADAPLD_SEM(3, 2, 2, 2);
+        ADAPLD_SEM(3, 4, 2, 2);
     }
     if (d <= 8192) {
-        if (R == 1) ADAPLD_SEM(4, 1, 3);
-        if (R == 4) ADAPLD_SEM(4, 4, 3);
-        ADAPLD_SEM(4, 2, 3);
+        if (R == 1) ADAPLD_SEM(4, 1, 2, 4);
+        if (R == 4) ADAPLD_SEM(4, 4, 1, 2);
+        ADAPLD_SEM(4, 2, 2, 2);
     }
     if (d <= 12288) {
-        if (R == 2) ADAPLD_SEM(6, 2, 2);
-        ADAPLD_SEM(6, 1, 2);
+        if (R == 2) ADAPLD_SEM(6, 2, 1, 2);
+        ADAPLD_SEM(6, 1, 2, 3);
     }
-    if (R == 2) ADAPLD_SEM(8, 2, 2);
-    ADAPLD_SEM(8, 1, 2);
+    if (R == 2) ADAPLD_SEM(8, 2, 1, 2);
+    ADAPLD_SEM(8, 1, 1, 4);
 #undef ADAPLD_SEM
 }
 

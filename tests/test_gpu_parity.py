@@ -340,8 +340,9 @@ def test_full_size_config(cfg):
     del hw
 
 
-TUNINGS = {64: ["1,4", "2,8", "3,16"], 4096: ["1,2", "2,4", "3,8"], 5120: ["1,2", "2,4"],
-           8192: ["1,1", "2,2", "3,4"], 12288: ["1,1", "2,2"], 16384: ["1,1", "2,2"]}
+TUNINGS = {64: ["1,4,2", "2,8,3", "3,16,4"], 4096: ["1,2,5", "2,4,2", "3,8,2"],
+           5120: ["1,2,3", "2,4,2"], 8192: ["1,1,8", "2,2,2", "1,4,3"],
+           12288: ["1,1,2", "2,2,2"], 16384: ["1,1,4", "2,2,2"]}
 
 
 @pytest.mark.parametrize("d", sorted(TUNINGS))
