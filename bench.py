@@ -58,6 +58,31 @@ def peaks():
     return 6800.0, "fallback"
 
 
+# ------------------------------------------------------- multi-process
+def max_over_ranks(value: float, device=None) -> float:
+    """The maximum of a per-rank value over the process group (the value
+    itself without one).  Used for the slowest rank's elapsed time."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, steps: int, max_ms: float) -> float:
+    """Whole-job steps/s: every rank runs `steps` steps of its own batch of B
+    sequences (weak scaling), so the job completes world*steps in the slowest
+    rank's time."""
+    return world * steps / (max_ms / 1000.0)
+
+
+def rank_seed(seed: int, rank: int) -> int:
+    """Each rank draws its own batch."""
+    return seed + rank
+
+
 # --------------------------------------------------------------- clocks
 class ClockSampler:
     """nvidia-smi sampling of SM clocks and throttle reasons during the timed
@@ -239,7 +264,7 @@ def run_native(args):
             dist.barrier()
 
     cfg = args.config
-    w = synth.make_workload(cfg, device=str(dev), seed=args.seed + rank, B=args.batch)
+    w = synth.make_workload(cfg, device=str(dev), seed=rank_seed(args.seed, rank), B=args.batch)
     p = native.make_params(w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, 0)
     eng = native.Engine(w.B, w.ld, w.d, p, device=dev)
     stream = torch.cuda.current_stream(dev)
@@ -294,12 +319,9 @@ def run_native(args):
     stage = {name: [r[2 * i].elapsed_time(r[2 * i + 1]) for r in ev]
              for i, name in enumerate(("lexical", "semantic", "tree"))}
     sem_ms = stage["semantic"]
-    t = torch.tensor([total_ms], device=dev)
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dev)
     ms_per_step = total_ms / K
-    value = world * K / (total_ms / 1000.0)
+    value = job_throughput(world, K, total_ms)
 
     # end-to-end through the public API from pinned host buffers
     e2e = None
@@ -326,10 +348,8 @@ def run_native(args):
         e1.record(stream)
         torch.cuda.synchronize(dev)
         barrier()
-        te = torch.tensor([e0.elapsed_time(e1)], device=dev)
-        if world > 1:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e = {"value": world * KE / (float(te.item()) / 1000.0), "unit": UNIT,
+        te = max_over_ranks(e0.elapsed_time(e1), dev)
+        e2e = {"value": job_throughput(world, KE, te), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
         del reps_h, dev_in
 

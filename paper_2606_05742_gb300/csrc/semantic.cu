@@ -14,17 +14,21 @@
 //    evict-first); a stage holds SR whole rows (one contiguous block).
 //  * 8 consumer warps own fixed column slices: thread t holds the query
 //    columns [8(t + 256c), +8) for c < MAXC in registers, so a row costs one
-//    16-byte shared load, 8 FMAs for <R, q> and 8 for |R|^2 per slice.  The
+//    16-byte shared load and packed f32x2 FMAs for <R, q> and |R|^2.  The
 //    2*SR partial sums of a stage are reduced across each warp with a
-//    reduce-scatter, then across warps through shared memory.
+//    reduce-scatter, then across warps through shared memory; warps 1-7
+//    signal them on a per-stage mbarrier that warp 0 waits on.
 //  * Warp 0 finishes the cosines and keeps a register-resident top-k (one
 //    entry per lane) that it updates with ballots.  At the end of each
 //    sequence segment it publishes its partial list; the last CTA to publish
 //    for a sequence (atomic counter) merges all partial lists, so the result
 //    does not depend on CTA timing.
-//  * Every mbarrier wait is bounded; on expiry the CTA raises
-//    ADAPLD_DEV_TIMEOUT, stops issuing copies, drains the copies in flight and
-//    exits without publishing.
+//  * Every wait inside the streaming loop is a bounded mbarrier wait; on
+//    expiry the CTA raises ADAPLD_DEV_TIMEOUT, stops issuing copies, drains
+//    the copies in flight, skips all further waits and exits without
+//    publishing.  The only named barriers are the full-CTA ones at the start
+//    and end of each sequence segment, which every consumer warp reaches in
+//    the same order whatever happened in between.
 #include <cstdio>
 #include <cstdlib>
 
@@ -43,6 +47,8 @@ struct SemArgs {
     Workspace ws;
     int nstages;
     int stage_bytes;
+    uint64_t wait_limit_ns;  // bound of every mbarrier wait
+    int stall;               // test switch: the producer issues no copy
 };
 
 // Reduce-scatter of N values across a warp (N a power of two <= 32): after
@@ -134,9 +140,10 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     uint8_t *ring = smem;
     float *red = (float *)(smem + (size_t)NS * stage_bytes);  // [max(NS,3)][32][8]
     float *qred = red + (NS > 3 ? NS : 3) * 32 * 8;            // [2][8]
-    uint64_t *full = (uint64_t *)(qred + 16);                  // [NS]
-    uint64_t *empty = full + kMaxStages2;                      // [NS]
-    volatile int *abort_flag = (volatile int *)(empty + kMaxStages2);
+    uint64_t *full = (uint64_t *)(qred + 16);                  // [NS] stage landed
+    uint64_t *empty = full + kMaxStages2;                      // [NS] stage consumed
+    uint64_t *redbar = empty + kMaxStages2;                    // [NS] partial sums written
+    volatile int *abort_flag = (volatile int *)(redbar + kMaxStages2);
 
     pdl_wait_then_release();  // the plan and the lexical outcomes come from the previous kernel
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
@@ -155,6 +162,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
         for (int s = 0; s < NS; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], kConsumers2 / 32);
+            mbar_init(&redbar[s], kConsumers2 / 32 - 1);
         }
         *abort_flag = 0;
         fence_barrier_init();
@@ -184,11 +192,11 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             for (int j = (int)(g - plan[b]); j < jend; j += SR) {
                 const int nrows = min(SR, jend - j);
                 const int s = it % NS, r = it / NS;
-                if (r > 0 && !mbar_wait_bounded(&empty[s], (r - 1) & 1)) {
+                if (r > 0 && !mbar_wait_bounded(&empty[s], (r - 1) & 1, args.wait_limit_ns)) {
                     failed = true;
                     break;
                 }
-                if (*abort_flag) {
+                if (*abort_flag || args.stall) {
                     failed = true;
                     break;
                 }
@@ -205,7 +213,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
             // drain the copies still in flight before the CTA may exit
             for (int i = max(0, it - NS); i < it; ++i)
-                (void)mbar_wait_bounded(&full[i % NS], (uint32_t)(i / NS) & 1);
+                (void)mbar_wait_bounded(&full[i % NS], (uint32_t)(i / NS) & 1, args.wait_limit_ns);
         }
         return;
     }
@@ -258,7 +266,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             const int nrows = min(SR, jend - j);
             const int s = it % NS;
             const uint32_t ph = (uint32_t)(it / NS) & 1;
-            if (!aborted && !mbar_wait_bounded(&full[s], ph)) {
+            if (!aborted && !mbar_wait_bounded(&full[s], ph, args.wait_limit_ns)) {
                 aborted = true;
                 *abort_flag = 1;
                 atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
@@ -296,10 +304,19 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             if (lane % GRP == 0) red[(s * 32 + lane / GRP) * 8 + warp] = acc[0];
             __syncwarp();
             if (warp != 0) {
-                if (lane == 0) mbar_arrive(&empty[s]);
-                named_bar_arrive(1 + s, kConsumers2);
+                if (lane == 0) {
+                    mbar_arrive(&redbar[s]);
+                    mbar_arrive(&empty[s]);
+                }
             } else {
-                named_bar_sync(1 + s, kConsumers2);
+                // the other warps' partial sums of this stage (bounded; once
+                // aborted the results are discarded and nothing is waited for)
+                if (*abort_flag) aborted = true;
+                if (!aborted && !mbar_wait_bounded(&redbar[s], ph, args.wait_limit_ns)) {
+                    aborted = true;
+                    *abort_flag = 1;
+                    atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
+                }
                 float dot = 0.f, ss = 0.f;
                 if (lane < nrows) {
 #pragma unroll
@@ -399,7 +416,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
 // partials, the barriers, the abort flag and the merge decision.
 inline size_t semantic_smem(int ns, int stage) {
     return (size_t)ns * stage + (size_t)(ns > 3 ? ns : 3) * 32 * 8 * 4 + 16 * 4 +
-           2 * kMaxStages2 * 8 + 16;
+           3 * kMaxStages2 * 8 + 16;
 }
 
 template <int MAXC, int SR>
@@ -482,7 +499,16 @@ cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_
     const int sms = semantic_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
     const SemTuning tun = semantic_tuning();
-    SemArgs args{a, ws, 0, 0};
+    SemArgs args{a, ws, 0, 0, kWaitLimitNs, 0};
+    // Test switch for the timeout path: the producer issues nothing, every
+    // consumer wait runs out after 20 ms, the call reports ADAPLD_DEV_TIMEOUT
+    // and publishes no result.  Never set in normal use.
+    if (const char *e = std::getenv("ADAPLD_TEST_SEMANTIC_STALL")) {
+        if (e[0] == '1') {
+            args.stall = 1;
+            args.wait_limit_ns = 20000000ull;
+        }
+    }
     const int d = a.d, R = tun.rows;
 #define ADAPLD_SEM(MAXC, SR, CPS, NS)                                                       \
     return launch_variant<MAXC, SR>(args, sms, tun.ctas_per_sm ? tun.ctas_per_sm : CPS,       \

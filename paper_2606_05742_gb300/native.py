@@ -289,21 +289,42 @@ class Engine:
         return self.out
 
     def run_from_host(self, tokens_h, lengths_h, reps_h, query_h, dev_inputs, host_out,
-                      stream=None):
+                      stream=None, copy_streams: int = 4):
         """End-to-end step from pinned host inputs: copies them into the
         device buffers ``dev_inputs`` (tokens, lengths, reps, query), runs the
         step and copies every output back into the pinned ``host_out`` list
-        (same order as :meth:`Outputs.tensors`).  Returns bytes moved
-        (host->device, device->host)."""
+        (same order as :meth:`Outputs.tensors`).  The representation cache is
+        copied in ``copy_streams`` row blocks on side streams so that several
+        copy engines share the host link.  Returns bytes moved (host->device,
+        device->host)."""
+        import torch
+        main = torch.cuda.current_stream(self.device) if stream is None else stream
         tok_d, len_d, reps_d, q_d = dev_inputs
+        if getattr(self, "_copy_streams", None) is None or len(self._copy_streams) != copy_streams:
+            self._copy_streams = [torch.cuda.Stream(device=self.device)
+                                  for _ in range(copy_streams)]
         h2d = 0
-        for src, dst in ((tokens_h, tok_d), (lengths_h, len_d), (reps_h, reps_d),
-                         (query_h, q_d)):
-            dst.copy_(src, non_blocking=True)
-            h2d += src.numel() * src.element_size()
-        self.run(tok_d, len_d, reps_d, q_d, stream=stream)
-        d2h = 0
-        for src, dst in zip(self.out.tensors(), host_out):
-            dst.copy_(src, non_blocking=True)
-            d2h += src.numel() * src.element_size()
+        start = torch.cuda.Event()
+        start.record(main)
+        rows_h = reps_h.view(-1, reps_h.shape[-1])
+        rows_d = reps_d.view(-1, reps_d.shape[-1])
+        n = rows_h.shape[0]
+        bounds = [n * i // copy_streams for i in range(copy_streams + 1)]
+        for s, lo, hi in zip(self._copy_streams, bounds[:-1], bounds[1:]):
+            s.wait_event(start)
+            with torch.cuda.stream(s):
+                rows_d[lo:hi].copy_(rows_h[lo:hi], non_blocking=True)
+            done = torch.cuda.Event()
+            done.record(s)
+            main.wait_event(done)
+        h2d += reps_h.numel() * reps_h.element_size()
+        with torch.cuda.stream(main):
+            for src, dst in ((tokens_h, tok_d), (lengths_h, len_d), (query_h, q_d)):
+                dst.copy_(src, non_blocking=True)
+                h2d += src.numel() * src.element_size()
+            self.run(tok_d, len_d, reps_d, q_d, stream=main)
+            d2h = 0
+            for src, dst in zip(self.out.tensors(), host_out):
+                dst.copy_(src, non_blocking=True)
+                d2h += src.numel() * src.element_size()
         return h2d, d2h

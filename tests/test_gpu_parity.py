@@ -365,3 +365,47 @@ def test_long_history_many_chunks():
     for tau in (0.1, NEG_INF):
         P = P_of(w, tau=tau)
         check_all(w, run_step(w, P), P)
+
+
+def test_semantic_wait_timeout_is_reported_and_recoverable(monkeypatch):
+    """Failure path without a fault: with the test switch the semantic
+    kernel's producer issues no copy, so every bounded wait expires; the call
+    must report ADAPLD_DEV_TIMEOUT through the workspace status word, and the
+    next normal call on the same context must succeed with correct results."""
+    w = synth.make_workload(2, B=4, L=3000, d=256, nohit=1.0, seed=51)
+    P = P_of(w)
+    tok, ln, reps, q = to_dev(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    monkeypatch.setenv("ADAPLD_TEST_SEMANTIC_STALL", "1")
+    eng.run(tok, ln, reps, q)
+    torch.cuda.synchronize()
+    assert native.read_device_status(eng.ws) & native.DEV_TIMEOUT
+    monkeypatch.delenv("ADAPLD_TEST_SEMANTIC_STALL")
+    g = run_step(w, P)
+    check_all(w, g, P)
+
+
+def test_end_to_end_from_host_matches_device_path():
+    """The public end-to-end call (pinned host inputs, copies on side streams,
+    outputs copied back) returns what the device-resident call returns."""
+    w = synth.make_workload(4, B=12, L=900, d=128, seed=61)
+    P = P_of(w)
+    g = run_step(w, P)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    tok_h = torch.from_numpy(w.tokens).pin_memory()
+    len_h = torch.from_numpy(w.lengths).pin_memory()
+    reps_h = torch.from_numpy(w.reps.view(np.int16)).view(torch.bfloat16).pin_memory()
+    q_h = torch.from_numpy(w.query.view(np.int16)).view(torch.bfloat16).pin_memory()
+    dev = (torch.empty(tok_h.shape, dtype=tok_h.dtype, device="cuda"),
+           torch.empty(len_h.shape, dtype=len_h.dtype, device="cuda"),
+           torch.empty(reps_h.shape, dtype=reps_h.dtype, device="cuda"),
+           torch.empty(q_h.shape, dtype=q_h.dtype, device="cuda"))
+    host_out = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in eng.out.tensors()]
+    for _ in range(2):
+        h2d, d2h = eng.run_from_host(tok_h, len_h, reps_h, q_h, dev, host_out)
+        torch.cuda.synchronize()
+        names = ["hit_kind", "match_n", "cand", "score", "n_cand", "status", "anchor",
+                 "draft_tokens", "parents", "positions", "mask", "n_nodes", "stats"]
+        for name, t in zip(names, host_out):
+            assert np.array_equal(t.numpy(), g[name], equal_nan=True), name
+    assert h2d == w.tokens.nbytes + w.lengths.nbytes + w.reps.nbytes + w.query.nbytes
