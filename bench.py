@@ -49,6 +49,25 @@ def parse():
     return ap.parse_args()
 
 
+def semantic_traffic(algorithmic_bytes: int):
+    """DRAM traffic of one semantic-kernel launch, from the committed ncu
+    capture (traffic/algorithmic ratio, scaled to this launch's bytes, which
+    grow in proportion), or None once the kernel source differs from the
+    captured one."""
+    import hashlib
+    prof = os.path.join(ROOT, "profiles", "semantic_kernel_config5_B2.md")
+    csrc = os.path.join(ROOT, "paper_2606_05742_gb300", "csrc")
+    if not os.path.exists(prof):
+        return None
+    text = open(prof).read()
+    for name in ("semantic.cu", "common.cuh"):
+        h = hashlib.sha256(open(os.path.join(csrc, name), "rb").read()).hexdigest()
+        if f"{name} sha256 {h}" not in text:
+            return None
+    ratio = [ln.split(":", 1)[1] for ln in text.splitlines() if ln.startswith("traffic_ratio:")]
+    return int(float(ratio[0]) * algorithmic_bytes) if ratio else None
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -383,7 +402,8 @@ def run_native(args):
         "config": conf,
         "roofline": {"bound": "hbm", "kernel": "semantic_kernel",
                      "achieved": achieved, "peak": peak, "peak_kind": peak_kind,
-                     "unit": "GB/s", "frac": achieved / peak, "traffic": None,
+                     "unit": "GB/s", "frac": achieved / peak,
+                     "traffic": semantic_traffic(nbytes["semantic"]),
                      "algorithmic_bytes": nbytes["semantic"], "avg_launch_ms": sem_avg_ms},
         "step_hbm": {"achieved": step_gbs, "frac": step_gbs / peak,
                      "algorithmic_bytes": nbytes["step"]},
