@@ -68,6 +68,18 @@ def _load():
         lib.oracle_step.argtypes = [P, i64, P, P, i32, P, P, i32, i32, i32, i32, i32, i32,
                                     i32, f64, u32, i32, P, P, P, P, P, P, P, P, P, P, P, P]
         lib.oracle_step.restype = None
+        lib.oracle_step_emb.argtypes = [P, i64, P, P, i32, P, P, i32, P, i32, i32, i32, i32,
+                                        i32, i32, i32, f64, u32, i32, P, P, P, P, P, P, P, P,
+                                        P, P, P, P]
+        lib.oracle_step_emb.restype = None
+        lib.oracle_semantic_emb.argtypes = [P, i32, P, i32, i32, f64, P, P]
+        lib.oracle_semantic_emb.restype = i32
+        lib.oracle_successor_candidates_emb.argtypes = [P, i32, P, i32, P, i32, f64, i32, i32,
+                                                        i32, P, P]
+        lib.oracle_successor_candidates_emb.restype = i32
+        lib.oracle_tree_from_emb.argtypes = [P, i32, P, i32, P, i32, f64, i32, P, i32, P, i32,
+                                             i32, i32, i32, i32, u32, i32, P, P, P, P, P, P]
+        lib.oracle_tree_from_emb.restype = i32
         _lib = lib
     return _lib
 
@@ -114,6 +126,32 @@ def semantic(R, q, length: int, k: int, tau: float):
     return cand[:n].tolist(), score[:n].tolist()
 
 
+def semantic_emb(M, length: int, E, k: int, tau: float):
+    """Eq. 4 over token embeddings, cos(E[M[j]], E[M[len-1]]), capped at k:
+    returns ([positions], [scores]) best first."""
+    M = _c(M, np.int32)
+    E = _c(E, np.uint16)
+    cand = np.full(max(k, 1), -1, np.int32)
+    score = np.zeros(max(k, 1), np.float64)
+    n = _load().oracle_semantic_emb(_p(M), length, _p(E), E.shape[1], k, float(tau), _p(cand),
+                                    _p(score))
+    return cand[:n].tolist(), score[:n].tolist()
+
+
+def successor_candidates_emb(M, length: int, R, d: int, E, tau: float, j_star: int, b: int,
+                             k: int):
+    """Sec. 3.5 lexical-first backoff for branch token b (embedding fallback
+    when b never occurs), each candidate scored by Eq. 13."""
+    M = _c(M, np.int32)
+    R = _c(R, np.uint16)
+    E = _c(E, np.uint16)
+    t = np.zeros(max(k, 1), np.int32)
+    s = np.zeros(max(k, 1), np.float64)
+    n = _load().oracle_successor_candidates_emb(_p(M), length, _p(R), d, _p(E), E.shape[1],
+                                                float(tau), j_star, b, k, _p(t), _p(s))
+    return t[:n].tolist(), s[:n].tolist()
+
+
 def scores_all(R, q, length: int) -> np.ndarray:
     """Every Eq. 4 score cos(R[j], q), j in [0, length-2], in fp64."""
     R = _c(R, np.uint16)
@@ -156,9 +194,11 @@ class Tree:
 
 
 def tree_from(M, length: int, R, d: int, hit: int, cands, k: int, W: int, D: int,
-              succ_len: int = 1, flags: int = 0, topk_row=None) -> Tree:
+              succ_len: int = 1, flags: int = 0, topk_row=None, emb=None,
+              tau: float = 0.1) -> Tree:
     """Draft tree (Sec. 3.5, Algorithm 1) from a retrieval outcome and its
-    ranked candidate list (cands[0] is the anchor j*)."""
+    ranked candidate list (cands[0] is the anchor j*); with an embedding
+    table `emb`, successor drafting backs off to the embedding fallback."""
     M = _c(M, np.int32)
     R = _c(R, np.uint16)
     c = _c(cands, np.int32) if len(cands) else np.zeros(1, np.int32)
@@ -174,9 +214,14 @@ def tree_from(M, length: int, R, d: int, hit: int, cands, k: int, W: int, D: int
         trp, kn = _p(tr), tr.shape[0]
     else:
         trp, kn = None, 0
-    ext = _load().oracle_tree_from(_p(M), length, _p(R), d, hit, _p(c), len(cands), trp, kn,
-                                   k, W, D, succ_len, flags, nmax, _p(anchor), _p(tok), _p(par),
-                                   _p(pos), _p(mask), _p(nn))
+    if emb is not None:
+        E = _c(emb, np.uint16)
+        Ep, de = _p(E), E.shape[1]
+    else:
+        Ep, de = None, 0
+    ext = _load().oracle_tree_from_emb(_p(M), length, _p(R), d, Ep, de, float(tau), hit, _p(c),
+                                       len(cands), trp, kn, k, W, D, succ_len, flags, nmax,
+                                       _p(anchor), _p(tok), _p(par), _p(pos), _p(mask), _p(nn))
     return Tree(int(anchor[0]), tok, par, pos, mask, int(nn[0]), int(ext))
 
 
@@ -197,10 +242,12 @@ class StepResult:
 
 
 def step(tokens, lengths, reps, query, n_max: int, k: int, W: int, D: int,
-         succ_len: int = 1, tau: float = 0.1, flags: int = 0, next_topk=None) -> StepResult:
+         succ_len: int = 1, tau: float = 0.1, flags: int = 0, next_topk=None,
+         emb=None) -> StepResult:
     """One draft-construction step for a batch (layouts as in the library):
     tokens [B][ld] int32, lengths [B], reps [B][ld][d] bf16 bits,
-    query [B][d] bf16 bits, next_topk [B][ld][Kn] int32 or None."""
+    query [B][d] bf16 bits, next_topk [B][ld][Kn] int32 or None, emb [V][de]
+    bf16 bits (token embeddings) or None."""
     tokens = _c(tokens, np.int32)
     lengths = _c(lengths, np.int32)
     reps = _c(reps, np.uint16)
@@ -226,8 +273,13 @@ def step(tokens, lengths, reps, query, n_max: int, k: int, W: int, D: int,
         ntp, kn = _p(nt), nt.shape[2]
     else:
         ntp, kn = None, 0
-    _load().oracle_step(_p(tokens), ld, _p(lengths), _p(reps), d, _p(query), ntp, kn, B,
-                        n_max, k, W, D, succ_len, float(tau), flags, nmax,
-                        _p(hit), _p(mn), _p(anchor), _p(cand), _p(score), _p(nc), _p(tok),
-                        _p(par), _p(pos), _p(mask), _p(nn), _p(stats))
+    if emb is not None:
+        E = _c(emb, np.uint16)
+        Ep, de = _p(E), E.shape[1]
+    else:
+        Ep, de = None, 0
+    _load().oracle_step_emb(_p(tokens), ld, _p(lengths), _p(reps), d, _p(query), Ep, de, ntp,
+                            kn, B, n_max, k, W, D, succ_len, float(tau), flags, nmax,
+                            _p(hit), _p(mn), _p(anchor), _p(cand), _p(score), _p(nc), _p(tok),
+                            _p(par), _p(pos), _p(mask), _p(nn), _p(stats))
     return StepResult(hit, mn, anchor, cand, score, nc, tok, par, pos, mask, nn, stats)

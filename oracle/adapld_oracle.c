@@ -173,6 +173,40 @@ int32_t oracle_semantic(const uint16_t *R, int32_t d, const uint16_t *q,
     return n;
 }
 
+/*
+ * Semantic fallback over token embeddings (Sec. 3.3, Eq. 4 as printed): every
+ * position j in [0, len-2] is scored by cos(E[M[j]], E[a]) with a = M[len-1]
+ * and E the caller's token-embedding table (rows de elements apart); rows
+ * with score >= tau are kept and the best min(k, count) are returned in
+ * (score desc, j desc) order.  Returns the number written.
+ */
+int32_t oracle_semantic_emb(const int32_t *M, int32_t len, const uint16_t *E, int32_t de,
+                            int32_t k, double tau, int32_t *cand, double *score)
+{
+    int32_t rows = len - 1;
+    if (rows <= 0)
+        return 0;
+    const uint16_t *ea = E + (int64_t)M[len - 1] * de;
+    scored_pos *all = (scored_pos *)malloc(sizeof(scored_pos) * (size_t)rows);
+    int32_t cnt = 0;
+    for (int32_t j = 0; j < rows; ++j) {
+        double s = oracle_cosine(E + (int64_t)M[j] * de, ea, de);
+        if (s >= tau) {
+            all[cnt].s = s;
+            all[cnt].j = j;
+            ++cnt;
+        }
+    }
+    qsort(all, (size_t)cnt, sizeof(scored_pos), cmp_scored);
+    int32_t n = cnt < k ? cnt : k;
+    for (int32_t i = 0; i < n; ++i) {
+        cand[i] = all[i].j;
+        score[i] = all[i].s;
+    }
+    free(all);
+    return n;
+}
+
 /* All Eq. 4 scores of one sequence, for the tests' tolerance checks. */
 void oracle_scores_all(const uint16_t *R, int32_t d, const uint16_t *q,
                        int32_t len, double *out)
@@ -226,6 +260,44 @@ int32_t oracle_successor_candidates(const int32_t *M, int32_t len,
 }
 
 /*
+ * Successor candidates with the lexical-first backoff of Sec. 3.5 applied to
+ * the branch token b: the k most recent lexical occurrences of b; if there
+ * are none and an embedding table E is given, the semantic fallback of
+ * Eq. 4 with b as the query anchor (positions t in [0, len-2] with
+ * cos(E[M[t]], E[b]) >= tau, best k by (score desc, t desc)).  Each is then
+ * scored by Eq. 13 against R[j*+1].  Returns the count.
+ */
+int32_t oracle_successor_candidates_emb(const int32_t *M, int32_t len, const uint16_t *R,
+                                        int32_t d, const uint16_t *E, int32_t de,
+                                        double tau, int32_t j_star, int32_t b, int32_t k,
+                                        int32_t *t_out, double *s_out)
+{
+    int32_t cnt = oracle_successor_candidates(M, len, R, d, j_star, b, k, t_out, s_out);
+    if (cnt > 0 || E == NULL || len < 2)
+        return cnt;
+    const uint16_t *eb = E + (int64_t)b * de;
+    scored_pos *all = (scored_pos *)malloc(sizeof(scored_pos) * (size_t)(len - 1));
+    int32_t m = 0;
+    for (int32_t t = 0; t + 1 < len; ++t) {
+        double s = oracle_cosine(E + (int64_t)M[t] * de, eb, de);
+        if (s >= tau) {
+            all[m].s = s;
+            all[m].j = t;
+            ++m;
+        }
+    }
+    qsort(all, (size_t)m, sizeof(scored_pos), cmp_scored);
+    const uint16_t *ref = R + (int64_t)(j_star + 1) * d;
+    for (int32_t i = 0; i < m && i < k; ++i) {
+        t_out[cnt] = all[i].j;
+        s_out[cnt] = oracle_cosine(R + (int64_t)all[i].j * d, ref, d);
+        ++cnt;
+    }
+    free(all);
+    return cnt;
+}
+
+/*
  * Draft-tree construction (Sec. 3.5 and Algorithm 1) from a retrieval
  * outcome and its ranked candidate list (cand[0] is j*).
  *
@@ -245,13 +317,14 @@ int32_t oracle_successor_candidates(const int32_t *M, int32_t len,
  *
  * Returns the number of branches that received at least one successor.
  */
-int32_t oracle_tree_from(const int32_t *M, int32_t len, const uint16_t *R,
-                         int32_t d, int32_t hit, const int32_t *cand,
-                         int32_t n_cand, const int32_t *topk_row, int32_t Kn,
-                         int32_t k, int32_t W, int32_t D, int32_t succ_len,
-                         uint32_t flags, int32_t nmax, int32_t *anchor,
-                         int32_t *tok, int32_t *par, int32_t *pos,
-                         uint8_t *mask, int32_t *n_nodes)
+int32_t oracle_tree_from_emb(const int32_t *M, int32_t len, const uint16_t *R,
+                             int32_t d, const uint16_t *E, int32_t de, double tau,
+                             int32_t hit, const int32_t *cand,
+                             int32_t n_cand, const int32_t *topk_row, int32_t Kn,
+                             int32_t k, int32_t W, int32_t D, int32_t succ_len,
+                             uint32_t flags, int32_t nmax, int32_t *anchor,
+                             int32_t *tok, int32_t *par, int32_t *pos,
+                             uint8_t *mask, int32_t *n_nodes)
 {
     int32_t *depth = (int32_t *)malloc(sizeof(int32_t) * (size_t)(nmax > 0 ? nmax : 1));
     int32_t n = 0;
@@ -323,8 +396,8 @@ int32_t oracle_tree_from(const int32_t *M, int32_t len, const uint16_t *R,
                 ++n;
                 if (!want_succ)
                     continue;
-                int32_t c = oracle_successor_candidates(M, len, R, d, js, br[e],
-                                                        k, tc, sc);
+                int32_t c = oracle_successor_candidates_emb(M, len, R, d, E, de, tau,
+                                                            js, br[e], k, tc, sc);
                 if (c == 0)
                     continue;
                 int32_t best = 0;
@@ -360,28 +433,51 @@ int32_t oracle_tree_from(const int32_t *M, int32_t len, const uint16_t *R,
     return succ_ext;
 }
 
+/* The draft tree of the single-cache reading (no embedding table). */
+int32_t oracle_tree_from(const int32_t *M, int32_t len, const uint16_t *R,
+                         int32_t d, int32_t hit, const int32_t *cand,
+                         int32_t n_cand, const int32_t *topk_row, int32_t Kn,
+                         int32_t k, int32_t W, int32_t D, int32_t succ_len,
+                         uint32_t flags, int32_t nmax, int32_t *anchor,
+                         int32_t *tok, int32_t *par, int32_t *pos,
+                         uint8_t *mask, int32_t *n_nodes)
+{
+    return oracle_tree_from_emb(M, len, R, d, NULL, 0, 0.0, hit, cand, n_cand, topk_row, Kn,
+                                k, W, D, succ_len, flags, nmax, anchor, tok, par, pos, mask,
+                                n_nodes);
+}
+
 /*
  * One full draft-construction step for B sequences laid out as the library
  * lays them out: tokens[B][ld], reps[B][ld][d], query[B][d],
- * next_topk[B][ld][Kn] (may be NULL).  Per sequence: Eq. 3 -> (if empty and
- * the fallback is on) Eq. 4 -> Eq. 5 -> Eq. 6-7 -> Eq. 8-15 -> tree.
+ * next_topk[B][ld][Kn] (may be NULL), and optionally a token-embedding table
+ * E[V][de] (may be NULL).  Per sequence: Eq. 3 -> (if empty and the fallback
+ * is on) Eq. 4 -> Eq. 5 -> Eq. 6-7 -> Eq. 8-15 -> tree.
+ *
+ * Without E the fallback scores the representation cache itself (the
+ * single-cache reading: row j against the query), and those scores are also
+ * the rerank scores.  With E the fallback scores token embeddings as Eq. 4
+ * prints it, cos(E[M[j]], E[a]), keeps the best k, and Eq. 6 then reranks
+ * them by cos(R[j], q); successor drafting backs off to the same embedding
+ * fallback for a branch token that never occurs (Sec. 3.5).
  *
  * Outputs per sequence b: hit[b], match_n[b], anchor[b], cand[b][k],
- * score[b][k] (padding -1 / 0), n_cand[b], tree arrays [b][nmax]
- * (mask [b][nmax][nmax]) and n_nodes[b]; stats[4] = lexical, semantic and
- * empty retrievals and successor extensions.  A sequence whose length is
- * outside [1, ld] gets hit NONE and n_nodes 0.  With NO_LEX_RERANK the
- * lexical scores are NaN (not computed).
+ * score[b][k] (the ranking scores; padding -1 / 0), n_cand[b], tree arrays
+ * [b][nmax] (mask [b][nmax][nmax]) and n_nodes[b]; stats[4] = lexical,
+ * semantic and empty retrievals and successor extensions.  A sequence whose
+ * length is outside [1, ld] gets hit NONE and n_nodes 0.  With
+ * NO_LEX_RERANK the lexical scores are NaN (not computed).
  */
-void oracle_step(const int32_t *tokens, int64_t ld, const int32_t *lengths,
-                 const uint16_t *reps, int32_t d, const uint16_t *query,
-                 const int32_t *next_topk, int32_t Kn, int32_t B,
-                 int32_t n_max, int32_t k, int32_t W, int32_t D,
-                 int32_t succ_len, double tau, uint32_t flags, int32_t nmax,
-                 int32_t *hit, int32_t *match_n, int32_t *anchor,
-                 int32_t *cand, double *score, int32_t *n_cand, int32_t *tok,
-                 int32_t *par, int32_t *pos, uint8_t *mask, int32_t *n_nodes,
-                 int64_t *stats)
+void oracle_step_emb(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                     const uint16_t *reps, int32_t d, const uint16_t *query,
+                     const uint16_t *E, int32_t de,
+                     const int32_t *next_topk, int32_t Kn, int32_t B,
+                     int32_t n_max, int32_t k, int32_t W, int32_t D,
+                     int32_t succ_len, double tau, uint32_t flags, int32_t nmax,
+                     int32_t *hit, int32_t *match_n, int32_t *anchor,
+                     int32_t *cand, double *score, int32_t *n_cand, int32_t *tok,
+                     int32_t *par, int32_t *pos, uint8_t *mask, int32_t *n_nodes,
+                     int64_t *stats)
 {
     for (int32_t s = 0; s < 4; ++s)
         stats[s] = 0;
@@ -422,16 +518,21 @@ void oracle_step(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                 oracle_rerank(R, d, q, cb, sb, nc);
             }
         } else if (!(flags & OR_NO_SEMANTIC)) {
-            nc = oracle_semantic(R, d, q, len, k, tau, cb, sb);
+            if (E != NULL) {
+                nc = oracle_semantic_emb(M, len, E, de, k, tau, cb, sb);
+                oracle_rerank(R, d, q, cb, sb, nc);
+            } else {
+                nc = oracle_semantic(R, d, q, len, k, tau, cb, sb);
+            }
             hit[b] = nc > 0 ? OR_SEM : OR_NONE;
         }
         n_cand[b] = nc;
         const int32_t *row = NULL;
         if (next_topk != NULL && nc > 0)
             row = next_topk + ((int64_t)b * ld + cb[0]) * Kn;
-        int32_t ext = oracle_tree_from(M, len, R, d, hit[b], cb, nc, row, Kn,
-                                       k, W, D, succ_len, flags, nmax,
-                                       &anchor[b], tb, pb, ob, mb, &n_nodes[b]);
+        int32_t ext = oracle_tree_from_emb(M, len, R, d, E, de, tau, hit[b], cb, nc, row, Kn,
+                                           k, W, D, succ_len, flags, nmax,
+                                           &anchor[b], tb, pb, ob, mb, &n_nodes[b]);
         if (hit[b] == OR_LEX)
             stats[0]++;
         else if (hit[b] == OR_SEM)
@@ -440,4 +541,20 @@ void oracle_step(const int32_t *tokens, int64_t ld, const int32_t *lengths,
             stats[2]++;
         stats[3] += ext;
     }
+}
+
+/* oracle_step_emb without an embedding table (the single-cache reading). */
+void oracle_step(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                 const uint16_t *reps, int32_t d, const uint16_t *query,
+                 const int32_t *next_topk, int32_t Kn, int32_t B,
+                 int32_t n_max, int32_t k, int32_t W, int32_t D,
+                 int32_t succ_len, double tau, uint32_t flags, int32_t nmax,
+                 int32_t *hit, int32_t *match_n, int32_t *anchor,
+                 int32_t *cand, double *score, int32_t *n_cand, int32_t *tok,
+                 int32_t *par, int32_t *pos, uint8_t *mask, int32_t *n_nodes,
+                 int64_t *stats)
+{
+    oracle_step_emb(tokens, ld, lengths, reps, d, query, NULL, 0, next_topk, Kn, B, n_max, k,
+                    W, D, succ_len, tau, flags, nmax, hit, match_n, anchor, cand, score,
+                    n_cand, tok, par, pos, mask, n_nodes, stats);
 }

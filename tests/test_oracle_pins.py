@@ -468,3 +468,98 @@ def test_semantic_threshold_is_inclusive():
     assert c == [2, 1] and s[1] == 0.6
     c, s = oracle.semantic(R, q, 4, 8, 0.0)
     assert c == [2, 1, 0] and s[2] == 0.0
+
+
+# ------------------------------------------------- token-embedding fallback
+def test_worked_example_embedding():
+    g = load_golden("worked_example_embedding.txt")
+    M = np.array(ints(g["tokens"]), np.int32)
+    L = len(M)
+    n_max, k, W, D, sl, d = (int(g[x][0]) for x in ("n_max", "k", "W", "D", "succ_len", "d"))
+    E = rows_to_bf16([[float(x) for x in g[f"emb{v}"]] for v in range(6)], d)
+    R = rows_to_bf16([[float(x) for x in g[f"row{i}"]] for i in range(L)], d)
+    q = rows_to_bf16([[float(x) for x in g["query"]]], d)[0]
+    res = oracle.step(M[None], [L], R[None], q[None], n_max, k, W, D, sl, float(g["tau"][0]),
+                      emb=E)
+    assert res.hit[0] == int(g["hit"][0]) == oracle.SEM
+    assert res.cand[0, : res.n_cand[0]].tolist() == ints(g["cand"])
+    np.testing.assert_allclose(res.score[0, : res.n_cand[0]], [float(x) for x in g["score"]],
+                               atol=1e-15)
+    assert res.anchor[0] == int(g["anchor"][0])
+    n = res.n_nodes[0]
+    assert res.tokens[0, :n].tolist() == ints(g["tree_tokens"])
+    assert res.parents[0, :n].tolist() == ints(g["tree_parents"])
+    assert res.positions[0, :n].tolist() == ints(g["tree_positions"])
+    single = oracle.step(M[None], [L], R[None], q[None], n_max, k, W, D, sl, 0.1)
+    assert single.cand[0, :2].tolist() == [2, 3]
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_embedding_fallback_reduces_to_single_cache(seed):
+    """All-distinct tokens with E = R (token v's embedding is row v) and the
+    query equal to the anchor's row make Eq. 4 over embeddings coincide with
+    the single-cache fallback, which is pinned above."""
+    rng = np.random.default_rng(700 + seed)
+    L, d, k = int(rng.integers(3, 80)), 16, 5
+    R = synth.f32_to_bf16_bits(rng.standard_normal((L, d)).astype(np.float32))
+    M = np.arange(L, dtype=np.int32)
+    q = R[L - 1]
+    for tau in (0.1, NEG_INF):
+        assert oracle.semantic_emb(M, L, R, k, tau) == oracle.semantic(R, q, L, k, tau)
+    # the steps agree up to successor drafting, which only the embedding mode
+    # can back off for a branch token with no earlier occurrence
+    a = oracle.step(M[None], [L], R[None], q[None], 3, k, 2, 4, 1, NEG_INF, oracle.NO_SUCC,
+                    emb=R)
+    b = oracle.step(M[None], [L], R[None], q[None], 3, k, 2, 4, 1, NEG_INF, oracle.NO_SUCC)
+    for name in ("hit", "cand", "score", "anchor", "tokens", "parents", "mask", "n_nodes"):
+        assert np.array_equal(getattr(a, name), getattr(b, name)), name
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_embedding_fallback_bruteforce(seed):
+    rng = np.random.default_rng(800 + seed)
+    V, L, de, k = int(rng.integers(3, 9)), int(rng.integers(2, 40)), 8, 4
+    M = rng.integers(0, V, size=L).astype(np.int32)
+    E = rows_to_bf16(rng.integers(-2, 3, size=(V, 3)).tolist(), de)
+    Ef = synth.bf16_bits_to_f32(E).astype(np.float64)
+    ea = Ef[M[-1]]
+    s = np.array([Ef[v] @ ea / (np.linalg.norm(Ef[v]) * np.linalg.norm(ea))
+                  if np.linalg.norm(Ef[v]) * np.linalg.norm(ea) > 0 else 0.0 for v in M[:-1]])
+    j = np.arange(L - 1)
+    for tau in (0.1, NEG_INF):
+        keep = np.flatnonzero(s >= tau)
+        order = keep[np.lexsort((-j[keep], -s[keep]))][:k]
+        c, sc = oracle.semantic_emb(M, L, E, k, tau)
+        assert c == order.tolist()
+        np.testing.assert_allclose(sc, s[order], atol=1e-12)
+
+
+@pytest.mark.parametrize("seed", range(20))
+def test_successor_backoff_bruteforce(seed):
+    """A branch token that never occurs earlier backs off to the embedding
+    fallback with the branch token as the query anchor (Sec. 3.5)."""
+    rng = np.random.default_rng(900 + seed)
+    V, L, d, k = 8, int(rng.integers(4, 30)), 8, 3
+    M = rng.integers(0, V - 2, size=L).astype(np.int32)   # tokens V-2, V-1 never occur
+    E = rows_to_bf16(rng.integers(-2, 3, size=(V, 3)).tolist(), d)
+    R = rows_to_bf16(rng.integers(-2, 3, size=(L, 3)).tolist(), d)
+    js = int(rng.integers(0, L - 1))
+    Ef = synth.bf16_bits_to_f32(E).astype(np.float64)
+    Rf = synth.bf16_bits_to_f32(R).astype(np.float64)
+
+    def cos(x, y):
+        n = np.linalg.norm(x) * np.linalg.norm(y)
+        return float(x @ y / n) if n > 0 else 0.0
+
+    for b in (V - 1, int(M[0])):
+        occ = [t for t in range(L - 2, -1, -1) if M[t] == b][:k]
+        if not occ:
+            es = [(cos(Ef[M[t]], Ef[b]), t) for t in range(L - 1)]
+            es = [x for x in es if x[0] >= 0.1]
+            occ = [t for _, t in sorted(es, key=lambda x: (-x[0], -x[1]))[:k]]
+        exp_s = [cos(Rf[t], Rf[js + 1]) for t in occ]
+        t, sc = oracle.successor_candidates_emb(M, L, R, d, E, 0.1, js, b, k)
+        assert t == occ
+        np.testing.assert_allclose(sc, exp_s, atol=1e-12)
+    # without a table a token that never occurs has no successor candidates
+    assert oracle.successor_candidates(M, L, R, d, js, V - 1, k) == ([], [])
