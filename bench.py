@@ -41,6 +41,8 @@ def parse():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--config", type=int, default=5)
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--embeddings", action="store_true",
+                    help="two-representation mode: token-embedding fallback (vocab x d table)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override B (profiling of small cases; not the headline workload)")
     ap.add_argument("--e2e-steps", type=int, default=5)
@@ -287,9 +289,12 @@ def run_native(args):
     p = native.make_params(w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, 0)
     eng = native.Engine(w.B, w.ld, w.d, p, device=dev)
     stream = torch.cuda.current_stream(dev)
+    emb = None
+    if args.embeddings:
+        emb = synth.make_embeddings(w, synth.CONFIGS[cfg]["V"], w.d, rank_seed(args.seed, rank))
 
     for _ in range(max(3, args.warmup)):
-        eng.run(w.tokens, w.lengths, w.reps, w.query)
+        eng.run(w.tokens, w.lengths, w.reps, w.query, emb=emb)
     torch.cuda.synchronize(dev)
     if native.read_device_status(eng.ws) != 0:
         raise RuntimeError("device status raised during warm-up")
@@ -317,7 +322,7 @@ def run_native(args):
         time.sleep(0.3)
     start.record(stream)
     for i in range(K):
-        native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws)
+        native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws, emb=emb)
     end.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
@@ -327,7 +332,7 @@ def run_native(args):
     startb.record(stream)
     for i in range(K):
         native.step(w.tokens, w.lengths, w.reps, w.query, p, eng.out, eng.ws,
-                    events=native.StepEvents(*[e.cuda_event for e in ev[i]]))
+                    events=native.StepEvents(*[e.cuda_event for e in ev[i]]), emb=emb)
     endb.record(stream)
     torch.cuda.synchronize(dev)
     barrier()
@@ -344,7 +349,7 @@ def run_native(args):
 
     # end-to-end through the public API from pinned host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and emb is None:
         tok_h = w.tokens.cpu().pin_memory()
         len_h = w.lengths.cpu().pin_memory()
         reps_h = torch.empty(w.reps.shape, dtype=w.reps.dtype, pin_memory=True)
@@ -388,6 +393,9 @@ def run_native(args):
         cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample.desc}
     hk = g["hit_kind"]
     conf = workload_config(cfg)
+    if emb is not None:
+        conf["workload"] += (f" + token-embedding fallback ({emb.shape[0]} x {emb.shape[1]} "
+                             "table; two-representation mode)")
     if args.batch is not None:
         conf["workload"] += f" (resized: B={w.B})"
         conf["B"] = conf["global_batch"] = w.B
@@ -403,7 +411,7 @@ def run_native(args):
         "roofline": {"bound": "hbm", "kernel": "semantic_kernel",
                      "achieved": achieved, "peak": peak, "peak_kind": peak_kind,
                      "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": semantic_traffic(nbytes["semantic"]),
+                     "traffic": semantic_traffic(nbytes["semantic"]) if emb is None else None,
                      "algorithmic_bytes": nbytes["semantic"], "avg_launch_ms": sem_avg_ms},
         "step_hbm": {"achieved": step_gbs, "frac": step_gbs / peak,
                      "algorithmic_bytes": nbytes["step"]},
@@ -411,7 +419,7 @@ def run_native(args):
         "ms_per_step_with_stage_events": total_b_ms / K,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 4 * K,
+        "gpu_launches": (6 if emb is not None else 4) * K,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

@@ -71,6 +71,9 @@ typedef struct CUstream_st *adapld_stream_t;
 #define ADAPLD_ERR_TAU (-14)          /* tau is NaN                            */
 #define ADAPLD_ERR_STATIC_LIMIT (-15) /* B > ADAPLD_STATIC_MAX_B for the
                                          workspace-free entry point           */
+#define ADAPLD_ERR_EMBEDDINGS (-16)   /* embedding table NULL or misaligned,
+                                         vocab < 1, or dim not a multiple of 8
+                                         in [8, 16384]                        */
 #define ADAPLD_ERR_CUDA (-20)         /* a CUDA runtime call failed            */
 
 /* ---- retrieval outcome per sequence (Eq. 5, Algorithm 1) ------------------- */
@@ -83,6 +86,8 @@ typedef struct CUstream_st *adapld_stream_t;
 #define ADAPLD_SEQ_BAD_CANDIDATE 2 /* adapld_build_draft_tree() was given a
                                       candidate outside [0, len_b-2]: the
                                       sequence is treated as retrieving nothing */
+#define ADAPLD_SEQ_BAD_TOKEN 4 /* a token id outside [0, vocab) met the
+                                  embedding table: row 0 was used instead */
 
 /* ---- device status bits (adapld_read_device_status) ------------------------ */
 #define ADAPLD_DEV_TIMEOUT 1  /* a bounded wait in a kernel expired; that
@@ -178,6 +183,20 @@ typedef struct adapld_step_out {
     adapld_tree_out tree;
 } adapld_step_out;
 
+/*
+ * Token-embedding table of the target model, for the two-representation mode
+ * (Sec. 3.3, Eq. 4 as printed: the fallback compares token embeddings
+ * e_{M_j} with e_a; the hidden-state cache then reranks the candidates,
+ * Eq. 6).  table: [vocab][dim] bf16 bits, 16-byte aligned, dim a multiple of 8
+ * in [8, 16384].  Token ids outside [0, vocab) read row 0 and raise
+ * ADAPLD_SEQ_BAD_TOKEN for their sequence.
+ */
+typedef struct adapld_embeddings {
+    const uint16_t *table;
+    int32_t vocab;
+    int32_t dim;
+} adapld_embeddings;
+
 /* Optional CUDA events recorded around each kernel of adapld_step_ex(), for
  * timing a single stage inside a step.  Any member may be NULL.  The events
  * are cudaEvent_t handles, passed as void*. */
@@ -250,14 +269,34 @@ int adapld_semantic_topk(const uint16_t *reps, int64_t ld, int32_t d, const uint
  * recent positions t <= len-2 holding b, pick the one maximising
  * cos(R[t], R[j*+1]) and append tokens[t+1 .. t+succ_len] (clipped at
  * len-1).
- * status [B] may be NULL.
+ * emb (nullable) selects the two-representation mode: semantic hits are
+ * reranked by Eq. 6 as well, and a branch token that never occurs backs off
+ * to the embedding fallback with the branch token as the anchor (Sec. 3.5).
+ * status [B] may be NULL; its ADAPLD_SEQ_BAD_TOKEN bit is kept, the others
+ * are overwritten.
  */
 int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                             const uint16_t *reps, int32_t d, const uint16_t *query, int32_t B,
                             const int32_t *hit_kind, int32_t *cand, float *score,
                             const int32_t *n_cand, const int32_t *next_topk, int32_t Kn,
-                            const adapld_params *p, const adapld_tree_out *out, int32_t *status,
-                            void *ws, size_t ws_bytes, adapld_stream_t stream);
+                            const adapld_embeddings *emb, const adapld_params *p,
+                            const adapld_tree_out *out, int32_t *status, void *ws,
+                            size_t ws_bytes, adapld_stream_t stream);
+
+/*
+ * Semantic fallback over token embeddings (Sec. 3.3, Eq. 4 as printed).
+ * For every selected sequence (active == NULL selects all) with a valid
+ * length: score(j) = cos(E[tokens[j]], E[tokens[len-1]]) for every j in
+ * [0, len-2]; rows with score >= tau are kept and the best min(k, count) by
+ * (score desc, j desc) are written to cand / score, n_cand[b] = count (the
+ * hidden-state rerank of Eq. 6 is adapld_build_draft_tree's).  Unselected
+ * rows are left untouched.  status [B] (nullable) receives
+ * ADAPLD_SEQ_BAD_TOKEN for a token id outside the table.
+ */
+int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                          const adapld_embeddings *emb, const uint8_t *active, int32_t B,
+                          int32_t k, float tau, int32_t *cand, float *score, int32_t *n_cand,
+                          int32_t *status, void *ws, size_t ws_bytes, adapld_stream_t stream);
 
 /*
  * One full draft-construction step for B sequences: lexical anchoring, the
@@ -271,12 +310,21 @@ int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const
                 const adapld_params *p, const adapld_step_out *out, void *ws, size_t ws_bytes,
                 adapld_stream_t stream);
 
-/* adapld_step() that also records the given CUDA events around its kernels. */
+/*
+ * adapld_step() with two options.  emb (nullable) selects the
+ * two-representation mode: the fallback scores token embeddings (Eq. 4 as
+ * printed), semantic candidates are reranked by the hidden states (Eq. 6),
+ * and successor drafting backs off to the embedding fallback for a branch
+ * token that never occurs (Sec. 3.5); cand / score then hold the reranked
+ * candidates and their Eq. 6 scores.  events (nullable) are CUDA events
+ * recorded around the step's kernels.
+ */
 int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                    const uint16_t *reps, int32_t d, const uint16_t *query,
                    const int32_t *next_topk, int32_t Kn, int32_t B, const adapld_params *p,
                    const adapld_step_out *out, void *ws, size_t ws_bytes,
-                   const adapld_step_events *events, adapld_stream_t stream);
+                   const adapld_embeddings *emb, const adapld_step_events *events,
+                   adapld_stream_t stream);
 
 /*
  * adapld_semantic_topk_static(): adapld_semantic_topk() for callers that cannot

@@ -44,6 +44,13 @@ int check_ws(void *ws, size_t ws_bytes, int32_t B, int64_t ld, int32_t W) {
     return ADAPLD_OK;
 }
 
+int check_emb(const adapld_embeddings *e) {
+    if (!e) return ADAPLD_OK;
+    if (!e->table || !aligned16(e->table) || e->vocab < 1) return ADAPLD_ERR_EMBEDDINGS;
+    if (e->dim < 8 || e->dim > 16384 || (e->dim % 8) != 0) return ADAPLD_ERR_EMBEDDINGS;
+    return ADAPLD_OK;
+}
+
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA; }
 
 int record(void *ev, cudaStream_t s) {
@@ -90,6 +97,7 @@ const char *adapld_status_string(int code) {
         case ADAPLD_ERR_TOPK_TABLE: return "next_topk needs Kn in [1, 64]";
         case ADAPLD_ERR_TAU: return "tau must not be NaN";
         case ADAPLD_ERR_STATIC_LIMIT: return "B exceeds ADAPLD_STATIC_MAX_B (1024) for the workspace-free entry point";
+        case ADAPLD_ERR_EMBEDDINGS: return "embedding table NULL or misaligned, vocab < 1, or dim not a multiple of 8 in [8, 16384]";
         case ADAPLD_ERR_CUDA: return "a CUDA runtime call failed";
         default: return "unknown status";
     }
@@ -131,12 +139,34 @@ int adapld_semantic_topk(const uint16_t *reps, int64_t ld, int32_t d, const uint
     return cuda_status(launch_semantic(a, w, s));
 }
 
+int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                          const adapld_embeddings *emb, const uint8_t *active, int32_t B,
+                          int32_t k, float tau, int32_t *cand, float *score, int32_t *n_cand,
+                          int32_t *status, void *ws, size_t ws_bytes, adapld_stream_t stream) {
+    if (!tokens || !lengths || !emb || !cand || !score || !n_cand) return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_emb(emb));
+    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
+    if (std::isnan(tau)) return ADAPLD_ERR_TAU;
+    ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
+    cudaStream_t s = (cudaStream_t)stream;
+    Workspace w = layout_workspace(ws, B, ld, 1);
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    SemLaunch a{emb->table, ld, emb->dim, nullptr, lengths, active, B, k, tau, cand, score, n_cand,
+                nullptr, false};
+    a.tokens = tokens;
+    a.vocab = emb->vocab;
+    a.status = status;
+    return cuda_status(launch_semantic(a, w, s));
+}
+
 int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                             const uint16_t *reps, int32_t d, const uint16_t *query, int32_t B,
                             const int32_t *hit_kind, int32_t *cand, float *score,
                             const int32_t *n_cand, const int32_t *next_topk, int32_t Kn,
-                            const adapld_params *p, const adapld_tree_out *out, int32_t *status,
-                            void *ws, size_t ws_bytes, adapld_stream_t stream) {
+                            const adapld_embeddings *emb, const adapld_params *p,
+                            const adapld_tree_out *out, int32_t *status, void *ws,
+                            size_t ws_bytes, adapld_stream_t stream) {
     if (!tokens || !lengths || !reps || !query || !hit_kind || !cand || !score || !n_cand || !out)
         return ADAPLD_ERR_NULL;
     if (!out->anchor || !out->draft_tokens || !out->parents || !out->positions || !out->mask ||
@@ -147,12 +177,14 @@ int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *le
     ADAPLD_TRY(check_dim(d));
     if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
     if (next_topk && (Kn < 1 || Kn > kMaxW)) return ADAPLD_ERR_TOPK_TABLE;
+    ADAPLD_TRY(check_emb(emb));
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, p->branch_width));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
     TreeLaunch a{tokens, ld, lengths, reps, d, query, B, hit_kind, cand, score, n_cand,
                  next_topk, next_topk ? Kn : 0, *p, *out, status};
+    if (emb) a.emb = *emb;
     return cuda_status(launch_tree(a, w, s));
 }
 
@@ -160,7 +192,8 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                    const uint16_t *reps, int32_t d, const uint16_t *query,
                    const int32_t *next_topk, int32_t Kn, int32_t B, const adapld_params *p,
                    const adapld_step_out *out, void *ws, size_t ws_bytes,
-                   const adapld_step_events *ev, adapld_stream_t stream) {
+                   const adapld_embeddings *emb, const adapld_step_events *ev,
+                   adapld_stream_t stream) {
     if (!tokens || !lengths || !reps || !query || !out) return ADAPLD_ERR_NULL;
     if (!out->hit_kind || !out->match_n || !out->cand || !out->score || !out->n_cand)
         return ADAPLD_ERR_NULL;
@@ -172,6 +205,7 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
     ADAPLD_TRY(check_dim(d));
     if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
     if (next_topk && (Kn < 1 || Kn > kMaxW)) return ADAPLD_ERR_TOPK_TABLE;
+    ADAPLD_TRY(check_emb(emb));
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, p->branch_width));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
@@ -188,6 +222,14 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
         ADAPLD_TRY(record(ev ? ev->semantic_begin : nullptr, s));
         SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
                      out->n_cand, out->hit_kind, true};
+        if (emb) {  // Eq. 4 over token embeddings
+            sa.reps = emb->table;
+            sa.d = emb->dim;
+            sa.query = nullptr;
+            sa.tokens = tokens;
+            sa.vocab = emb->vocab;
+            sa.status = out->status;
+        }
         ADAPLD_TRY(cuda_status(launch_semantic(sa, w, s)));
         ADAPLD_TRY(record(ev ? ev->semantic_end : nullptr, s));
     }
@@ -195,6 +237,7 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
     ADAPLD_TRY(record(ev ? ev->tree_begin : nullptr, s));
     TreeLaunch ta{tokens, ld, lengths, reps, d, query, B, out->hit_kind, out->cand, out->score,
                   out->n_cand, next_topk, next_topk ? Kn : 0, *p, to, out->status};
+    if (emb) ta.emb = *emb;
     ADAPLD_TRY(cuda_status(launch_tree(ta, w, s)));
     return record(ev ? ev->tree_end : nullptr, s);
 }
@@ -204,7 +247,7 @@ int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const
                 const adapld_params *p, const adapld_step_out *out, void *ws, size_t ws_bytes,
                 adapld_stream_t stream) {
     return adapld_step_ex(tokens, ld, lengths, reps, d, query, next_topk, Kn, B, p, out, ws,
-                          ws_bytes, nullptr, stream);
+                          ws_bytes, nullptr, nullptr, stream);
 }
 
 int adapld_read_device_status(const void *ws, int32_t *status, adapld_stream_t stream) {

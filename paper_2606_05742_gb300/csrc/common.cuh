@@ -34,6 +34,9 @@ struct Workspace {
     int32_t *done2;          // [B]  semantic kernel: CTAs done per sequence
     int32_t *ticket4;        // [B]  successor scan: slices done per sequence
     int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
+    int32_t *npairs;         // [1]  successor backoff: (sequence, branch) pairs
+    int32_t *gticket4;       // [1]  successor scan: sequences done
+    int32_t *done3;          // [B*W] successor backoff: CTAs done per pair
     int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
     int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
     int32_t *slots2;         // [B + kMaxGrid2][kSlotInts] partial top-k lists
@@ -43,6 +46,12 @@ struct Workspace {
     int32_t *rr_cand;        // [B][kMaxK] reranked lexical candidates (successor scan)
     float *rr_score;         // [B][kMaxK] their scores
     float *score5;           // [B][W*kMaxK] scores computed by the tree kernel
+    int64_t *plan3;          // [B*W+1] successor backoff plan
+    int32_t *slots3;         // [B*W + kMaxGrid2][kSlotInts] its partial lists
+    int32_t *pair_b;         // [B*W] real sequence of each backoff pair
+    int32_t *pair_tok;       // [B*W] its branch token (the query anchor)
+    int32_t *pair_out;       // [B*W] its row b*W + w in succ / succ_n
+    float *succ_es;          // [B*W][kMaxK] backoff candidates' embedding scores
     size_t counters_bytes;
     size_t total_bytes;
     int C1, S4, W;
@@ -67,15 +76,19 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         off = align_up(off + bytes, 256);
         return r;
     };
-    w.dev_status = (int32_t *)take(sizeof(int32_t) * (2 + 4 * (size_t)B));
+    const size_t BW = (size_t)B * w.W;
+    w.counters_bytes = sizeof(int32_t) * (4 + 4 * (size_t)B + BW);
+    w.dev_status = (int32_t *)take(w.counters_bytes);
     if (p) {
         w.global_ticket = w.dev_status + 1;
-        w.ticket1 = w.dev_status + 2;
+        w.npairs = w.dev_status + 2;
+        w.gticket4 = w.dev_status + 3;
+        w.ticket1 = w.dev_status + 4;
         w.done2 = w.ticket1 + B;
         w.ticket4 = w.done2 + B;
         w.ticket5 = w.ticket4 + B;
+        w.done3 = w.ticket5 + B;
     }
-    w.counters_bytes = sizeof(int32_t) * (2 + 4 * (size_t)B);
     w.part1 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1 * kPart1Ints);
     w.plan = (int64_t *)take(sizeof(int64_t) * ((size_t)B + 1));
     w.slots2 = (int32_t *)take(sizeof(int32_t) * ((size_t)B + kMaxGrid2) * kSlotInts);
@@ -85,6 +98,12 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.rr_cand = (int32_t *)take(sizeof(int32_t) * (size_t)B * kMaxK);
     w.rr_score = (float *)take(sizeof(float) * (size_t)B * kMaxK);
     w.score5 = (float *)take(sizeof(float) * (size_t)B * w.W * kMaxK);
+    w.plan3 = (int64_t *)take(sizeof(int64_t) * (BW + 1));
+    w.slots3 = (int32_t *)take(sizeof(int32_t) * (BW + kMaxGrid2) * kSlotInts);
+    w.pair_b = (int32_t *)take(sizeof(int32_t) * BW);
+    w.pair_tok = (int32_t *)take(sizeof(int32_t) * BW);
+    w.pair_out = (int32_t *)take(sizeof(int32_t) * BW);
+    w.succ_es = (float *)take(sizeof(float) * BW * kMaxK);
     w.total_bytes = off;
     return w;
 }
@@ -175,6 +194,12 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
 __device__ __forceinline__ uint64_t l2_evict_first_policy() {
     uint64_t pol;
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+    return pol;
+}
+
+__device__ __forceinline__ uint64_t l2_evict_normal_policy() {
+    uint64_t pol;
+    asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(pol));
     return pol;
 }
 
@@ -351,11 +376,25 @@ struct SemLaunch {
     int32_t *n_cand;
     int32_t *hit_kind;       // step path: set SEM / NONE at the final merge
     bool plan_ready;         // step path: the lexical kernel built the plan
+    // token-embedding rows (Eq. 4 as printed): `reps` is then the embedding
+    // table [vocab][d] and row j of sequence b is reps[tokens[b*ld + j]]
+    const int32_t *tokens = nullptr;
+    int32_t vocab = 0;
+    // virtual sequences (successor backoff): sequence p scores the positions
+    // of real sequence vseq_b[p] against reps[vseq_tok[p]] and writes row
+    // vseq_out[p] of cand / score (row stride out_stride) and n_cand; their
+    // count is *nvseq; plan, slots and counters come from the backoff part
+    // of the workspace
+    const int32_t *vseq_b = nullptr, *vseq_tok = nullptr, *vseq_out = nullptr;
+    const int32_t *nvseq = nullptr;
+    int32_t out_stride = 0;  // 0: k
+    int32_t *status = nullptr;  // per real sequence ADAPLD_SEQ_* bits (nullable)
 };
 cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_t s);
 
 struct TreeLaunch {
     const int32_t *tokens;
+    // (the token-embedding table, when given, is the last member)
     int64_t ld;
     const int32_t *lengths;
     const uint16_t *reps;
@@ -371,6 +410,7 @@ struct TreeLaunch {
     adapld_params p;
     adapld_tree_out out;
     int32_t *status;
+    adapld_embeddings emb = {nullptr, 0, 0};  // token embeddings (two-representation mode)
 };
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s);
 

@@ -49,7 +49,27 @@ struct SemArgs {
     int stage_bytes;
     uint64_t wait_limit_ns;  // bound of every mbarrier wait
     int stall;               // test switch: the producer issues no copy
+    const int64_t *plan;     // row prefix sums over the (virtual) sequences
+    int32_t *done;           // per-sequence count of CTAs that published
+    int32_t *slots;          // partial top-k lists
 };
+
+// The real sequence, the query token and the output row of (virtual)
+// sequence p.
+__device__ __forceinline__ int real_seq(const SemLaunch &a, int p) {
+    return a.vseq_b ? a.vseq_b[p] : p;
+}
+__device__ __forceinline__ int out_row(const SemLaunch &a, int p) {
+    return a.vseq_out ? a.vseq_out[p] : p;
+}
+
+// Token id of position j of real sequence b, clamped into the table (an
+// out-of-range id reads row 0 and marks the sequence).
+__device__ __forceinline__ int table_row(const SemLaunch &a, int b, int tok) {
+    if (tok >= 0 && tok < a.vocab) return tok;
+    if (a.status) atomicOr(a.status + b, ADAPLD_SEQ_BAD_TOKEN);
+    return 0;
+}
 
 // Reduce-scatter of N values across a warp (N a power of two <= 32): after
 // the call, lanes with lane % (32/N) == 0 hold in v[0] the warp total of
@@ -129,7 +149,7 @@ constexpr int semantic_min_blocks() {
     return MAXC * (SR * 4 + 8) > 72 ? 1 : 2;
 }
 
-template <int MAXC, int SR>
+template <int MAXC, int SR, bool GATHER>
 __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, SR>()))
     semantic_kernel(SemArgs args) {
     const SemLaunch &a = args.p;
@@ -148,8 +168,10 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     pdl_wait_then_release();  // the plan and the lexical outcomes come from the previous kernel
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
     const int grid = gridDim.x, c = blockIdx.x;
-    const int B = a.B, d = a.d, k = a.k;
-    const int64_t *plan = ws.plan;
+    const int B = a.nvseq ? *a.nvseq : a.B, d = a.d, k = a.k;
+    const int ostride = a.out_stride ? a.out_stride : k;
+    if (B <= 0) return;
+    const int64_t *plan = args.plan;
     const int64_t G = plan[B];
     if (G < 0 || G > (int64_t)B * a.ld) {  // never expected: the plan is corrupt
         if (t == 0 && c == 0) atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
@@ -174,41 +196,71 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
 
     // ------------------------------------------------------------ producer
     if (warp == kProducerWarp) {
-        if (lane != 0) return;
-        const uint64_t pol = l2_evict_first_policy();
+        // Gathered rows need their token ids: the whole warp keeps a window
+        // of 32 upcoming ids; lane 0 issues the copies.
+        if (!GATHER && lane != 0) return;
+        // streamed cache rows are read once; embedding rows of frequent
+        // tokens come back, so they stay ordinary L2 citizens
+        const uint64_t pol = GATHER ? l2_evict_normal_policy() : l2_evict_first_policy();
         int it = 0;
         bool failed = false;
-        int b = b_first;
+        int p = b_first;
         int64_t g = g0;
         while (g < g1 && !failed) {
-            while (b < B - 1 && plan[b + 1] <= g) ++b;
-            const int64_t seg_end = min(plan[b + 1], g1);
+            while (p < B - 1 && plan[p + 1] <= g) ++p;
+            const int64_t seg_end = min(plan[p + 1], g1);
             if (seg_end <= g) {  // never expected: a corrupt plan
-                atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
+                if (lane == 0) atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
                 break;
             }
-            const int jend = (int)(seg_end - plan[b]);
+            const int b = real_seq(a, p);
+            const int jend = (int)(seg_end - plan[p]);
             const uint8_t *base = (const uint8_t *)(a.reps + (int64_t)b * a.ld * d);
-            for (int j = (int)(g - plan[b]); j < jend; j += SR) {
+            const int32_t *Mb = GATHER ? a.tokens + (int64_t)b * a.ld : nullptr;
+            int win = -1, wtok = 0;
+            for (int j = (int)(g - plan[p]); j < jend; j += SR) {
                 const int nrows = min(SR, jend - j);
                 const int s = it % NS, r = it / NS;
-                if (r > 0 && !mbar_wait_bounded(&empty[s], (r - 1) & 1, args.wait_limit_ns)) {
-                    failed = true;
-                    break;
+                int ok = 1;
+                if (lane == 0) {
+                    if (r > 0 && !mbar_wait_bounded(&empty[s], (r - 1) & 1, args.wait_limit_ns))
+                        ok = 0;
+                    if (*abort_flag || args.stall) ok = 0;
                 }
-                if (*abort_flag || args.stall) {
+                if (GATHER) ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) {
                     failed = true;
                     break;
                 }
                 const uint32_t bytes = (uint32_t)(nrows * row_bytes);
-                mbar_arrive_expect_tx(&full[s], bytes);
-                bulk_g2s(ring + (size_t)s * stage_bytes, base + (size_t)j * row_bytes, bytes,
-                         &full[s], pol);
+                uint8_t *dst = ring + (size_t)s * stage_bytes;
+                if (GATHER) {
+                    if (win < 0 || j + nrows > win + 32) {
+                        win = j;
+                        wtok = j + lane < jend ? Mb[j + lane] : 0;
+                    }
+                    int rowtok[SR];
+#pragma unroll
+                    for (int rr = 0; rr < SR; ++rr)
+                        rowtok[rr] = __shfl_sync(0xffffffffu, wtok, (j - win + rr) & 31);
+                    if (lane == 0) {
+                        mbar_arrive_expect_tx(&full[s], bytes);
+#pragma unroll
+                        for (int rr = 0; rr < SR; ++rr)
+                            if (rr < nrows)
+                                bulk_g2s(dst + (size_t)rr * row_bytes,
+                                         a.reps + (int64_t)table_row(a, b, rowtok[rr]) * d,
+                                         (uint32_t)row_bytes, &full[s], pol);
+                    }
+                } else {
+                    mbar_arrive_expect_tx(&full[s], bytes);
+                    bulk_g2s(dst, base + (size_t)j * row_bytes, bytes, &full[s], pol);
+                }
                 ++it;
             }
             g = seg_end;
         }
-        if (failed) {
+        if (failed && lane == 0) {
             *abort_flag = 1;
             atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
             // drain the copies still in flight before the CTA may exit
@@ -228,19 +280,27 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     tk.reset();
     bool aborted = false;
     int it = 0, segno = 0;
-    int b = b_first;
+    int p = b_first;
     int64_t g = g0;
     const float tau = a.tau;
     while (g < g1) {
-        while (b < B - 1 && plan[b + 1] <= g) ++b;
-        const int64_t seg_end = min(plan[b + 1], g1);
+        while (p < B - 1 && plan[p + 1] <= g) ++p;
+        const int64_t seg_end = min(plan[p + 1], g1);
         if (seg_end <= g) break;  // never expected: a corrupt plan (flagged by the producer)
-        const int jbeg = (int)(g - plan[b]);
-        const int jend = (int)(seg_end - plan[b]);
+        const int jbeg = (int)(g - plan[p]);
+        const int jend = (int)(seg_end - plan[p]);
 
         // query slice of this sequence (registers) and |q|^2
         float qpart = 0.f;
-        const uint16_t *q = a.query + (int64_t)b * d;
+        const uint16_t *q;
+        if (GATHER) {
+            const int b = real_seq(a, p);
+            const int qt = a.vseq_tok ? a.vseq_tok[p]
+                                      : a.tokens[(int64_t)b * a.ld + a.lengths[b] - 1];
+            q = a.reps + (int64_t)table_row(a, b, qt) * d;
+        } else {
+            q = a.query + (int64_t)p * d;
+        }
 #pragma unroll
         for (int cc = 0; cc < MAXC; ++cc) {
             const uint4 w = colok[cc] ? ldg_nc_v4(q + (t + kConsumers2 * cc) * 8)
@@ -336,13 +396,13 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
 
         // ---- end of this CTA's segment of sequence b: publish; the CTA that
         // publishes last for b merges every partial list, with all 8 warps
-        const int cfirst = cta_of(plan[b], G, grid);
-        const int clast = cta_of(plan[b + 1] - 1, G, grid);
+        const int cfirst = cta_of(plan[p], G, grid);
+        const int clast = cta_of(plan[p + 1] - 1, G, grid);
         volatile int *s_flag = (volatile int *)abort_flag + 1;  // the merge decision
         if (warp == 0) {
             int last = 0;
             if (!aborted && !*abort_flag) {
-                int32_t *sp = ws.slots2 + (int64_t)(b + c) * kSlotInts;
+                int32_t *sp = args.slots + (int64_t)(p + c) * kSlotInts;
                 if (lane == 0) sp[0] = tk.n;
                 if (lane < tk.n) {
                     sp[1 + lane] = tk.j;
@@ -355,7 +415,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
                     expected = 0;
                     for (int cc = cfirst; cc <= clast; ++cc) expected += cta_nonempty(cc, G, grid);
                 }
-                if (lane == 0) last = atomicAdd(ws.done2 + b, 1) == expected - 1;
+                if (lane == 0) last = atomicAdd(args.done + p, 1) == expected - 1;
                 last = __shfl_sync(0xffffffffu, last, 0);
             }
             if (lane == 0) *s_flag = last;
@@ -375,7 +435,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
                 for (int u = 0; u < 4; ++u) {
                     const int cc = cc0 + u;
                     const bool ok = cc <= clast && cta_nonempty(cc, G, grid);
-                    const int32_t *op = ws.slots2 + (int64_t)(b + (ok ? cc : c)) * kSlotInts;
+                    const int32_t *op = args.slots + (int64_t)(p + (ok ? cc : c)) * kSlotInts;
                     n[u] = ok ? __ldcg(op) : 0;
                     xj[u] = ok ? __ldcg(op + 1 + lane) : -1;
                     xs[u] = ok ? __int_as_float(__ldcg(op + 1 + kMaxK + lane)) : 0.f;
@@ -395,13 +455,14 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
                 f.reset();
                 for (int w = 0; w < 8; ++w)
                     f.insert(lane < wl_n[w], wl_s[w * 32 + lane], wl_j[w * 32 + lane], k);
+                const int64_t orow = out_row(a, p);
                 if (lane < k) {
-                    a.cand[(int64_t)b * k + lane] = lane < f.n ? f.j : -1;
-                    a.score[(int64_t)b * k + lane] = lane < f.n ? f.s : 0.f;
+                    a.cand[orow * ostride + lane] = lane < f.n ? f.j : -1;
+                    a.score[orow * ostride + lane] = lane < f.n ? f.s : 0.f;
                 }
                 if (lane == 0) {
-                    a.n_cand[b] = f.n;
-                    if (a.hit_kind) a.hit_kind[b] = f.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
+                    a.n_cand[orow] = f.n;
+                    if (a.hit_kind) a.hit_kind[orow] = f.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
                 }
             }
             named_bar_sync(kBarMerge, kConsumers2);  // before red is reused by the next stage
@@ -419,11 +480,11 @@ inline size_t semantic_smem(int ns, int stage) {
            3 * kMaxStages2 * 8 + 16;
 }
 
-template <int MAXC, int SR>
+template <int MAXC, int SR, bool GATHER>
 cudaError_t launch_variant(const SemArgs &args0, int sms, int ctas_per_sm, int stages,
                            cudaStream_t s) {
     SemArgs args = args0;
-    auto kern = semantic_kernel<MAXC, SR>;
+    auto kern = semantic_kernel<MAXC, SR, GATHER>;
     const int stage = (int)align_up((size_t)SR * args.p.d * 2, 128);
     // shared memory budget per CTA for the requested CTAs per SM
     const size_t per_sm = 227 * 1024;
@@ -499,7 +560,12 @@ cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_
     const int sms = semantic_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
     const SemTuning tun = semantic_tuning();
-    SemArgs args{a, ws, 0, 0, kWaitLimitNs, 0};
+    SemArgs args{a, ws, 0, 0, kWaitLimitNs, 0, ws.plan, ws.done2, ws.slots2};
+    if (a.nvseq) {  // the successor backoff pass has its own plan, counters and slots
+        args.plan = ws.plan3;
+        args.done = ws.done3;
+        args.slots = ws.slots3;
+    }
     // Test switch for the timeout path: the producer issues nothing, every
     // consumer wait runs out after 20 ms, the call reports ADAPLD_DEV_TIMEOUT
     // and publishes no result.  Never set in normal use.
@@ -511,8 +577,8 @@ cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_
     }
     const int d = a.d, R = tun.rows;
 #define ADAPLD_SEM(MAXC, SR, CPS, NS)                                                       \
-    return launch_variant<MAXC, SR>(args, sms, tun.ctas_per_sm ? tun.ctas_per_sm : CPS,       \
-                                    tun.stages ? tun.stages : NS, s)
+    return (a.tokens ? launch_variant<MAXC, SR, true> : launch_variant<MAXC, SR, false>)(    \
+        args, sms, tun.ctas_per_sm ? tun.ctas_per_sm : CPS, tun.stages ? tun.stages : NS, s)
     if (d <= 2048) {
         if (R == 4) ADAPLD_SEM(1, 4, 2, 2);
         if (R == 16) ADAPLD_SEM(1, 16, 2, 2);

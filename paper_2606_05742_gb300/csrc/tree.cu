@@ -144,6 +144,7 @@ __device__ float block_load_vec(const uint16_t *v, float *dst, int d, float *scr
 struct SeqView {
     int len;
     bool valid, cand_ok, lex, sem, branch_on, need_succ;
+    bool rr;  // the candidates are (re)ranked by Eq. 6 in this stage
     int nc;
 };
 
@@ -169,6 +170,10 @@ __device__ __forceinline__ SeqView view_of(const TreeLaunch &a, int b) {
     v.branch_on = !(flags & ADAPLD_NO_BRANCH) && W > 0 && (v.lex || v.sem);
     v.need_succ = v.branch_on && !(flags & ADAPLD_NO_SUCC) &&
                   (v.sem || (v.lex && (flags & ADAPLD_SUCC_ON_STRICT)));
+    // lexical hits are reranked unless switched off; semantic hits only in
+    // the two-representation mode (otherwise their retrieval scores already
+    // are the rerank scores)
+    v.rr = (v.lex && !(flags & ADAPLD_NO_LEX_RERANK)) || (v.sem && a.emb.table != nullptr);
     return v;
 }
 
@@ -259,18 +264,17 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
         s_score[t] = a.score[(int64_t)b * k + t];
     }
     __syncthreads();
-    if (v.lex) {  // successors on a strict hit: rerank first (each slice alike)
-        if (!(a.p.flags & ADAPLD_NO_LEX_RERANK)) {
-            const uint16_t *q = a.query + (int64_t)b * d;
-            for (int ci = warp; ci < v.nc; ci += nwarps) {
-                const float cs = warp_cosine(R + (int64_t)s_cand[ci] * d, q, d);
-                if (lane == 0) s_score[ci] = cs;
-            }
-            __syncthreads();
-            if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc);
-        } else if (t < v.nc) {
-            s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
+    if (v.rr) {  // the ranking the branches depend on (each slice alike)
+        const uint16_t *q = a.query + (int64_t)b * d;
+        for (int ci = warp; ci < v.nc; ci += nwarps) {
+            const float cs = warp_cosine(R + (int64_t)s_cand[ci] * d, q, d);
+            if (lane == 0) s_score[ci] = cs;
         }
+        __syncthreads();
+        if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc);
+        __syncthreads();
+    } else if (v.lex) {
+        if (t < v.nc) s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
         __syncthreads();
     }
     const int nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc);
@@ -315,12 +319,59 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
             (int)gridDim.x, k, [&](int s2) { return __ldcg(pw + s2 * stride); },
             [&](int s2, int i) { return __ldcg(pw + s2 * stride + 1 + i); },
             ws.succ + ((int64_t)b * ws.W + w) * kMaxK);
-        if (lane == 0) ws.succ_n[(int64_t)b * ws.W + w] = total;
+        if (lane == 0) {
+            ws.succ_n[(int64_t)b * ws.W + w] = total;
+            // Sec. 3.5: a branch token that never occurs backs off to the
+            // embedding fallback with the branch token as the anchor
+            if (total == 0 && a.emb.table) {
+                const int idx = atomicAdd(ws.npairs, 1);
+                ws.pair_b[idx] = b;
+                ws.pair_tok[idx] = s_br[w];
+                ws.pair_out[idx] = b * ws.W + w;
+            }
+        }
     }
-    if (v.lex && t < v.nc) {
+    if ((v.lex || v.rr) && t < v.nc) {
         ws.rr_cand[(int64_t)b * kMaxK + t] = s_cand[t];
         ws.rr_score[(int64_t)b * kMaxK + t] = s_score[t];
     }
+}
+
+// The plan of the successor backoff pass: row prefix sums over the
+// (sequence, branch) pairs registered by succ_scan_kernel (one CTA).
+__global__ void __launch_bounds__(256) backoff_plan_kernel(TreeArgs args) {
+    const TreeLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int64_t scratch[8];
+    pdl_wait_then_release();
+    const int n = *ws.npairs;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int64_t carry = 0;
+    for (int base = 0; base < n; base += 256) {
+        const int p = base + threadIdx.x;
+        int64_t rows = 0;
+        if (p < n) {
+            const int len = a.lengths[ws.pair_b[p]];
+            rows = len >= 2 ? len - 1 : 0;
+        }
+        int64_t incl = rows;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t u = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += u;
+        }
+        if (lane == 31) scratch[warp] = incl;
+        __syncthreads();
+        int64_t before = 0, all = 0;
+        for (int w = 0; w < 8; ++w) {
+            if (w < warp) before += scratch[w];
+            all += scratch[w];
+        }
+        if (p < n) ws.plan3[p] = carry + before + incl - rows;
+        carry += all;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) ws.plan3[n] = carry;
 }
 
 // ---------------------------------------------------------------------------
@@ -354,7 +405,7 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
 
     // ---- ranked candidates (the successor scan reranked a strict hit already)
     if (t < v.nc) {
-        if (v.need_succ && v.lex) {
+        if (v.need_succ && (v.lex || v.rr)) {
             s_cand[t] = __ldcg(ws.rr_cand + (int64_t)b * kMaxK + t);
             s_score[t] = __ldcg(ws.rr_score + (int64_t)b * kMaxK + t);
         } else {
@@ -368,7 +419,7 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
 
     // the rows this sequence scores, and the CTAs that share them: lexical
     // candidates against the query, or successor candidate (w, i) at w*k + i
-    const bool rerank = v.lex && !v.need_succ && !(flags & ADAPLD_NO_LEX_RERANK);
+    const bool rerank = v.rr && !v.need_succ;
     const int ntasks = v.need_succ ? nb * k : (rerank ? v.nc : 0);
     const int nctas = max(1, (ntasks + kRowsPerCta5 - 1) / kRowsPerCta5);
     if (r5 >= nctas) return;
@@ -511,7 +562,7 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
                           (node_path[i] == node_path[j] && j <= i && node_path[i] != 0));
         mk[idx] = anc ? 1 : 0;
     }
-    if (v.lex && t < k) {
+    if ((v.lex || v.rr) && t < k) {
         a.cand[(int64_t)b * k + t] = t < v.nc ? s_cand[t] : -1;
         a.score[(int64_t)b * k + t] = t < v.nc ? s_score[t] : 0.f;
     }
@@ -522,8 +573,9 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
             atomicAdd(a.out.stats + (v.lex ? 0 : (v.sem ? 1 : 2)), 1);
             if (s_misc[3]) atomicAdd(a.out.stats + 3, s_misc[3]);
         }
-        if (a.status)
-            a.status[b] = (v.valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) |
+        if (a.status)  // the embedding fallback may have flagged a token id
+            a.status[b] = (a.status[b] & ADAPLD_SEQ_BAD_TOKEN) |
+                          (v.valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) |
                           (v.cand_ok ? 0 : ADAPLD_SEQ_BAD_CANDIDATE);
     }
 }
@@ -540,6 +592,22 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
         cudaError_t e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), 0, s,
                                          args);
         if (e != cudaSuccess) return e;
+        if (a.emb.table) {  // successor backoff over token embeddings
+            e = launch_dependent(backoff_plan_kernel, dim3(1), dim3(256), 0, s, args);
+            if (e != cudaSuccess) return e;
+            SemLaunch sl{a.emb.table, a.ld, a.emb.dim, nullptr, a.lengths, nullptr, a.B, k,
+                         a.p.tau, ws.succ, ws.succ_es, ws.succ_n, nullptr, true};
+            sl.tokens = a.tokens;
+            sl.vocab = a.emb.vocab;
+            sl.vseq_b = ws.pair_b;
+            sl.vseq_tok = ws.pair_tok;
+            sl.vseq_out = ws.pair_out;
+            sl.nvseq = ws.npairs;
+            sl.out_stride = kMaxK;
+            sl.status = a.status;
+            e = launch_semantic(sl, ws, s);
+            if (e != cudaSuccess) return e;
+        }
     }
     const size_t smem = (size_t)a.d * sizeof(float);
     cudaError_t e = cudaFuncSetAttribute(tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

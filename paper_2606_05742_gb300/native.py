@@ -26,6 +26,7 @@ NO_BRANCH = 8
 NO_SUCC = 16
 SEQ_BAD_LENGTH = 1
 SEQ_BAD_CANDIDATE = 2
+SEQ_BAD_TOKEN = 4
 DEV_TIMEOUT = 1
 DEV_INTERNAL = 2
 
@@ -33,7 +34,7 @@ EXPORTED = [
     "adapld_tree_nodes", "adapld_workspace_bytes", "adapld_status_string",
     "adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
     "adapld_step", "adapld_step_ex", "adapld_read_device_status",
-    "adapld_semantic_topk_static",
+    "adapld_semantic_topk_static", "adapld_embedding_topk",
 ]
 STATIC_MAX_B = 1024
 ERR_STATIC_LIMIT = -15
@@ -71,6 +72,16 @@ class StepOut(ctypes.Structure):
                 ("tree", TreeOut)]
 
 
+class Embeddings(ctypes.Structure):
+    """Token-embedding table [vocab][dim] bf16 (two-representation mode)."""
+    _fields_ = [("table", ctypes.c_void_p), ("vocab", ctypes.c_int32), ("dim", ctypes.c_int32)]
+
+    @staticmethod
+    def of(table) -> "Embeddings":
+        V, dim = table.shape
+        return Embeddings(table.data_ptr(), V, dim)
+
+
 class StepEvents(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in
                 ("lexical_begin", "lexical_end", "semantic_begin", "semantic_end",
@@ -101,15 +112,17 @@ def load() -> ctypes.CDLL:
         lib.adapld_semantic_topk.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P, P, P, sz,
                                              P]
         lib.adapld_build_draft_tree.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, i32, P,
-                                                P, P, P, sz, P]
+                                                P, P, P, P, sz, P]
         lib.adapld_step.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P]
-        lib.adapld_step_ex.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P, P]
+        lib.adapld_step_ex.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P, P, P]
+        lib.adapld_embedding_topk.argtypes = [P, i64, P, P, P, i32, i32, f32, P, P, P, P, P, sz,
+                                              P]
         lib.adapld_read_device_status.argtypes = [P, P, P]
         lib.adapld_semantic_topk_static.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P,
                                                     P, P]
         for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
                   "adapld_step", "adapld_step_ex", "adapld_read_device_status",
-                  "adapld_semantic_topk_static"):
+                  "adapld_semantic_topk_static", "adapld_embedding_topk"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -179,17 +192,31 @@ def _tree_out(anchor, draft_tokens, parents, positions, mask, n_nodes, stats=Non
 
 
 def build_draft_tree(tokens, lengths, reps, query, hit_kind, cand, score, n_cand, p: Params,
-                     out: "Outputs", ws, next_topk=None, stream=None) -> None:
+                     out: "Outputs", ws, next_topk=None, emb=None, stream=None) -> None:
     B, ld, d = reps.shape
     to = _tree_out(out.anchor, out.draft_tokens, out.parents, out.positions, out.mask,
                    out.n_nodes, out.stats)
     kn = next_topk.shape[2] if next_topk is not None else 0
+    e = Embeddings.of(emb) if emb is not None else None
     rc = load().adapld_build_draft_tree(
         _ptr(tokens), ld, _ptr(lengths), _ptr(reps), d, _ptr(query), B, _ptr(hit_kind),
-        _ptr(cand), _ptr(score), _ptr(n_cand), _ptr(next_topk), kn, ctypes.byref(p),
+        _ptr(cand), _ptr(score), _ptr(n_cand), _ptr(next_topk), kn,
+        ctypes.byref(e) if e is not None else None, ctypes.byref(p),
         ctypes.byref(to), _ptr(out.status), _ptr(ws), ws.numel() * ws.element_size(),
         _stream(stream))
     _check(rc, "adapld_build_draft_tree")
+
+
+def embedding_topk(tokens, lengths, emb, k: int, tau: float, cand, score, n_cand, ws,
+                   active=None, status=None, stream=None) -> None:
+    """Eq. 4 over token embeddings (adapld_embedding_topk)."""
+    B, ld = tokens.shape
+    e = Embeddings.of(emb)
+    rc = load().adapld_embedding_topk(_ptr(tokens), ld, _ptr(lengths), ctypes.byref(e),
+                                      _ptr(active), B, k, tau, _ptr(cand), _ptr(score),
+                                      _ptr(n_cand), _ptr(status), _ptr(ws),
+                                      ws.numel() * ws.element_size(), _stream(stream))
+    _check(rc, "adapld_embedding_topk")
 
 
 @dataclass
@@ -251,18 +278,22 @@ def allocate_workspace(B: int, ld: int, d: int, p: Params, device="cuda"):
 
 
 def step(tokens, lengths, reps, query, p: Params, out: Outputs, ws, next_topk=None,
-         events: Optional[StepEvents] = None, stream=None) -> None:
-    """One draft-construction step (adapld_step / adapld_step_ex)."""
+         events: Optional[StepEvents] = None, stream=None, emb=None) -> None:
+    """One draft-construction step (adapld_step, or adapld_step_ex with
+    events and/or a token-embedding table `emb` [vocab][dim] bf16)."""
     B, ld, d = reps.shape
     so = out.c_struct()
     kn = next_topk.shape[2] if next_topk is not None else 0
     lib = load()
     args = (_ptr(tokens), ld, _ptr(lengths), _ptr(reps), d, _ptr(query), _ptr(next_topk), kn, B,
             ctypes.byref(p), ctypes.byref(so), _ptr(ws), ws.numel() * ws.element_size())
-    if events is None:
+    if events is None and emb is None:
         rc = lib.adapld_step(*args, _stream(stream))
     else:
-        rc = lib.adapld_step_ex(*args, ctypes.byref(events), _stream(stream))
+        e = Embeddings.of(emb) if emb is not None else None
+        rc = lib.adapld_step_ex(*args, ctypes.byref(e) if e is not None else None,
+                                ctypes.byref(events) if events is not None else None,
+                                _stream(stream))
     _check(rc, "adapld_step")
 
 
@@ -284,8 +315,10 @@ class Engine:
         self.out = Outputs.allocate(B, p, device)
         self.ws = allocate_workspace(B, ld, d, p, device)
 
-    def run(self, tokens, lengths, reps, query, next_topk=None, events=None, stream=None):
-        step(tokens, lengths, reps, query, self.p, self.out, self.ws, next_topk, events, stream)
+    def run(self, tokens, lengths, reps, query, next_topk=None, events=None, stream=None,
+            emb=None):
+        step(tokens, lengths, reps, query, self.p, self.out, self.ws, next_topk, events, stream,
+             emb)
         return self.out
 
     def run_from_host(self, tokens_h, lengths_h, reps_h, query_h, dev_inputs, host_out,

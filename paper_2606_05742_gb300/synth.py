@@ -282,3 +282,52 @@ def make_next_topk(tokens: np.ndarray, lengths: np.ndarray, V: int, Kn: int,
                     row.append(t)
             out[b, j] = row
     return out
+
+
+def make_embeddings(w: Workload, V: int, de: int, seed: int = 0, synonyms: int = 3):
+    """A token-embedding table E[V][de] (bf16) for the two-representation
+    mode: i.i.d. N(0,1) rows, and for every forced lexical miss, `synonyms`
+    tokens of its history (always including the token just before the
+    anchor) get rows E[a] + 0.3 N(0, I) around the anchor's row, so the
+    embedding fallback (Eq. 4) finds them and a candidate right before the
+    anchor makes the anchor itself a branch token with no earlier
+    occurrence (the successor backoff of Sec. 3.5).  numpy uint16 bits on
+    the CPU, a torch bf16 tensor when the workload lives on a GPU."""
+    tokens = w.tokens if isinstance(w.tokens, np.ndarray) else w.tokens.cpu().numpy()
+    lengths = w.lengths if isinstance(w.lengths, np.ndarray) else w.lengths.cpu().numpy()
+    rng = np.random.default_rng([seed, 31337, V, de])
+    plants = []
+    for b in w.forced:
+        ln = int(lengths[b])
+        if ln < 3:
+            continue
+        a = int(tokens[b, ln - 1])
+        hist = tokens[b, : ln - 1]
+        pick = {int(hist[-1])}
+        cand = np.unique(hist[hist != a])
+        extra = rng.permutation(cand)[: max(0, synonyms - 1)]
+        pick.update(int(x) for x in extra)
+        pick.discard(a)
+        plants.append((a, sorted(pick)))
+    if w.device == "cpu":
+        E = rng.standard_normal((V, de), dtype=np.float32)
+        for a, vs in plants:
+            for v in vs:
+                E[v] = E[a] + np.float32(NOISE) * rng.standard_normal(de, dtype=np.float32)
+        return f32_to_bf16_bits(E)
+    import torch
+    dev = torch.device(w.device)
+    g = torch.Generator(device=dev)
+    g.manual_seed(int(rng.integers(0, 2**62)))
+    E = torch.empty((V, de), dtype=torch.bfloat16, device=dev)
+    chunk = max(1, (1 << 26) // de)
+    for r0 in range(0, V, chunk):
+        r1 = min(V, r0 + chunk)
+        E[r0:r1] = torch.randn((r1 - r0, de), generator=g, device=dev,
+                               dtype=torch.float32).to(torch.bfloat16)
+    for a, vs in plants:
+        ea = E[a].float()
+        for v in vs:
+            E[v] = (ea + NOISE * torch.randn(de, generator=g, device=dev,
+                                             dtype=torch.float32)).to(torch.bfloat16)
+    return E

@@ -93,10 +93,48 @@ def check_semantic_list(gc, gs, gn, s_all, eps, k, tau, rep: Report, where=""):
         assert len(bad) == 0, f"{where}: rows {bad[:5]} above tau missing"
 
 
-def _successor_ok(M, length, R, d, js, btok, chain, k, succ_len):
+def check_candidate_set(C, s_all, eps, k, tau, where=""):
+    """A candidate set (any order) is a valid top-k-above-tau set under the
+    fp64 scores within the bound (membership, count, completeness)."""
+    n_rows = len(s_all)
+    assert len(set(C)) == len(C), f"{where}: duplicate candidates {C}"
+    assert all(0 <= j < n_rows for j in C), f"{where}: candidate out of range {C}"
+    for j in C:
+        assert s_all[j] >= tau - eps[j], f"{where}: row {j} below tau"
+    n_lo = min(k, int((s_all >= tau + eps).sum()))
+    n_hi = min(k, int((s_all >= tau - eps).sum()))
+    assert n_lo <= len(C) <= n_hi, f"{where}: count {len(C)} not in [{n_lo}, {n_hi}]"
+    inside = np.zeros(n_rows, bool)
+    inside[C] = True
+    out_idx = np.flatnonzero(~inside & (s_all >= tau - eps))
+    if len(C) == k and C:
+        worst = min(C, key=lambda j: (s_all[j], j))
+        bad = out_idx[s_all[out_idx] > s_all[worst] + eps[out_idx] + eps[worst]]
+        assert len(bad) == 0, f"{where}: rows {bad[:5]} beat the worst candidate"
+    elif len(out_idx):
+        bad = out_idx[s_all[out_idx] >= tau + eps[out_idx]]
+        assert len(bad) == 0, f"{where}: rows {bad[:5]} above tau missing"
+
+
+def emb_scores(M, length, E):
+    """cos(E[M[j]], E[M[len-1]]) for j in [0, len-2] (fp64) and the bounds."""
+    rows = np.ascontiguousarray(E[np.asarray(M[: length - 1])])
+    ea = E[int(M[length - 1])]
+    return oracle.scores_all(rows, ea, length), eps_rows(rows, ea, E.shape[1]) if length > 1 \
+        else np.zeros(0)
+
+
+def _successor_ok(M, length, R, d, js, btok, chain, k, succ_len, emb=None, tau=0.1):
     """The GPU's successor chain for branch token btok is the continuation of
-    some occurrence whose Eq. 13 score is within the bound of the best."""
-    ts, ss = oracle.successor_candidates(M, length, R, d, js, btok, k)
+    some candidate whose Eq. 13 score is within the bound of the best (the
+    candidates being the lexical occurrences, or the embedding backoff)."""
+    if emb is not None:
+        ts, ss = oracle.successor_candidates_emb(M, length, R, d, emb, tau, js, btok, 2 * k)
+        lex = [t for t in range(length - 2, -1, -1) if M[t] == btok]
+        if lex:
+            ts, ss = ts[:k], ss[:k]
+    else:
+        ts, ss = oracle.successor_candidates(M, length, R, d, js, btok, k)
     if not ts:
         return chain == []
     ss = np.asarray(ss)
@@ -121,7 +159,8 @@ def _chain_nodes(par, n, head):
         nodes.append(cur)
 
 
-def compare_sequence(b, M, length, ld, R, q, g, P, rep: Report, topk_table=None, full_eps=True):
+def compare_sequence(b, M, length, ld, R, q, g, P, rep: Report, topk_table=None, full_eps=True,
+                     emb=None):
     """Checks sequence b of a GPU step (host dict g) against the oracle.
     P: dict(n_max, k, W, D, succ_len, tau, flags); topk_table: this
     sequence's [ld][Kn] next-token table or None."""
@@ -163,6 +202,24 @@ def compare_sequence(b, M, length, ld, R, q, g, P, rep: Report, topk_table=None,
             tied = C != oc
     elif flags & oracle.NO_SEMANTIC:
         assert hit == oracle.NONE and gn == 0, where
+    elif emb is not None:
+        # Eq. 4 over token embeddings selects the set, Eq. 6 orders it
+        s_emb, e_emb = emb_scores(M, length, emb)
+        C = [int(x) for x in gc[:gn]]
+        assert (np.asarray(gc[gn:]) == -1).all(), f"{where}: cand padding"
+        check_candidate_set(C, s_emb, e_emb, k, tau, where)
+        assert hit == (oracle.SEM if gn else oracle.NONE), where
+        if gn:
+            s_map = dict(zip(*oracle.rerank(R, q, C)))
+            e = eps_rows(R[np.asarray(C)], q, d)
+            for i, j in enumerate(C):
+                err = abs(float(gs[i]) - s_map[j])
+                rep.max_score_err = max(rep.max_score_err, err)
+                assert err <= SCORE_ATOL, f"{where}: rerank score {err}"
+            for i in range(len(C) - 1):
+                assert s_map[C[i + 1]] <= s_map[C[i]] + e[i] + e[i + 1], f"{where}: rerank order"
+        oc, _ = oracle.semantic_emb(M, length, emb, k, tau)
+        tied = sorted(C) != sorted(oc) or C != oracle.rerank(R, q, oc)[0]
     else:
         s_all = oracle.scores_all(R, q, length)
         eps = eps_rows(R[: length - 1], q, d) if full_eps else np.full(length - 1, eps_uniform(d))
@@ -173,7 +230,8 @@ def compare_sequence(b, M, length, ld, R, q, g, P, rep: Report, topk_table=None,
     # conditional tree: the oracle's construction from the GPU's ranked list
     cands = [int(x) for x in gc[:gn]]
     topk_row = topk_table[cands[0]] if (topk_table is not None and cands) else None
-    T = oracle.tree_from(M, length, R, d, hit, cands, k, W, D, sl, flags, topk_row)
+    T = oracle.tree_from(M, length, R, d, hit, cands, k, W, D, sl, flags, topk_row, emb=emb,
+                         tau=tau)
     n = int(g["n_nodes"][b])
     assert int(g["anchor"][b]) == T.anchor, where
     gt, gp, gpos, gm = g["draft_tokens"][b], g["parents"][b], g["positions"][b], g["mask"][b]
@@ -192,8 +250,8 @@ def compare_sequence(b, M, length, ld, R, q, g, P, rep: Report, topk_table=None,
         for c, nodes in succ_nodes.items():
             chain = [int(gt[i]) for i in nodes]
             if chain != [int(T.tokens[i]) for i in nodes]:
-                assert _successor_ok(M, length, R, d, T.anchor, int(gt[c]), chain, k, sl), \
-                    f"{where}: successor below node {c}"
+                assert _successor_ok(M, length, R, d, T.anchor, int(gt[c]), chain, k, sl,
+                                     emb, tau), f"{where}: successor below node {c}"
                 tied = True
     if tied:
         rep.tie_resolved += 1

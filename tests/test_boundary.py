@@ -40,7 +40,7 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_status_strings(lib):
-    for code in (0, -1, -2, -3, -4, -5, -6, -7, -8, -9, -10, -11, -12, -13, -14, -15, -20):
+    for code in (0, -1, -2, -3, -4, -5, -6, -7, -8, -9, -10, -11, -12, -13, -14, -15, -16, -20):
         s = native.status_string(code)
         assert s and s != "unknown status"
     assert native.status_string(-999) == "unknown status"
@@ -132,13 +132,25 @@ def test_entry_point_argument_errors(lib):
     to = native.TreeOut(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None)
     p = native.make_params(3, 8, 2, 8)
     assert L.adapld_build_draft_tree(FAKE, 64, FAKE, FAKE, 16, FAKE, 2, FAKE, FAKE, FAKE, FAKE,
-                                     None, 0, ctypes.byref(p), None, None, FAKE, 1 << 30,
+                                     None, 0, None, ctypes.byref(p), None, None, FAKE, 1 << 30,
                                      None) == -1
     bad = native.make_params(3, 8, 2, 8, 1)
     bad.k = 0
     assert L.adapld_build_draft_tree(FAKE, 64, FAKE, FAKE, 16, FAKE, 2, FAKE, FAKE, FAKE, FAKE,
-                                     None, 0, ctypes.byref(bad), ctypes.byref(to), None, FAKE,
-                                     1 << 30, None) == -4
+                                     None, 0, None, ctypes.byref(bad), ctypes.byref(to), None,
+                                     FAKE, 1 << 30, None) == -4
+    for e in (native.Embeddings(None, 10, 16), native.Embeddings(FAKE + 2, 10, 16),
+              native.Embeddings(FAKE, 0, 16), native.Embeddings(FAKE, 10, 12)):
+        assert L.adapld_build_draft_tree(FAKE, 64, FAKE, FAKE, 16, FAKE, 2, FAKE, FAKE, FAKE,
+                                         FAKE, None, 0, ctypes.byref(e), ctypes.byref(p),
+                                         ctypes.byref(to), None, FAKE, 1 << 30, None) == -16
+        assert L.adapld_embedding_topk(FAKE, 64, FAKE, ctypes.byref(e), None, 2, 8, 0.1, FAKE,
+                                       FAKE, FAKE, None, FAKE, 1 << 30, None) == -16
+    good = native.Embeddings(FAKE, 10, 16)
+    assert L.adapld_embedding_topk(FAKE, 64, FAKE, None, None, 2, 8, 0.1, FAKE, FAKE, FAKE,
+                                   None, FAKE, 1 << 30, None) == -1
+    assert L.adapld_embedding_topk(FAKE, 64, FAKE, ctypes.byref(good), None, 2, 0, 0.1, FAKE,
+                                   FAKE, FAKE, None, FAKE, 1 << 30, None) == -4
     v = ctypes.c_int32(0)
     assert L.adapld_read_device_status(None, ctypes.byref(v), None) == -1
 

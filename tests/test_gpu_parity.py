@@ -45,11 +45,12 @@ def params(P):
                               P["flags"])
 
 
-def run_step(w, P, next_topk=None):
+def run_step(w, P, next_topk=None, emb=None):
     tok, ln, reps, q = to_dev(w)
     eng = native.Engine(w.B, w.ld, w.d, params(P))
     nt = torch.from_numpy(next_topk).cuda() if next_topk is not None else None
-    eng.run(tok, ln, reps, q, next_topk=nt)
+    E = torch.from_numpy(emb.view(np.int16)).cuda().view(torch.bfloat16) if emb is not None else None
+    eng.run(tok, ln, reps, q, next_topk=nt, emb=E)
     torch.cuda.synchronize()
     assert native.read_device_status(eng.ws) == 0
     return eng.out.to_host()
@@ -64,13 +65,13 @@ def succ_extensions(g, b):
     return sum(1 for h in heads if (par == h).any())
 
 
-def check_all(w, g, P, next_topk=None, full_eps=True, seqs=None):
+def check_all(w, g, P, next_topk=None, full_eps=True, seqs=None, emb=None):
     rep = parity.Report()
     seqs = range(w.B) if seqs is None else seqs
     for b in seqs:
         parity.compare_sequence(b, w.tokens[b], int(w.lengths[b]), w.ld, w.reps[b], w.query[b],
                                 g, P, rep, None if next_topk is None else next_topk[b],
-                                full_eps)
+                                full_eps, emb)
     hk = g["hit_kind"]
     exp_stats = [int((hk == 1).sum()), int((hk == 2).sum()), int(w.B - (hk == 1).sum() - (hk == 2).sum()),
                  sum(succ_extensions(g, b) for b in range(w.B))]
@@ -409,3 +410,120 @@ def test_end_to_end_from_host_matches_device_path():
         for name, t in zip(names, host_out):
             assert np.array_equal(t.numpy(), g[name], equal_nan=True), name
     assert h2d == w.tokens.nbytes + w.lengths.nbytes + w.reps.nbytes + w.query.nbytes
+
+
+# --------------------------------------------- token-embedding (two-representation) mode
+EMB_CASES = [  # (cfg, B, L, d, de, V, seed)
+    (2, 8, 1500, 128, 64, 4096, 0), (5, 4, 3000, 256, 4096, 8192, 1),
+    (3, 6, 2000, 640, 136, 3000, 2), (4, 20, 500, 64, 8, 2048, 3),
+    (5, 3, 1200, 64, 8192, 2048, 4),
+]
+
+
+@pytest.mark.parametrize("cfg,B,L,d,de,V,seed", EMB_CASES)
+def test_embedding_mode(cfg, B, L, d, de, V, seed):
+    """Eq. 4 over token embeddings, Eq. 6 rerank of the semantic candidates,
+    and the successor backoff of Sec. 3.5, against the oracle."""
+    w = synth.make_workload(cfg, B=B, L=L, d=d, V=V, nohit=0.6, seed=seed)
+    E = synth.make_embeddings(w, V, de, seed)
+    backoff = 0
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        g = run_step(w, P, emb=E)
+        check_all(w, g, P, emb=E)
+        o = oracle.step(w.tokens, w.lengths, w.reps, w.query, w.n_max, w.k, w.W, w.D,
+                        w.succ_len, tau, 0, emb=E)
+        assert (o.hit == g["hit_kind"]).all()
+        for b in range(w.B):
+            if o.hit[b] == oracle.SEM:
+                L_b = int(w.lengths[b])
+                backoff += sum(1 for i in range(1, int(o.n_nodes[b]))
+                               if o.parents[b, i] == 0 and
+                               not (w.tokens[b, : L_b - 1] == o.tokens[b, i]).any())
+    print("branches needing the backoff:", backoff)
+
+
+def test_embedding_mode_with_next_token_table():
+    w = synth.make_workload(2, B=6, L=700, d=64, V=4096, nohit=0.5, seed=71)
+    E = synth.make_embeddings(w, 4096, 64, 71)
+    tk = synth.make_next_topk(w.tokens, w.lengths, 4096, 5)
+    P = P_of(w)
+    check_all(w, run_step(w, P, next_topk=tk, emb=E), P, next_topk=tk, emb=E)
+
+
+def test_embedding_topk_standalone():
+    w = synth.make_workload(3, B=7, L=2500, d=16, V=5000, nohit=1.0, seed=72)
+    de = 256
+    E = synth.make_embeddings(w, 5000, de, 72)
+    tok, ln, _, _ = to_dev(w)
+    Ed = torch.from_numpy(E.view(np.int16)).cuda().view(torch.bfloat16)
+    p = native.make_params(w.n_max, w.k, w.W, w.D)
+    ws = native.allocate_workspace(w.B, w.ld, w.d, p)
+    cand = torch.full((w.B, w.k), -7, dtype=torch.int32, device="cuda")
+    score = torch.zeros((w.B, w.k), dtype=torch.float32, device="cuda")
+    n = torch.full((w.B,), -7, dtype=torch.int32, device="cuda")
+    status = torch.zeros(w.B, dtype=torch.int32, device="cuda")
+    active = (torch.arange(w.B, device="cuda") != 3).to(torch.uint8)
+    for tau in (0.1, NEG_INF):
+        native.embedding_topk(tok, ln, Ed, w.k, tau, cand, score, n, ws, active=active,
+                              status=status)
+        torch.cuda.synchronize()
+        assert native.read_device_status(ws) == 0
+        rep = parity.Report()
+        for b in range(w.B):
+            if b == 3:
+                assert int(n[b]) == -7
+                continue
+            L_b = int(w.lengths[b])
+            s_all, eps = parity.emb_scores(w.tokens[b], L_b, E)
+            parity.check_semantic_list(cand[b].cpu().numpy(), score[b].cpu().numpy(), int(n[b]),
+                                       s_all, eps, w.k, tau, rep, f"seq {b}")
+        assert int(status.sum()) == 0
+
+
+def test_embedding_mode_token_out_of_table():
+    """A token id outside the table reads row 0 and is flagged, no fault."""
+    w = synth.make_workload(2, B=3, L=400, d=32, V=1000, nohit=1.0, seed=73)
+    E = synth.make_embeddings(w, 1000, 32, 73)
+    w.tokens[1, 10] = 5000
+    w.tokens[2, 399] = -3           # the anchor itself
+    P = P_of(w)
+    tok, ln, reps, q = to_dev(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    eng.run(tok, ln, reps, q, emb=torch.from_numpy(E.view(np.int16)).cuda().view(torch.bfloat16))
+    torch.cuda.synchronize()
+    assert native.read_device_status(eng.ws) == 0
+    st = eng.out.status.cpu().numpy()
+    assert st[1] & native.SEQ_BAD_TOKEN and st[2] & native.SEQ_BAD_TOKEN
+    assert not st[0] & native.SEQ_BAD_TOKEN
+
+
+def test_full_size_embedding_config5():
+    """Config 5 with a 128256 x 8192 embedding table (2.1 GB), launched as the
+    benchmark's embedding mode does; the oracle checks the forced misses."""
+    w = synth.make_workload(5, device="cuda")
+    V, de = synth.CONFIGS[5]["V"], w.d
+    Ed = synth.make_embeddings(w, V, de, 0)
+    P = P_of(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    eng.run(w.tokens, w.lengths, w.reps, w.query, emb=Ed)
+    torch.cuda.synchronize()
+    assert native.read_device_status(eng.ws) == 0
+    g = eng.out.to_host()
+    tokens = w.tokens.cpu().numpy()
+    lengths = w.lengths.cpu().numpy()
+    E = Ed.view(torch.int16).cpu().numpy().view(np.uint16)
+    sample = [int(b) for b in w.forced][:3]
+    rep = parity.Report()
+
+    def one(b):
+        R = w.reps[b].view(torch.int16).cpu().numpy().view(np.uint16)
+        q = w.query[b].view(torch.int16).cpu().numpy().view(np.uint16)
+        parity.compare_sequence(b, tokens[b], int(lengths[b]), w.ld, R, q, g, P, rep,
+                                full_eps=False, emb=E)
+
+    with ThreadPoolExecutor(max_workers=3) as ex:
+        list(ex.map(one, sample))
+    print(f"config 5 with embeddings: sample {sample}: {rep}")
+    for b in sample:
+        assert g["hit_kind"][b] == 2
