@@ -80,6 +80,11 @@ def _load():
         lib.oracle_tree_from_emb.argtypes = [P, i32, P, i32, P, i32, f64, i32, P, i32, P, i32,
                                              i32, i32, i32, i32, u32, i32, P, P, P, P, P, P]
         lib.oracle_tree_from_emb.restype = i32
+        lib.oracle_verify_greedy.argtypes = [P, i32, P, P, i32, P, P, P]
+        lib.oracle_verify_greedy.restype = i32
+        lib.oracle_accept_greedy.argtypes = [P, i32, P, P, P, i32, i32, P, P, P, P, i64, P, P, P,
+                                             i32, P, P]
+        lib.oracle_accept_greedy.restype = None
         _lib = lib
     return _lib
 
@@ -283,3 +288,57 @@ def step(tokens, lengths, reps, query, n_max: int, k: int, W: int, D: int,
                             _p(hit), _p(mn), _p(anchor), _p(cand), _p(score), _p(nc), _p(tok),
                             _p(par), _p(pos), _p(mask), _p(nn), _p(stats))
     return StepResult(hit, mn, anchor, cand, score, nc, tok, par, pos, mask, nn, stats)
+
+
+def verify_greedy(logits, tokens, parents, n_nodes: int):
+    """Greedy tree verification (Sec. 3.6, Eq. 16 at temperature 0): returns
+    (accepted draft count, new tokens incl. the bonus, path of nodes)."""
+    lg = _c(logits, np.uint16)
+    tk = _c(tokens, np.int32)
+    pr = _c(parents, np.int32)
+    N, V = lg.shape
+    nt = np.full(max(N, 1), -1, np.int32)
+    path = np.zeros(max(N, 1), np.int32)
+    nn = np.zeros(1, np.int32)
+    acc = _load().oracle_verify_greedy(_p(lg), V, _p(tk), _p(pr), n_nodes, _p(nt), _p(path),
+                                       _p(nn))
+    n = int(nn[0])
+    return int(acc), nt[:n].tolist(), path[:n].tolist()
+
+
+@dataclass
+class AcceptResult:
+    n_accept: np.ndarray
+    new_tokens: np.ndarray
+    n_new: np.ndarray
+    full: np.ndarray
+
+
+def accept_greedy(logits, draft_tokens, parents, n_nodes, tokens=None, lengths=None,
+                  node_reps=None, reps=None, query=None) -> AcceptResult:
+    """Verification and append for a batch; tokens/lengths/reps/query (numpy,
+    modified in place) are optional (all or none for the append)."""
+    lg = _c(logits, np.uint16)
+    B, N, V = lg.shape
+    tk = _c(draft_tokens, np.int32)
+    pr = _c(parents, np.int32)
+    nn = _c(n_nodes, np.int32)
+    n_acc = np.zeros(B, np.int32)
+    new = np.zeros((B, N), np.int32)
+    n_new = np.zeros(B, np.int32)
+    full = np.zeros(B, np.int32)
+    if tokens is not None:
+        assert tokens.dtype == np.int32 and tokens.flags.c_contiguous
+        ld = tokens.shape[1]
+        args = [_p(tokens), ld, _p(lengths)]
+    else:
+        args = [None, 0, None]
+    if node_reps is not None:
+        nr = _c(node_reps, np.uint16)
+        d = nr.shape[2]
+        args += [_p(nr), _p(reps), d, _p(query)]
+    else:
+        args += [None, None, 0, None]
+    _load().oracle_accept_greedy(_p(lg), V, _p(tk), _p(pr), _p(nn), B, N, _p(n_acc), _p(new),
+                                 _p(n_new), *args, _p(full))
+    return AcceptResult(n_acc, new, n_new, full)

@@ -558,3 +558,95 @@ void oracle_step(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                     W, D, succ_len, tau, flags, nmax, hit, match_n, anchor, cand, score,
                     n_cand, tok, par, pos, mask, n_nodes, stats);
 }
+
+/*
+ * Greedy verification of one draft tree (Sec. 3.6; Appendix C, Eq. 16: at
+ * temperature 0 a draft token is accepted iff it equals the target model's
+ * greedy choice).  logits[i][v] (bf16 bits, rows V apart) are the target's
+ * next-token logits after tree node i; its choice there is the first index
+ * of the maximum.  From the root, the child of the current node whose token
+ * equals the choice at the current node is accepted, until there is none.
+ * The new tokens are the accepted draft tokens followed by the choice after
+ * the last accepted node (the bonus token of Algorithm 1); path[0] is the
+ * root and path[i] the i-th accepted node.  Returns the number of accepted
+ * draft tokens; *n_new is that plus one (0 for an empty tree).
+ */
+int32_t oracle_verify_greedy(const uint16_t *logits, int32_t V, const int32_t *tok,
+                             const int32_t *par, int32_t n_nodes, int32_t *new_tokens,
+                             int32_t *path, int32_t *n_new)
+{
+    *n_new = 0;
+    if (n_nodes < 1)
+        return 0;
+    int32_t cur = 0, n_acc = 0;
+    for (;;) {
+        const uint16_t *row = logits + (int64_t)cur * V;
+        int32_t best = 0;
+        for (int32_t v = 1; v < V; ++v)
+            if (bf16_bits_to_double(row[v]) > bf16_bits_to_double(row[best]))
+                best = v;
+        path[n_acc] = cur;
+        int32_t next = -1;
+        for (int32_t i = 1; i < n_nodes; ++i)
+            if (par[i] == cur && tok[i] == best) {
+                next = i;
+                break;
+            }
+        if (next < 0) {
+            new_tokens[n_acc] = best;  /* the bonus token */
+            *n_new = n_acc + 1;
+            return n_acc;
+        }
+        new_tokens[n_acc] = tok[next];
+        ++n_acc;
+        cur = next;
+    }
+}
+
+/*
+ * Verification and the memory append for B sequences (Algorithm 1: append
+ * the accepted tokens and the bonus token, update the context).  Per
+ * sequence: oracle_verify_greedy on logits[b] ([N][V]); then, if
+ * len + n_new <= ld, tokens[b][len + i] = new_tokens[i], lengths[b] += n_new
+ * and, when node_reps ([B][N][d]) is given, reps[b][len + i] =
+ * node_reps[b][path[i]] (the hidden state after each new position's
+ * predecessor) and query[b] = node_reps[b][path[n_new - 1]]; otherwise
+ * full[b] = 1 and nothing is appended.  n_accept[b], new_tokens[b][N]
+ * (padding -1) and n_new[b] are always written.
+ */
+void oracle_accept_greedy(const uint16_t *logits, int32_t V, const int32_t *tok,
+                          const int32_t *par, const int32_t *n_nodes, int32_t B, int32_t N,
+                          int32_t *n_accept, int32_t *new_tokens, int32_t *n_new,
+                          int32_t *tokens, int64_t ld, int32_t *lengths,
+                          const uint16_t *node_reps, uint16_t *reps, int32_t d,
+                          uint16_t *query, int32_t *full)
+{
+    int32_t *path = (int32_t *)malloc(sizeof(int32_t) * (size_t)(N > 0 ? N : 1));
+    for (int32_t b = 0; b < B; ++b) {
+        int32_t *nt = new_tokens + (int64_t)b * N;
+        for (int32_t i = 0; i < N; ++i)
+            nt[i] = -1;
+        full[b] = 0;
+        n_accept[b] = oracle_verify_greedy(logits + (int64_t)b * N * V, V,
+                                           tok + (int64_t)b * N, par + (int64_t)b * N,
+                                           n_nodes[b], nt, path, &n_new[b]);
+        if (tokens == NULL || n_new[b] == 0)
+            continue;
+        int32_t len = lengths[b];
+        if (len + n_new[b] > ld) {
+            full[b] = 1;
+            continue;
+        }
+        for (int32_t i = 0; i < n_new[b]; ++i)
+            tokens[(int64_t)b * ld + len + i] = nt[i];
+        if (node_reps != NULL) {
+            for (int32_t i = 0; i < n_new[b]; ++i)
+                memcpy(reps + ((int64_t)b * ld + len + i) * d,
+                       node_reps + ((int64_t)b * N + path[i]) * d, sizeof(uint16_t) * (size_t)d);
+            memcpy(query + (int64_t)b * d, node_reps + ((int64_t)b * N + path[n_new[b] - 1]) * d,
+                   sizeof(uint16_t) * (size_t)d);
+        }
+        lengths[b] = len + n_new[b];
+    }
+    free(path);
+}

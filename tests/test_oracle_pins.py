@@ -563,3 +563,120 @@ def test_successor_backoff_bruteforce(seed):
         np.testing.assert_allclose(sc, exp_s, atol=1e-12)
     # without a table a token that never occurs has no successor candidates
     assert oracle.successor_candidates(M, L, R, d, js, V - 1, k) == ([], [])
+
+
+# ---------------------------------------------------- greedy verification
+def _logits_rows(g, case, N, V):
+    L = np.zeros((N, V), np.float32)
+    for i in range(N):
+        key = f"{case}_node{i}"
+        if key in g:
+            vals = g[key]
+            for t, v in zip(vals[0::2], vals[1::2]):
+                L[i, int(t)] = float(v)
+    return synth.f32_to_bf16_bits(L)
+
+
+@pytest.mark.parametrize("case", ["A", "B", "C"])
+def test_worked_example_verify(case):
+    g = load_golden("worked_example_verify.txt")
+    tok = np.array(ints(g["tree_tokens"]), np.int32)
+    par = np.array(ints(g["tree_parents"]), np.int32)
+    V = int(g["vocab"][0])
+    lg = _logits_rows(g, case, len(tok), V)
+    acc, new, path = oracle.verify_greedy(lg, tok, par, len(tok))
+    assert acc == int(g[f"{case}_accept"][0])
+    assert new == ints(g[f"{case}_new"])
+    assert path == ints(g[f"{case}_path"])
+
+
+def _verify_bruteforce(lg, tok, par, n):
+    target = [int(np.argmax(synth.bf16_bits_to_f32(lg[i]))) for i in range(n)]
+    ok = [True] + [False] * (n - 1)
+    for i in range(1, n):
+        ok[i] = ok[par[i]] and tok[i] == target[par[i]]
+    deepest = max((i for i in range(n) if ok[i]), key=lambda i: _depth(par, i))
+    chain = []
+    cur = deepest
+    while cur != 0:
+        chain.append(cur)
+        cur = par[cur]
+    chain = chain[::-1]
+    return len(chain), [int(tok[c]) for c in chain] + [target[deepest]], [0] + chain
+
+
+def _depth(par, i):
+    d = 0
+    while par[i] >= 0:
+        i = par[i]
+        d += 1
+    return d
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_verify_bruteforce_on_built_trees(seed):
+    """Trees built by the oracle itself; logits with small integer values so
+    maxima tie often; numpy's argmax takes the first maximum."""
+    rng = np.random.default_rng(1000 + seed)
+    M, L, R, q, d = _random_case(rng)
+    flags = [0, oracle.SUCC_ON_STRICT][seed % 2]
+    res = oracle.step(M[None], [L], R[None], q[None], 3, 4, 3, 5, 2, NEG_INF, flags)
+    n = int(res.n_nodes[0])
+    tok, par = res.tokens[0, :n], res.parents[0, :n]
+    V = 6
+    # bias each node's logits towards a child's token half of the time
+    lg = rng.integers(-2, 3, size=(n, V)).astype(np.float32)
+    for i in range(n):
+        kids = [c for c in range(n) if par[c] == i]
+        if kids and rng.random() < 0.6:
+            t = int(tok[kids[int(rng.integers(len(kids)))]])
+            if t < V:
+                lg[i, t] = 5.0
+    M2 = np.where(tok >= V, V - 1, tok).astype(np.int32)   # keep tokens inside the vocabulary
+    lgb = synth.f32_to_bf16_bits(lg)
+    assert oracle.verify_greedy(lgb, M2, par, n) == _verify_bruteforce(lgb, M2, par, n)
+
+
+def test_verify_chain_is_longest_matching_prefix():
+    """A chain tree (prompt-lookup draft): the accepted tokens are the longest
+    prefix of the draft agreeing with the target's choices."""
+    rng = np.random.default_rng(5)
+    for _ in range(30):
+        n = int(rng.integers(1, 9))
+        tok = rng.integers(0, 4, size=n).astype(np.int32)
+        par = np.arange(-1, n - 1, dtype=np.int32)
+        target = rng.integers(0, 4, size=n)
+        lg = np.full((n, 4), -1.0, np.float32)
+        lg[np.arange(n), target] = 1.0
+        acc, new, path = oracle.verify_greedy(synth.f32_to_bf16_bits(lg), tok, par, n)
+        m = 0
+        while m + 1 < n and tok[m + 1] == target[m]:
+            m += 1
+        assert acc == m and new == tok[1:m + 1].tolist() + [int(target[m])]
+
+
+def test_accept_appends_tokens_and_rows():
+    rng = np.random.default_rng(6)
+    B, N, V, d, ld = 3, 5, 12, 8, 10
+    tok = np.tile(np.array([7, 3, 5, 7, 9], np.int32), (B, 1))
+    par = np.tile(np.array([-1, 0, 1, 2, 0], np.int32), (B, 1))
+    n_nodes = np.array([5, 5, 0], np.int32)
+    lg = np.zeros((B, N, V), np.float32)
+    lg[0, 0, 3] = lg[0, 1, 5] = lg[0, 2, 4] = 1.0      # accept 3, 5; bonus 4
+    lg[1, 0, 9] = lg[1, 4, 2] = 1.0                    # accept 9; bonus 2
+    lgb = synth.f32_to_bf16_bits(lg)
+    tokens = np.arange(B * ld, dtype=np.int32).reshape(B, ld)
+    lengths = np.array([5, 9, 4], np.int32)
+    node_reps = synth.f32_to_bf16_bits(rng.standard_normal((B, N, d)).astype(np.float32))
+    reps = np.zeros((B, ld, d), np.uint16)
+    query = np.zeros((B, d), np.uint16)
+    t0, r0 = tokens.copy(), reps.copy()
+    r = oracle.accept_greedy(lgb, tok, par, n_nodes, tokens, lengths, node_reps, reps, query)
+    assert r.n_accept.tolist() == [2, 1, 0] and r.n_new.tolist() == [3, 2, 0]
+    assert r.new_tokens[0, :3].tolist() == [3, 5, 4] and r.new_tokens[1, :2].tolist() == [9, 2]
+    assert r.full.tolist() == [0, 1, 0]                 # 9 + 2 > 10: no room
+    assert lengths.tolist() == [8, 9, 4]
+    assert tokens[0, 5:8].tolist() == [3, 5, 4] and (tokens[1] == t0[1]).all()
+    assert (reps[0, 5] == node_reps[0, 0]).all() and (reps[0, 6] == node_reps[0, 1]).all()
+    assert (reps[0, 7] == node_reps[0, 2]).all() and (query[0] == node_reps[0, 2]).all()
+    assert (reps[1] == r0[1]).all() and (reps[2] == r0[2]).all()
