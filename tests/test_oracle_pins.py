@@ -680,3 +680,17 @@ def test_accept_appends_tokens_and_rows():
     assert (reps[0, 5] == node_reps[0, 0]).all() and (reps[0, 6] == node_reps[0, 1]).all()
     assert (reps[0, 7] == node_reps[0, 2]).all() and (query[0] == node_reps[0, 2]).all()
     assert (reps[1] == r0[1]).all() and (reps[2] == r0[2]).all()
+
+
+def test_accept_exact_fit():
+    """An append that fills the capacity exactly (len + n_new == ld) happens."""
+    tok = np.array([[7, 3, 5, 7, 9]], np.int32)
+    par = np.array([[-1, 0, 1, 2, 0]], np.int32)
+    lg = np.zeros((1, 5, 12), np.float32)
+    lg[0, 0, 3] = lg[0, 1, 5] = lg[0, 2, 4] = 1.0      # 3 new tokens
+    tokens = np.zeros((1, 10), np.int32)
+    lengths = np.array([7], np.int32)
+    r = oracle.accept_greedy(synth.f32_to_bf16_bits(lg), tok, par, np.array([5], np.int32),
+                             tokens, lengths)
+    assert r.full.tolist() == [0] and lengths.tolist() == [10]
+    assert tokens[0, 7:].tolist() == [3, 5, 4]
