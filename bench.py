@@ -45,6 +45,9 @@ def parse():
                     help="two-representation mode: token-embedding fallback (vocab x d table)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override B (profiling of small cases; not the headline workload)")
+    ap.add_argument("--verify", action="store_true",
+                    help="also time greedy verification of the step's trees against "
+                         "synthetic target logits [B][nodes][V]")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -347,6 +350,36 @@ def run_native(args):
     ms_per_step = total_ms / K
     value = job_throughput(world, K, total_ms)
 
+    # greedy verification (Sec. 3.6) of this step's trees against synthetic
+    # target logits; not part of the step (the target model sits in between)
+    verify = None
+    if args.verify:
+        V = synth.CONFIGS[cfg]["V"]
+        Bn, N = eng.out.draft_tokens.shape
+        gen = torch.Generator(device=dev)
+        gen.manual_seed(rank_seed(args.seed, rank))
+        logits = torch.randn((Bn, N, V), generator=gen, device=dev).to(torch.bfloat16)
+        n_acc = torch.empty(Bn, dtype=torch.int32, device=dev)
+        new_t = torch.empty((Bn, N), dtype=torch.int32, device=dev)
+        n_new = torch.empty(Bn, dtype=torch.int32, device=dev)
+        trees = (eng.out.draft_tokens, eng.out.parents, eng.out.n_nodes)
+        for _ in range(3):
+            native.accept_greedy(logits, *trees, n_acc, new_t, n_new, eng.ws)
+        v0 = torch.cuda.Event(enable_timing=True)
+        v1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        v0.record(stream)
+        for _ in range(K):
+            native.accept_greedy(logits, *trees, n_acc, new_t, n_new, eng.ws)
+        v1.record(stream)
+        torch.cuda.synchronize(dev)
+        vms = v0.elapsed_time(v1) / K
+        nodes = int(eng.out.n_nodes.sum().item())
+        vbytes = nodes * V * 2
+        verify = {"ms": vms, "logits_bytes": vbytes, "gbs": vbytes / (vms / 1000.0) / 1e9,
+                  "vocab": V, "nodes": nodes}
+        del logits
+
     # end-to-end through the public API from pinned host buffers
     e2e = None
     if not args.no_e2e and emb is None:
@@ -419,6 +452,7 @@ def run_native(args):
         "ms_per_step_with_stage_events": total_b_ms / K,
         "cpu_baseline": cpu,
         "e2e": e2e,
+        "verify": verify,
         "gpu_launches": (6 if emb is not None else 4) * K,
         "clocks": clk,
     }

@@ -56,7 +56,7 @@ typedef struct CUstream_st *adapld_stream_t;
 /* ---- status codes --------------------------------------------------------- */
 #define ADAPLD_OK 0
 #define ADAPLD_ERR_NULL (-1)          /* a required pointer is NULL            */
-#define ADAPLD_ERR_BATCH (-2)         /* B < 1                                 */
+#define ADAPLD_ERR_BATCH (-2)         /* B outside [1, 65535]                  */
 #define ADAPLD_ERR_NMAX (-3)          /* n_max outside [1, 8]                  */
 #define ADAPLD_ERR_K (-4)             /* k outside [1, 32]                     */
 #define ADAPLD_ERR_WIDTH (-5)         /* branch_width outside [0, 64]          */
@@ -74,6 +74,8 @@ typedef struct CUstream_st *adapld_stream_t;
 #define ADAPLD_ERR_EMBEDDINGS (-16)   /* embedding table NULL or misaligned,
                                          vocab < 1, or dim not a multiple of 8
                                          in [8, 16384]                        */
+#define ADAPLD_ERR_VOCAB (-17)        /* V < 8 or V % 8 != 0, or logits not
+                                         16-byte aligned                      */
 #define ADAPLD_ERR_CUDA (-20)         /* a CUDA runtime call failed            */
 
 /* ---- retrieval outcome per sequence (Eq. 5, Algorithm 1) ------------------- */
@@ -88,6 +90,8 @@ typedef struct CUstream_st *adapld_stream_t;
                                       sequence is treated as retrieving nothing */
 #define ADAPLD_SEQ_BAD_TOKEN 4 /* a token id outside [0, vocab) met the
                                   embedding table: row 0 was used instead */
+#define ADAPLD_SEQ_FULL 8      /* adapld_accept_greedy(): the append would
+                                  pass ld, nothing was appended          */
 
 /* ---- device status bits (adapld_read_device_status) ------------------------ */
 #define ADAPLD_DEV_TIMEOUT 1  /* a bounded wait in a kernel expired; that
@@ -358,6 +362,44 @@ int adapld_semantic_topk_static(const uint16_t *reps, int64_t ld, int32_t d,
                                 const uint8_t *active, int32_t B, int32_t k, float tau,
                                 int32_t *cand, float *score, int32_t *n_cand,
                                 adapld_stream_t stream);
+
+/*
+ * Greedy verification of the draft trees and the append to the memory
+ * (Sec. 3.6; Appendix C, Eq. 16: at temperature 0 a draft token is accepted
+ * iff it equals the target model's greedy choice; Algorithm 1,
+ * VerifyAndAccept and the append).  The target model itself is the caller's.
+ *   logits [B][N][V] bf16: the target's next-token logits after each tree
+ *            node (tree-attention forward); rows of nodes >= n_nodes[b] are
+ *            not read.  V % 8 == 0, 16-byte aligned, no NaN.
+ *   draft_tokens, parents [B][N], n_nodes [B]: the trees (adapld_tree_out);
+ *            node 0 is the root; parents[0] is not read.
+ *   The choice at a node is the first index of its maximum logit.  From the
+ *   root, the child whose token equals the choice at the current node is
+ *   accepted (the first such child in node order), until there is none.
+ *   n_accept [B]       accepted draft tokens
+ *   new_tokens [B][N]  accepted draft tokens, then the choice after the last
+ *                      accepted node (the bonus token); padding -1
+ *   n_new [B]          n_accept + 1 (0 for an empty tree)
+ * Append (tokens == NULL skips it; tokens and lengths go together): the new
+ * tokens go to tokens[b][len_b ..] and lengths[b] grows by n_new.  If
+ * node_reps ([B][N][d] bf16: the hidden state after each tree node, from the
+ * same forward) is given, reps rows len_b .. len_b+n_new-1 receive the states
+ * of the root and of the accepted nodes (row j holds the state after token
+ * j-1) and query[b] the state after the last accepted node; reps and query
+ * are then required and d valid.  A sequence whose append would pass ld gets
+ * ADAPLD_SEQ_FULL in status [B] (nullable) and no append; one with
+ * lengths[b] outside [0, ld] gets ADAPLD_SEQ_BAD_LENGTH and no append (the
+ * verification outputs are still written).  Uses the verification part of a
+ * workspace from adapld_workspace_bytes() for the same B (any ld, d and
+ * parameters); N <= 1024.  Calls sharing a workspace must not overlap.
+ */
+int adapld_accept_greedy(const uint16_t *logits, int32_t V, const int32_t *draft_tokens,
+                         const int32_t *parents, const int32_t *n_nodes, int32_t B, int32_t N,
+                         int32_t *n_accept, int32_t *new_tokens, int32_t *n_new,
+                         int32_t *tokens, int64_t ld, int32_t *lengths,
+                         const uint16_t *node_reps, uint16_t *reps, int32_t d,
+                         uint16_t *query, int32_t *status, void *ws, size_t ws_bytes,
+                         adapld_stream_t stream);
 
 /* Synchronises `stream` and returns in *status the ADAPLD_DEV_* bits raised by
  * the most recent call that used workspace `ws` (0 = none). */

@@ -26,7 +26,7 @@ int check_params(const adapld_params *p) {
 }
 
 int check_shape(int32_t B, int64_t ld) {
-    if (B < 1) return ADAPLD_ERR_BATCH;
+    if (B < 1 || B > 65535) return ADAPLD_ERR_BATCH;
     if (ld < 1) return ADAPLD_ERR_LD;
     if ((int64_t)B * ld >= ((int64_t)1 << 31)) return ADAPLD_ERR_TOO_LARGE;
     return ADAPLD_OK;
@@ -83,7 +83,7 @@ const char *adapld_status_string(int code) {
     switch (code) {
         case ADAPLD_OK: return "ok";
         case ADAPLD_ERR_NULL: return "a required pointer is NULL";
-        case ADAPLD_ERR_BATCH: return "batch size B must be >= 1";
+        case ADAPLD_ERR_BATCH: return "batch size B must be in [1, 65535]";
         case ADAPLD_ERR_NMAX: return "n_max must be in [1, 8]";
         case ADAPLD_ERR_K: return "k must be in [1, 32]";
         case ADAPLD_ERR_WIDTH: return "branch_width must be in [0, 64]";
@@ -98,6 +98,7 @@ const char *adapld_status_string(int code) {
         case ADAPLD_ERR_TAU: return "tau must not be NaN";
         case ADAPLD_ERR_STATIC_LIMIT: return "B exceeds ADAPLD_STATIC_MAX_B (1024) for the workspace-free entry point";
         case ADAPLD_ERR_EMBEDDINGS: return "embedding table NULL or misaligned, vocab < 1, or dim not a multiple of 8 in [8, 16384]";
+        case ADAPLD_ERR_VOCAB: return "V must be a positive multiple of 8 and logits 16-byte aligned";
         case ADAPLD_ERR_CUDA: return "a CUDA runtime call failed";
         default: return "unknown status";
     }
@@ -248,6 +249,35 @@ int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const
                 adapld_stream_t stream) {
     return adapld_step_ex(tokens, ld, lengths, reps, d, query, next_topk, Kn, B, p, out, ws,
                           ws_bytes, nullptr, nullptr, stream);
+}
+
+int adapld_accept_greedy(const uint16_t *logits, int32_t V, const int32_t *draft_tokens,
+                         const int32_t *parents, const int32_t *n_nodes, int32_t B, int32_t N,
+                         int32_t *n_accept, int32_t *new_tokens, int32_t *n_new,
+                         int32_t *tokens, int64_t ld, int32_t *lengths,
+                         const uint16_t *node_reps, uint16_t *reps, int32_t d,
+                         uint16_t *query, int32_t *status, void *ws, size_t ws_bytes,
+                         adapld_stream_t stream) {
+    if (!logits || !draft_tokens || !parents || !n_nodes || !n_accept || !new_tokens || !n_new)
+        return ADAPLD_ERR_NULL;
+    if (B < 1 || B > 65535) return ADAPLD_ERR_BATCH;
+    if (N < 1 || N > kMaxNodes) return ADAPLD_ERR_TOO_LARGE;
+    if (V < 8 || (V % 8) != 0 || !aligned16(logits)) return ADAPLD_ERR_VOCAB;
+    if ((tokens == nullptr) != (lengths == nullptr)) return ADAPLD_ERR_NULL;
+    if (tokens && ld < 1) return ADAPLD_ERR_LD;
+    if (node_reps) {
+        if (!tokens || !reps || !query) return ADAPLD_ERR_NULL;
+        ADAPLD_TRY(check_dim(d));
+        if (!aligned16(node_reps) || !aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
+    }
+    // the layout for ld = 1 and W = 1, which every workspace for this B covers
+    ADAPLD_TRY(check_ws(ws, ws_bytes, B, 1, 1));
+    const Workspace w = layout_workspace(ws, B, 1, 1);
+    cudaStream_t s = (cudaStream_t)stream;
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    VerifyLaunch a{logits, V, draft_tokens, parents, n_nodes, B, N, n_accept, new_tokens, n_new,
+                   tokens, ld, lengths, node_reps, reps, d, query, status};
+    return cuda_status(launch_verify(a, w, s));
 }
 
 int adapld_read_device_status(const void *ws, int32_t *status, adapld_stream_t stream) {

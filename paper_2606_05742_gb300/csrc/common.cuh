@@ -36,6 +36,7 @@ struct Workspace {
     int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
     int32_t *npairs;         // [1]  successor backoff: (sequence, branch) pairs
     int32_t *gticket4;       // [1]  successor scan: sequences done
+    int32_t *vticket;        // [B]  verification: node CTAs done per sequence
     int32_t *done3;          // [B*W] successor backoff: CTAs done per pair
     int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
     int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
@@ -52,6 +53,7 @@ struct Workspace {
     int32_t *pair_tok;       // [B*W] its branch token (the query anchor)
     int32_t *pair_out;       // [B*W] its row b*W + w in succ / succ_n
     float *succ_es;          // [B*W][kMaxK] backoff candidates' embedding scores
+    int32_t *vtarget;        // [B][kMaxNodes] verification: the target's choice per node
     size_t counters_bytes;
     size_t total_bytes;
     int C1, S4, W;
@@ -77,7 +79,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         return r;
     };
     const size_t BW = (size_t)B * w.W;
-    w.counters_bytes = sizeof(int32_t) * (4 + 4 * (size_t)B + BW);
+    w.counters_bytes = sizeof(int32_t) * (4 + 5 * (size_t)B + BW);
     w.dev_status = (int32_t *)take(w.counters_bytes);
     if (p) {
         w.global_ticket = w.dev_status + 1;
@@ -87,7 +89,8 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         w.done2 = w.ticket1 + B;
         w.ticket4 = w.done2 + B;
         w.ticket5 = w.ticket4 + B;
-        w.done3 = w.ticket5 + B;
+        w.vticket = w.ticket5 + B;
+        w.done3 = w.vticket + B;
     }
     w.part1 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1 * kPart1Ints);
     w.plan = (int64_t *)take(sizeof(int64_t) * ((size_t)B + 1));
@@ -104,6 +107,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.pair_tok = (int32_t *)take(sizeof(int32_t) * BW);
     w.pair_out = (int32_t *)take(sizeof(int32_t) * BW);
     w.succ_es = (float *)take(sizeof(float) * BW * kMaxK);
+    w.vtarget = (int32_t *)take(sizeof(int32_t) * (size_t)B * kMaxNodes);
     w.total_bytes = off;
     return w;
 }
@@ -413,5 +417,22 @@ struct TreeLaunch {
     adapld_embeddings emb = {nullptr, 0, 0};  // token embeddings (two-representation mode)
 };
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s);
+
+struct VerifyLaunch {
+    const uint16_t *logits;  // [B][N][V] bf16
+    int32_t V;
+    const int32_t *draft_tokens, *parents, *n_nodes;
+    int32_t B, N;
+    int32_t *n_accept, *new_tokens, *n_new;
+    int32_t *tokens;         // append (nullable, with lengths)
+    int64_t ld;
+    int32_t *lengths;
+    const uint16_t *node_reps;  // [B][N][d] (nullable)
+    uint16_t *reps;
+    int32_t d;
+    uint16_t *query;
+    int32_t *status;         // nullable
+};
+cudaError_t launch_verify(const VerifyLaunch &a, const Workspace &ws, cudaStream_t s);
 
 }  // namespace adapld

@@ -27,6 +27,7 @@ NO_SUCC = 16
 SEQ_BAD_LENGTH = 1
 SEQ_BAD_CANDIDATE = 2
 SEQ_BAD_TOKEN = 4
+SEQ_FULL = 8
 DEV_TIMEOUT = 1
 DEV_INTERNAL = 2
 
@@ -34,7 +35,7 @@ EXPORTED = [
     "adapld_tree_nodes", "adapld_workspace_bytes", "adapld_status_string",
     "adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
     "adapld_step", "adapld_step_ex", "adapld_read_device_status",
-    "adapld_semantic_topk_static", "adapld_embedding_topk",
+    "adapld_semantic_topk_static", "adapld_embedding_topk", "adapld_accept_greedy",
 ]
 STATIC_MAX_B = 1024
 ERR_STATIC_LIMIT = -15
@@ -120,9 +121,12 @@ def load() -> ctypes.CDLL:
         lib.adapld_read_device_status.argtypes = [P, P, P]
         lib.adapld_semantic_topk_static.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P,
                                                     P, P]
+        lib.adapld_accept_greedy.argtypes = [P, i32, P, P, P, i32, i32, P, P, P, P, i64, P, P,
+                                             P, i32, P, P, P, sz, P]
         for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
                   "adapld_step", "adapld_step_ex", "adapld_read_device_status",
-                  "adapld_semantic_topk_static", "adapld_embedding_topk"):
+                  "adapld_semantic_topk_static", "adapld_embedding_topk",
+                  "adapld_accept_greedy"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -295,6 +299,23 @@ def step(tokens, lengths, reps, query, p: Params, out: Outputs, ws, next_topk=No
                                 ctypes.byref(events) if events is not None else None,
                                 _stream(stream))
     _check(rc, "adapld_step")
+
+
+def accept_greedy(logits, draft_tokens, parents, n_nodes, n_accept, new_tokens, n_new, ws,
+                  tokens=None, lengths=None, node_reps=None, reps=None, query=None,
+                  status=None, stream=None) -> None:
+    """Greedy tree verification and the memory append (adapld_accept_greedy).
+    logits [B][N][V] bf16; optional append into tokens/lengths (and, with
+    node_reps [B][N][d], reps/query)."""
+    B, N, V = logits.shape
+    ld = tokens.shape[1] if tokens is not None else 0
+    d = node_reps.shape[2] if node_reps is not None else 0
+    rc = load().adapld_accept_greedy(
+        _ptr(logits), V, _ptr(draft_tokens), _ptr(parents), _ptr(n_nodes), B, N, _ptr(n_accept),
+        _ptr(new_tokens), _ptr(n_new), _ptr(tokens), ld, _ptr(lengths), _ptr(node_reps),
+        _ptr(reps), d, _ptr(query), _ptr(status), _ptr(ws), ws.numel() * ws.element_size(),
+        _stream(stream))
+    _check(rc, "adapld_accept_greedy")
 
 
 def read_device_status(ws, stream=None) -> int:

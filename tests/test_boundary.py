@@ -40,7 +40,8 @@ def test_library_exports_every_declared_symbol(lib):
 
 
 def test_status_strings(lib):
-    for code in (0, -1, -2, -3, -4, -5, -6, -7, -8, -9, -10, -11, -12, -13, -14, -15, -16, -20):
+    for code in (0, -1, -2, -3, -4, -5, -6, -7, -8, -9, -10, -11, -12, -13, -14, -15, -16, -17,
+                 -20):
         s = native.status_string(code)
         assert s and s != "unknown status"
     assert native.status_string(-999) == "unknown status"
@@ -77,6 +78,7 @@ def _step(lib, **kw):
     (dict(tokens=None), -1),
     (dict(reps=None), -1),
     (dict(B=0), -2),
+    (dict(B=65536, ld=1), -2),
     (dict(p=native.make_params(0, 8, 2, 8)), -3),
     (dict(p=native.make_params(9, 8, 2, 8)), -3),
     (dict(p=native.make_params(3, 0, 2, 8)), -4),
@@ -153,6 +155,40 @@ def test_entry_point_argument_errors(lib):
                                    FAKE, FAKE, None, FAKE, 1 << 30, None) == -4
     v = ctypes.c_int32(0)
     assert L.adapld_read_device_status(None, ctypes.byref(v), None) == -1
+
+
+def _accept(lib, **kw):
+    a = dict(logits=FAKE, V=64, draft_tokens=FAKE, parents=FAKE, n_nodes=FAKE, B=2, N=8,
+             n_accept=FAKE, new_tokens=FAKE, n_new=FAKE, tokens=None, ld=0, lengths=None,
+             node_reps=None, reps=None, d=0, query=None, status=None, ws=FAKE,
+             ws_bytes=1 << 30)
+    a.update(kw)
+    return lib.adapld_accept_greedy(*a.values(), None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(logits=None), -1),
+    (dict(n_new=None), -1),
+    (dict(tokens=FAKE), -1),                       # tokens without lengths
+    (dict(lengths=FAKE), -1),
+    (dict(tokens=FAKE, lengths=FAKE, ld=16, node_reps=FAKE, d=16), -1),  # no reps/query
+    (dict(B=0), -2),
+    (dict(B=65536), -2),
+    (dict(N=0), -11),
+    (dict(N=1025), -11),
+    (dict(V=0), -17),
+    (dict(V=60), -17),
+    (dict(logits=FAKE + 2), -17),
+    (dict(tokens=FAKE, lengths=FAKE, ld=0), -10),
+    (dict(tokens=FAKE, lengths=FAKE, ld=16, node_reps=FAKE, reps=FAKE, query=FAKE, d=12), -7),
+    (dict(tokens=FAKE, lengths=FAKE, ld=16, node_reps=FAKE + 8, reps=FAKE, query=FAKE, d=16),
+     -8),
+    (dict(ws=None), -9),
+    (dict(ws_bytes=64), -9),
+    (dict(ws=FAKE + 4), -8),
+])
+def test_accept_argument_errors(lib, kw, code):
+    assert _accept(lib, **kw) == code
 
 
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
