@@ -48,6 +48,9 @@ def parse():
     ap.add_argument("--verify", action="store_true",
                     help="also time greedy verification of the step's trees against "
                          "synthetic target logits [B][nodes][V]")
+    ap.add_argument("--flags", default="",
+                    help="ablation variants (Table 4), comma-separated: no_lex_rerank, "
+                         "succ_on_strict, no_semantic, no_branch, no_succ")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -198,21 +201,52 @@ class OracleSample:
                + self.n_hit * t[self.hit] * self.L / self.rows)
         return 1.0 / est
 
+    def rate_parallel(self, threads: int) -> float:
+        """The same oracle over a whole batch of truncated sequences (n_miss
+        copies of the miss, n_hit of the hit), one sequence per task on a
+        pool of ``threads`` host threads (the C oracle runs outside the GIL),
+        wall time extrapolated linearly to full length."""
+        import concurrent.futures as cf
+
+        import oracle
+        w = self.w
+        seqs = [self.miss] * self.n_miss + [self.hit] * self.n_hit
+
+        def one(b):
+            oracle.step(w.tokens[b:b + 1], w.lengths[b:b + 1], w.reps[b:b + 1],
+                        w.query[b:b + 1], w.n_max, w.k, w.W, w.D, w.succ_len, w.tau)
+
+        with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+            s = time.perf_counter()
+            list(ex.map(one, seqs))
+            wall = time.perf_counter() - s
+        return 1.0 / (wall * (self.L - 1) / (self.rows - 1))
+
+    def parallel_desc(self, threads: int) -> str:
+        plural = "s" if threads > 1 else ""
+        return self.desc.replace("oracle (1 thread)", f"oracle ({threads} thread{plural}, one "
+                                 "sequence per task)") + " (wall time of the batch)"
+
+
+def host_threads(batch: int) -> int:
+    return max(1, min(batch, os.cpu_count() or 1))
+
 
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
     sample = OracleSample(args.config, args.seed, rows=4096)
+    threads = host_threads(sample.n_miss + sample.n_hit)
     for _ in range(args.warmup):
-        sample.rate()
+        sample.rate_parallel(threads)
     vals = []
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        vals.append(sample.rate())
+        vals.append(sample.rate_parallel(threads))
         if time.perf_counter() - t0 > 150:
             break
-    desc = sample.desc
+    desc = sample.parallel_desc(threads)
     value = statistics.median(vals)
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
@@ -220,7 +254,7 @@ def run_reference(args):
         "ms_per_step": 1000.0 / value, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(args.config),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
                          "sample": desc},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
@@ -236,26 +270,51 @@ def workload_config(cfg_id):
 
 
 # ---------------------------------------------------------- native arm
-def algorithmic_bytes(w, g, lengths, tokens):
+FLAG_NAMES = {"no_lex_rerank": 1, "succ_on_strict": 2, "no_semantic": 4, "no_branch": 8,
+              "no_succ": 16}
+
+
+def parse_flags(text):
+    flags = 0
+    for name in filter(None, (x.strip().lower() for x in text.split(","))):
+        if name not in FLAG_NAMES:
+            raise SystemExit(f"unknown flag {name!r}; known: {', '.join(FLAG_NAMES)}")
+        flags |= FLAG_NAMES[name]
+    return flags
+
+
+def step_launches(flags, W, emb):
+    """Kernels one step launches (mirrors the launch sequence of adapld_step)."""
+    succ = W > 0 and not (flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"]))
+    n = 2 + (0 if flags & FLAG_NAMES["no_semantic"] else 1) + (1 if succ else 0)
+    if emb and succ:
+        n += 2                              # backoff plan + gathered semantic pass
+    return n
+
+
+def algorithmic_bytes(w, g, lengths, tokens, flags=0):
     """Bytes the step must move at minimum (no re-reads), per kernel."""
     d, k = w.d, w.k
     hk = g["hit_kind"]
-    active = hk != 1
+    semantic = not flags & FLAG_NAMES["no_semantic"]
+    active = (hk != 1) & semantic
     lex_bytes = int(4 * lengths.sum())
     sem_rows = int(sum(lengths[b] - 1 for b in range(w.B) if active[b] and lengths[b] >= 2))
     n_active = int(active.sum())
-    sem_bytes = sem_rows * d * 2 + n_active * d * 2 + 4 * w.B
+    sem_bytes = (sem_rows * d * 2 + n_active * d * 2 + 4 * w.B) if semantic else 0
     # tree kernel: rerank rows + query for lexical hits, successor scan + rows
+    succ_on = w.W > 0 and not flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"])
     gathered = 0
     succ_scan = 0
     for b in range(w.B):
         L = int(lengths[b])
-        if hk[b] == 1:
+        if hk[b] == 1 and not flags & FLAG_NAMES["no_lex_rerank"]:
             gathered += int(g["n_cand"][b]) + 1
-        elif hk[b] == 2:
+        if succ_on and (hk[b] == 2 or (hk[b] == 1 and flags & FLAG_NAMES["succ_on_strict"])):
             n = int(g["n_nodes"][b])
             par = g["parents"][b, :n]
-            heads = [i for i in range(1, n) if par[i] == 0]
+            # branch heads hang off the root; on a lexical hit node 1 is main[0]
+            heads = [i for i in range(1, n) if par[i] == 0 and not (hk[b] == 1 and i == 1)]
             succ_scan += 4 * (L - 1)
             gathered += 1
             for h in heads:
@@ -274,6 +333,7 @@ def run_native(args):
 
     from paper_2606_05742_gb300 import native, synth
 
+    flags = parse_flags(args.flags)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
@@ -289,7 +349,7 @@ def run_native(args):
 
     cfg = args.config
     w = synth.make_workload(cfg, device=str(dev), seed=rank_seed(args.seed, rank), B=args.batch)
-    p = native.make_params(w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, 0)
+    p = native.make_params(w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, flags)
     eng = native.Engine(w.B, w.ld, w.d, p, device=dev)
     stream = torch.cuda.current_stream(dev)
     emb = None
@@ -304,7 +364,7 @@ def run_native(args):
     g = eng.out.to_host()
     lengths = w.lengths.cpu().numpy()
     tokens = w.tokens.cpu().numpy()
-    nbytes = algorithmic_bytes(w, g, lengths, tokens)
+    nbytes = algorithmic_bytes(w, g, lengths, tokens, flags)
 
     # Timed region A (the headline): K steps back to back, CUDA events only at
     # the two ends, so consecutive kernels keep their programmatic-launch
@@ -343,9 +403,14 @@ def run_native(args):
     total_b_ms = startb.elapsed_time(endb)
     if native.read_device_status(eng.ws) != 0:
         raise RuntimeError("device status raised during the timed region")
+    semantic_on = not flags & FLAG_NAMES["no_semantic"]
     stage = {name: [r[2 * i].elapsed_time(r[2 * i + 1]) for r in ev]
-             for i, name in enumerate(("lexical", "semantic", "tree"))}
-    sem_ms = stage["semantic"]
+             for i, name in enumerate(("lexical", "semantic", "tree"))
+             if name != "semantic" or semantic_on}
+    # the dominant kernel: the semantic top-k, or without it the tree stage
+    dom_name, dom_kernel = (("semantic", "semantic_kernel") if semantic_on
+                            else ("tree", "succ_scan_kernel + tree_kernel"))
+    sem_ms = stage[dom_name]
     total_ms = max_over_ranks(total_ms, dev)
     ms_per_step = total_ms / K
     value = job_throughput(world, K, total_ms)
@@ -365,19 +430,24 @@ def run_native(args):
         trees = (eng.out.draft_tokens, eng.out.parents, eng.out.n_nodes)
         for _ in range(3):
             native.accept_greedy(logits, *trees, n_acc, new_t, n_new, eng.ws)
-        v0 = torch.cuda.Event(enable_timing=True)
-        v1 = torch.cuda.Event(enable_timing=True)
+        # events around each call: the device time of one call (counter
+        # reset + kernel), whatever the host takes to issue the next one
+        vev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(K)]
+        for e0, e1 in vev:
+            e0.record(stream)
+            e1.record(stream)
         torch.cuda.synchronize(dev)
-        v0.record(stream)
-        for _ in range(K):
+        for e0, e1 in vev:
+            e0.record(stream)
             native.accept_greedy(logits, *trees, n_acc, new_t, n_new, eng.ws)
-        v1.record(stream)
+            e1.record(stream)
         torch.cuda.synchronize(dev)
-        vms = v0.elapsed_time(v1) / K
+        vms = statistics.median(e0.elapsed_time(e1) for e0, e1 in vev)
         nodes = int(eng.out.n_nodes.sum().item())
         vbytes = nodes * V * 2
         verify = {"ms": vms, "logits_bytes": vbytes, "gbs": vbytes / (vms / 1000.0) / 1e9,
-                  "vocab": V, "nodes": nodes}
+                  "vocab": V, "nodes": nodes, "timing": "median over calls of per-call events"}
         del logits
 
     # end-to-end through the public API from pinned host buffers
@@ -417,18 +487,25 @@ def run_native(args):
 
     peak, peak_kind = peaks()
     sem_avg_ms = sum(sem_ms) / len(sem_ms)
-    achieved = nbytes["semantic"] / (sem_avg_ms / 1000.0) / 1e9
+    achieved = nbytes[dom_name] / (sem_avg_ms / 1000.0) / 1e9
     step_gbs = nbytes["step"] / (ms_per_step / 1000.0) / 1e9
     cpu = None
     if not args.no_cpu_baseline:
-        sample = OracleSample(cfg, args.seed, rows=16384)
-        v = statistics.median([sample.rate() for _ in range(3)])
-        cpu = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample.desc}
+        sample = OracleSample(cfg, args.seed, rows=65536)
+        threads = host_threads(sample.n_miss + sample.n_hit)
+        v1 = statistics.median([sample.rate() for _ in range(3)])
+        vp = statistics.median([sample.rate_parallel(threads) for _ in range(3)])
+        cpu = {"value": vp, "unit": UNIT, "cores": threads, "kind": "oracle",
+               "sample": sample.parallel_desc(threads), "value_1_thread": v1,
+               "sample_1_thread": sample.desc}
     hk = g["hit_kind"]
     conf = workload_config(cfg)
     if emb is not None:
         conf["workload"] += (f" + token-embedding fallback ({emb.shape[0]} x {emb.shape[1]} "
                              "table; two-representation mode)")
+    if flags:
+        conf["workload"] += f" ablation: {args.flags}"
+        conf["flags"] = flags
     if args.batch is not None:
         conf["workload"] += f" (resized: B={w.B})"
         conf["B"] = conf["global_batch"] = w.B
@@ -441,11 +518,12 @@ def run_native(args):
         "warmup": max(3, args.warmup), "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": conf,
-        "roofline": {"bound": "hbm", "kernel": "semantic_kernel",
+        "roofline": {"bound": "hbm", "kernel": dom_kernel,
                      "achieved": achieved, "peak": peak, "peak_kind": peak_kind,
                      "unit": "GB/s", "frac": achieved / peak,
-                     "traffic": semantic_traffic(nbytes["semantic"]) if emb is None else None,
-                     "algorithmic_bytes": nbytes["semantic"], "avg_launch_ms": sem_avg_ms},
+                     "traffic": (semantic_traffic(nbytes["semantic"])
+                                 if emb is None and semantic_on else None),
+                     "algorithmic_bytes": nbytes[dom_name], "avg_launch_ms": sem_avg_ms},
         "step_hbm": {"achieved": step_gbs, "frac": step_gbs / peak,
                      "algorithmic_bytes": nbytes["step"]},
         "stage_ms": {name: sum(v) / len(v) for name, v in stage.items()},
@@ -453,7 +531,7 @@ def run_native(args):
         "cpu_baseline": cpu,
         "e2e": e2e,
         "verify": verify,
-        "gpu_launches": (6 if emb is not None else 4) * K,
+        "gpu_launches": step_launches(flags, w.W, emb is not None) * K,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

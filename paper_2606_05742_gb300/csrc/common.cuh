@@ -36,7 +36,7 @@ struct Workspace {
     int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
     int32_t *npairs;         // [1]  successor backoff: (sequence, branch) pairs
     int32_t *gticket4;       // [1]  successor scan: sequences done
-    int32_t *vticket;        // [B]  verification: node CTAs done per sequence
+    int32_t *vticket;        // [B]  verification: CTAs done per sequence
     int32_t *done3;          // [B*W] successor backoff: CTAs done per pair
     int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
     int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
@@ -53,7 +53,8 @@ struct Workspace {
     int32_t *pair_tok;       // [B*W] its branch token (the query anchor)
     int32_t *pair_out;       // [B*W] its row b*W + w in succ / succ_n
     float *succ_es;          // [B*W][kMaxK] backoff candidates' embedding scores
-    int32_t *vtarget;        // [B][kMaxNodes] verification: the target's choice per node
+    unsigned long long *vpart;  // [B][N][S], N*S <= kMaxNodes: verification, packed
+                                //   (logit, index) maximum per node and row split
     size_t counters_bytes;
     size_t total_bytes;
     int C1, S4, W;
@@ -107,7 +108,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.pair_tok = (int32_t *)take(sizeof(int32_t) * BW);
     w.pair_out = (int32_t *)take(sizeof(int32_t) * BW);
     w.succ_es = (float *)take(sizeof(float) * BW * kMaxK);
-    w.vtarget = (int32_t *)take(sizeof(int32_t) * (size_t)B * kMaxNodes);
+    w.vpart = (unsigned long long *)take(sizeof(unsigned long long) * (size_t)B * kMaxNodes);
     w.total_bytes = off;
     return w;
 }

@@ -3,15 +3,21 @@
 // iff it equals the target model's greedy choice; Algorithm 1 appends the
 // accepted tokens and the bonus token).
 //
-// verify_kernel, grid (N nodes, B), 512 threads.  CTA (i, b) streams the
-// target's next-token logits after node i (V bf16, 16-byte loads) and keeps
-// the first index of the maximum; CTAs of nodes >= n_nodes[b] exit.  The last
-// CTA of a sequence (atomic ticket) loads the tree and the choices into
-// shared memory, walks from the root with warp ballots (the child whose token
-// equals the choice at the current node), writes the new tokens (accepted
-// draft tokens, then the choice after the last accepted node) and appends
-// them, with the hidden states of the root and the accepted nodes, to the
-// memory.
+// The work is the argmax of every tree node's logit row (N rows of V bf16
+// per sequence, HBM-bound), then a walk over at most N nodes.
+//
+// verify_kernel, grid (S splits, N nodes, B), 256 threads.  CTA (s, i, b)
+// reads split s of node i's row in 32 KB groups (8 independent 16-byte
+// loads per thread, all issued before any is used; groups s, s + S, ...)
+// and keeps the first index of the maximum, stored as a 64-bit key that
+// orders by value, then by the smaller index (S <= 1024 / N keeps the
+// partial keys within the workspace).  CTAs of nodes >= n_nodes[b] exit at
+// once.  The last CTA of a sequence (atomic ticket over n_nodes[b] x S CTAs)
+// takes the largest key per node, loads the tree into shared memory,
+// walks from the root with warp ballots (the child whose token equals the
+// choice at the current node), writes the new tokens (accepted draft tokens,
+// then the choice after the last accepted node) and appends them, with the
+// hidden states of the root and the accepted nodes, to the memory.
 #include <climits>
 
 #include "common.cuh"
@@ -20,16 +26,50 @@ namespace adapld {
 
 namespace {
 
-constexpr int kThreadsV = 512;
+constexpr int kThreadsV = 256;
+constexpr int kLoadsV = 8;                          // 16-byte loads per thread
+constexpr int kChunksV = kThreadsV * kLoadsV;       // 16-byte chunks per CTA (32 KB)
 
 struct VerifyArgs {
     VerifyLaunch p;
     Workspace ws;
+    int S;  // splits per row
 };
 
 // (value, index) order of the choice: higher value, then the smaller index.
 __device__ __forceinline__ bool beats(float va, int ia, float vb, int ib) {
     return va > vb || (va == vb && ia < ib);
+}
+
+// A key whose unsigned order is the choice order: the value's bits made
+// monotone (negative values inverted, positive ones offset by the sign bit;
+// -0 folded onto +0 so that the two tie), then the complemented index.
+// Never 0 for a non-NaN value, so 0 means "no value yet".
+__device__ __forceinline__ unsigned long long choice_key(float v, int i) {
+    uint32_t u = __float_as_uint(v == 0.0f ? 0.0f : v);
+    u = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+    return ((unsigned long long)u << 32) | (0xffffffffu - (uint32_t)i);
+}
+
+// Index of a key; a row without a non-NaN value chooses index 0.
+__device__ __forceinline__ int key_index(unsigned long long key) {
+    return key == 0ull ? 0 : (int)(0xffffffffu - (uint32_t)(key & 0xffffffffull));
+}
+
+__device__ __forceinline__ void take8(uint4 w, int i0, float &bv, int &bi) {
+    const uint32_t w4[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float lo = bf16lo(w4[e]), hi = bf16hi(w4[e]);
+        if (beats(lo, i0 + 2 * e, bv, bi)) {
+            bv = lo;
+            bi = i0 + 2 * e;
+        }
+        if (beats(hi, i0 + 2 * e + 1, bv, bi)) {
+            bv = hi;
+            bi = i0 + 2 * e + 1;
+        }
+    }
 }
 
 __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
@@ -41,14 +81,13 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
     __shared__ int s_path[kMaxNodes];
     __shared__ int s_flag, s_nacc;
 
-    pdl_wait_then_release();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    const int node = blockIdx.x, b = blockIdx.y;
-    const int N = a.N, V = a.V;
+    const int split = blockIdx.x, node = blockIdx.y, b = blockIdx.z;
+    const int N = a.N, V = a.V, S = args.S;
     const int n = min(a.n_nodes[b], N);
     int32_t *new_b = a.new_tokens + (int64_t)b * N;
     if (n <= 0) {  // an empty tree: nothing to verify or append
-        if (node == 0) {
+        if (node == 0 && split == 0) {
             for (int i = t; i < N; i += kThreadsV) new_b[i] = -1;
             if (t == 0) {
                 a.n_accept[b] = 0;
@@ -60,25 +99,22 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
     }
     if (node >= n) return;
 
-    // ---- the target's choice after this node: first index of the maximum
+    // ---- this split of the target's row after the node: first index of the maximum
     const uint16_t *row = a.logits + ((int64_t)b * N + node) * V;
+    const int nch = V >> 3;
     float bv = -INFINITY;
     int bi = INT_MAX;
-    for (int ch = t; ch < (V >> 3); ch += kThreadsV) {
-        const uint4 w = ldg_nc_v4(row + (size_t)ch * 8);
-        const uint32_t w4[4] = {w.x, w.y, w.z, w.w};
+    for (int c0 = split * kChunksV; c0 < nch; c0 += S * kChunksV) {
+        uint4 w[kLoadsV];
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float lo = bf16lo(w4[e]), hi = bf16hi(w4[e]);
-            const int i0 = ch * 8 + 2 * e;
-            if (beats(lo, i0, bv, bi)) {
-                bv = lo;
-                bi = i0;
-            }
-            if (beats(hi, i0 + 1, bv, bi)) {
-                bv = hi;
-                bi = i0 + 1;
-            }
+        for (int u = 0; u < kLoadsV; ++u) {
+            const int ch = c0 + u * kThreadsV + t;
+            if (ch < nch) w[u] = ldg_nc_v4(row + (size_t)ch * 8);
+        }
+#pragma unroll
+        for (int u = 0; u < kLoadsV; ++u) {
+            const int ch = c0 + u * kThreadsV + t;
+            if (ch < nch) take8(w[u], ch * 8, bv, bi);
         }
     }
 #pragma unroll
@@ -96,14 +132,14 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
     }
     __syncthreads();
     if (t == 0) {
-        for (int w = 1; w < kThreadsV / 32; ++w)
-            if (beats(s_v[w], s_i[w], bv, bi)) {
-                bv = s_v[w];
-                bi = s_i[w];
+        for (int k = 1; k < kThreadsV / 32; ++k)
+            if (beats(s_v[k], s_i[k], bv, bi)) {
+                bv = s_v[k];
+                bi = s_i[k];
             }
-        ws.vtarget[(int64_t)b * kMaxNodes + node] = bi < V ? bi : 0;
+        ws.vpart[((int64_t)b * N + node) * S + split] = bi < V ? choice_key(bv, bi) : 0ull;
         __threadfence();
-        s_flag = atomicAdd(ws.vticket + b, 1) == n - 1;
+        s_flag = atomicAdd(ws.vticket + b, 1) == n * S - 1;
     }
     __syncthreads();
     if (!s_flag) return;
@@ -113,7 +149,10 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
     for (int i = t; i < n; i += kThreadsV) {
         s_tok[i] = a.draft_tokens[(int64_t)b * N + i];
         s_par[i] = a.parents[(int64_t)b * N + i];
-        s_tgt[i] = __ldcg(ws.vtarget + (int64_t)b * kMaxNodes + i);
+        const unsigned long long *kp = ws.vpart + ((int64_t)b * N + i) * S;
+        unsigned long long key = 0ull;
+        for (int j = 0; j < S; ++j) key = max(key, __ldcg(kp + j));
+        s_tgt[i] = key_index(key);
     }
     __syncthreads();
     if (warp == 0) {
@@ -161,11 +200,11 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
                 const int nch = a.d >> 3;
                 for (int idx = t; idx < n_new * nch; idx += kThreadsV) {
                     const int i = idx / nch, ch = idx % nch;
-                    const uint4 w = ldg_nc_v4(a.node_reps + ((int64_t)b * N + s_path[i]) * a.d +
+                    const uint4 r = ldg_nc_v4(a.node_reps + ((int64_t)b * N + s_path[i]) * a.d +
                                               (size_t)ch * 8);
-                    *(uint4 *)(a.reps + ((int64_t)b * a.ld + len + i) * a.d + (size_t)ch * 8) = w;
+                    *(uint4 *)(a.reps + ((int64_t)b * a.ld + len + i) * a.d + (size_t)ch * 8) = r;
                     if (i == n_new - 1)
-                        *(uint4 *)(a.query + (int64_t)b * a.d + (size_t)ch * 8) = w;
+                        *(uint4 *)(a.query + (int64_t)b * a.d + (size_t)ch * 8) = r;
                 }
             }
         }
@@ -182,8 +221,10 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
 }  // namespace
 
 cudaError_t launch_verify(const VerifyLaunch &a, const Workspace &ws, cudaStream_t s) {
-    VerifyArgs args{a, ws};
-    verify_kernel<<<dim3(a.N, a.B), kThreadsV, 0, s>>>(args);
+    const int groups = (int)(((int64_t)(a.V >> 3) + kChunksV - 1) / kChunksV);
+    const int S = max(1, min(groups, kMaxNodes / a.N));
+    VerifyArgs args{a, ws, S};
+    verify_kernel<<<dim3(S, a.N, a.B), kThreadsV, 0, s>>>(args);
     return cudaGetLastError();
 }
 

@@ -1,0 +1,73 @@
+"""Host-side helpers of bench.py (no GPU): ablation flag parsing, the launch
+count it reports, and the algorithmic byte count under each variant."""
+import numpy as np
+import pytest
+
+import bench
+from paper_2606_05742_gb300 import native
+
+
+def test_flag_names_match_the_library():
+    assert bench.FLAG_NAMES == {"no_lex_rerank": native.NO_LEX_RERANK,
+                                "succ_on_strict": native.SUCC_ON_STRICT,
+                                "no_semantic": native.NO_SEMANTIC,
+                                "no_branch": native.NO_BRANCH, "no_succ": native.NO_SUCC}
+    assert bench.parse_flags("") == 0
+    assert bench.parse_flags("no_succ, NO_BRANCH") == native.NO_SUCC | native.NO_BRANCH
+    with pytest.raises(SystemExit):
+        bench.parse_flags("no_such_flag")
+
+
+def test_step_launches():
+    assert bench.step_launches(0, 4, False) == 4          # lexical, semantic, scan, tree
+    assert bench.step_launches(0, 4, True) == 6           # + backoff plan + gathered pass
+    assert bench.step_launches(native.NO_SEMANTIC, 4, False) == 3
+    assert bench.step_launches(native.NO_SUCC, 4, True) == 3
+    assert bench.step_launches(native.NO_BRANCH | native.NO_SEMANTIC, 4, False) == 2
+    assert bench.step_launches(0, 0, False) == 3
+
+
+class _W:
+    B, d, k, W = 3, 16, 4, 2
+
+
+def test_algorithmic_bytes_by_variant():
+    L = 10
+    tokens = np.tile(np.arange(L, dtype=np.int32) % 5, (3, 1))
+    lengths = np.full(3, L, np.int32)
+    # sequence 0 lexical (3 candidates), 1 semantic, 2 nothing
+    g = {"hit_kind": np.array([1, 2, 0]), "n_cand": np.array([3, 2, 0]),
+         "n_nodes": np.array([4, 3, 1]),
+         "parents": np.array([[-1, 0, 1, 0], [-1, 0, 0, -1], [-1, -1, -1, -1]]),
+         "draft_tokens": np.array([[4, 0, 1, 2], [4, 1, 3, -1], [4, -1, -1, -1]])}
+    base = bench.algorithmic_bytes(_W, g, lengths, tokens)
+    assert base["lexical"] == 4 * 30
+    assert base["semantic"] == 2 * (9 * 16 * 2 + 16 * 2) + 4 * 3   # two sequences scan
+    no_sem = bench.algorithmic_bytes(_W, g, lengths, tokens, native.NO_SEMANTIC)
+    assert no_sem["semantic"] == 0
+    # rerank rows of the lexical hit: 3 candidates + the query
+    no_rr = bench.algorithmic_bytes(_W, g, lengths, tokens, native.NO_LEX_RERANK)
+    assert base["tree"] - no_rr["tree"] == 4 * 16 * 2
+    # successors of the semantic hit: scan 4*(L-1), the reference row, and
+    # min(k, occurrences) rows per branch head (tokens 1 and 3: 2 each in 0..8)
+    no_succ = bench.algorithmic_bytes(_W, g, lengths, tokens, native.NO_SUCC)
+    assert base["tree"] - no_succ["tree"] == 4 * 9 + (1 + 2 + 2) * 16 * 2
+    # text-rule successors add the lexical hit's branch head (node 3, token 2)
+    strict = bench.algorithmic_bytes(_W, g, lengths, tokens, native.SUCC_ON_STRICT)
+    assert strict["tree"] - base["tree"] == 4 * 9 + (1 + 2) * 16 * 2
+
+
+def test_reference_arm_prints_one_line(capsys):
+    """`bench.py --impl reference` times the oracle on host threads and prints
+    the contract's JSON line (small workload: config 1)."""
+    import json
+    import argparse
+    args = argparse.Namespace(config=1, seed=0, steps=2, warmup=1, gpus=1)
+    bench.run_reference(args)
+    out = [ln for ln in capsys.readouterr().out.splitlines() if ln.startswith("{")]
+    assert len(out) == 1
+    line = json.loads(out[0])
+    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"],
+                           "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}

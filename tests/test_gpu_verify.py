@@ -207,6 +207,48 @@ def test_hand_built_trees():
     assert gpu["new"][5, :3].tolist() == [20, 21, 33]
 
 
+def test_choice_across_row_splits():
+    """Rows long enough to be split over several CTAs (V = 40960): equal
+    maxima in different splits go to the first index; -0 and +0 tie; the
+    maximum at the last index; a row of equal values."""
+    V, N = 40960, 4
+    lg = np.full((1, N, V), -2.0, np.float32)
+    lg[0, 0, 30000] = 5.0
+    lg[0, 0, 100] = 5.0
+    lg[0, 1, :] = -1.0
+    lg[0, 2, 17000] = 0.0
+    lg[0, 2, 50] = -0.0
+    lg[0, 3, V - 1] = 7.0
+    draft = np.array([[0, 100, 0, 50]], np.int32)
+    par = np.array([[-1, 0, 1, 2]], np.int32)
+    nn = np.array([4], np.int32)
+    gpu, o, _ = run_both(synth.f32_to_bf16_bits(lg), draft, par, nn)
+    assert_same(gpu, o, None)
+    assert gpu["n_accept"][0] == 3
+    assert gpu["new"][0].tolist() == [100, 0, 50, V - 1]
+
+
+@pytest.mark.parametrize("N,depth", [(300, 200), (600, 450)])
+def test_deep_chains(N, depth):
+    """Chains of N nodes (N x S <= 1024 caps the row splits: at N = 600 one
+    CTA walks every 32 KB group of its row) accepted to a planted depth."""
+    V = 40960
+    rng = np.random.default_rng(N)
+    B = 2
+    draft = np.full((B, N), -1, np.int32)
+    par = np.full((B, N), -1, np.int32)
+    draft[:, 1:] = rng.integers(0, V, size=(B, N - 1))
+    par[:, 1:] = np.arange(N - 1)
+    nn = np.array([N, N - 7], np.int32)
+    lg = rng.integers(-4, 4, size=(B, N, V)).astype(np.float32)
+    for b in range(B):
+        for i in range(min(depth, int(nn[b]) - 1)):
+            lg[b, i, draft[b, i + 1]] = 9.0
+    gpu, o, _ = run_both(synth.f32_to_bf16_bits(lg), draft, par, nn)
+    assert_same(gpu, o, None)
+    assert gpu["n_accept"].tolist() == [depth, depth]
+
+
 def test_append_boundaries():
     """len + n_new == ld appends (exact fit); one more is FULL with nothing
     appended; a length outside [0, ld] is reported and nothing is appended."""
