@@ -152,45 +152,61 @@ __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
         }
     }
 
-    int32_t *part = ws.part1 + ((int64_t)b * ws.C1 + c) * kPart1Ints;
     __syncthreads();
-    if (t == 0) {
-        part[0] = cmax;
-        part[1] = cnt;
-    }
-    if (t < cnt) part[2 + t] = list[t];
-    __threadfence();
-    __syncthreads();
-    if (t == 0) flag = atomicAdd(ws.ticket1 + b, 1) == (int)gridDim.x - 1;
-    __syncthreads();
-    if (!flag) return;
-    __threadfence();
-
-    // ---- last chunk of sequence b: merge ------------------------------------
-    if (warp == 0) {
-        const int nchunks = (int)gridDim.x;
-        const int32_t *pb = ws.part1 + (int64_t)b * ws.C1 * kPart1Ints;
-        int best = 0;
-        for (int cc = lane; cc < nchunks; cc += 32) best = max(best, __ldcg(pb + cc * kPart1Ints));
-        best = warp_max_i(best);
-        int32_t *cb = a.cand + (int64_t)b * a.k;
-        int total = 0;
-        if (best > 0) {
-            total = warp_merge_desc(
-                nchunks, a.k,
-                [&](int cc) {
-                    const int32_t *pp = pb + cc * kPart1Ints;
-                    return __ldcg(pp) == best ? __ldcg(pp + 1) : 0;
-                },
-                [&](int cc, int i) { return __ldcg(pb + cc * kPart1Ints + 2 + i); }, cb);
+    if (gridDim.x == 1) {
+        // ---- the history is one chunk: its list is the result (no merge)
+        if (warp == 0) {
+            const int total = cmax > 0 ? cnt : 0;
+            if (lane < a.k) a.cand[(int64_t)b * a.k + lane] = lane < total ? list[lane] : -1;
+            if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
+            if (lane == 0) {
+                a.match_n[b] = cmax;
+                a.n_cand[b] = total;
+                a.hit_kind[b] = cmax > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
+                if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
+            }
         }
-        if (lane >= total && lane < a.k) cb[lane] = -1;
-        if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
-        if (lane == 0) {
-            a.match_n[b] = best;
-            a.n_cand[b] = total;
-            a.hit_kind[b] = best > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
-            if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
+    } else {
+        int32_t *part = ws.part1 + ((int64_t)b * ws.C1 + c) * kPart1Ints;
+        if (t == 0) {
+            part[0] = cmax;
+            part[1] = cnt;
+        }
+        if (t < cnt) part[2 + t] = list[t];
+        __threadfence();
+        __syncthreads();
+        if (t == 0) flag = atomicAdd(ws.ticket1 + b, 1) == (int)gridDim.x - 1;
+        __syncthreads();
+        if (!flag) return;
+        __threadfence();
+
+        // ---- last chunk of sequence b: merge --------------------------------
+        if (warp == 0) {
+            const int nchunks = (int)gridDim.x;
+            const int32_t *pb = ws.part1 + (int64_t)b * ws.C1 * kPart1Ints;
+            int best = 0;
+            for (int cc = lane; cc < nchunks; cc += 32)
+                best = max(best, __ldcg(pb + cc * kPart1Ints));
+            best = warp_max_i(best);
+            int32_t *cb = a.cand + (int64_t)b * a.k;
+            int total = 0;
+            if (best > 0) {
+                total = warp_merge_desc(
+                    nchunks, a.k,
+                    [&](int cc) {
+                        const int32_t *pp = pb + cc * kPart1Ints;
+                        return __ldcg(pp) == best ? __ldcg(pp + 1) : 0;
+                    },
+                    [&](int cc, int i) { return __ldcg(pb + cc * kPart1Ints + 2 + i); }, cb);
+            }
+            if (lane >= total && lane < a.k) cb[lane] = -1;
+            if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
+            if (lane == 0) {
+                a.match_n[b] = best;
+                a.n_cand[b] = total;
+                a.hit_kind[b] = best > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
+                if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
+            }
         }
     }
     if (!a.build_plan) return;

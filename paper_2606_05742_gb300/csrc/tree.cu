@@ -239,6 +239,21 @@ __device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int 
 }
 
 // ---------------------------------------------------------------------------
+// Publishes the successor-candidate count of branch w of sequence b.  A
+// branch token that never occurs earlier backs off (Sec. 3.5) to the
+// embedding fallback with the branch token as the anchor: with a table, the
+// (sequence, branch) pair is registered for the gathered pass.
+__device__ __forceinline__ void register_successors(const TreeLaunch &a, const Workspace &ws,
+                                                    int b, int w, int total, int token) {
+    ws.succ_n[(int64_t)b * ws.W + w] = total;
+    if (total == 0 && a.emb.table) {
+        const int idx = atomicAdd(ws.npairs, 1);
+        ws.pair_b[idx] = b;
+        ws.pair_tok[idx] = token;
+        ws.pair_out[idx] = b * ws.W + w;
+    }
+}
+
 __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     const TreeLaunch &a = args.p;
     const Workspace &ws = args.ws;
@@ -284,9 +299,13 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     for (int i = t; i < p1 - p0; i += kThreads4) s_tok[i] = M[p0 + i];
     __syncthreads();
     constexpr int U = 8;  // 32-position groups tested per pass (independent loads)
+    // one slice: its lists are the merged result, written in place (no merge)
+    const bool single = gridDim.x == 1;
     for (int w = warp; w < nb; w += nwarps) {
         const int bt = s_br[w];
-        int32_t *pp = ws.part4 + (((int64_t)b * ws.S4 + sl) * ws.W + w) * kPart4Ints;
+        int32_t *part =
+            single ? nullptr : ws.part4 + (((int64_t)b * ws.S4 + sl) * ws.W + w) * kPart4Ints;
+        int32_t *lst = single ? ws.succ + ((int64_t)b * ws.W + w) * kMaxK : part + 1;
         int cnt = 0;
         for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32 * U) {
             unsigned m[U];
@@ -299,36 +318,33 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
             for (int u = 0; u < U; ++u) {
                 const int p = top - 32 * u - lane;
                 const int rank = cnt + __popc(m[u] & ((1u << lane) - 1u));
-                if (((m[u] >> lane) & 1u) && rank < k) pp[1 + rank] = p;
+                if (((m[u] >> lane) & 1u) && rank < k) lst[rank] = p;
                 cnt += __popc(m[u]);
             }
         }
-        if (lane == 0) pp[0] = min(cnt, k);
-    }
-    __threadfence();
-    __syncthreads();
-    if (t == 0) s_misc[2] = atomicAdd(ws.ticket4 + b, 1) == (int)gridDim.x - 1;
-    __syncthreads();
-    if (!s_misc[2]) return;
-    __threadfence();
-    // last slice: merge, most recent first
-    for (int w = warp; w < nb; w += nwarps) {
-        const int32_t *pw = ws.part4 + ((int64_t)b * ws.S4 * ws.W + w) * kPart4Ints;
-        const int64_t stride = (int64_t)ws.W * kPart4Ints;  // next slice, same branch
-        const int total = warp_merge_desc(
-            (int)gridDim.x, k, [&](int s2) { return __ldcg(pw + s2 * stride); },
-            [&](int s2, int i) { return __ldcg(pw + s2 * stride + 1 + i); },
-            ws.succ + ((int64_t)b * ws.W + w) * kMaxK);
         if (lane == 0) {
-            ws.succ_n[(int64_t)b * ws.W + w] = total;
-            // Sec. 3.5: a branch token that never occurs backs off to the
-            // embedding fallback with the branch token as the anchor
-            if (total == 0 && a.emb.table) {
-                const int idx = atomicAdd(ws.npairs, 1);
-                ws.pair_b[idx] = b;
-                ws.pair_tok[idx] = s_br[w];
-                ws.pair_out[idx] = b * ws.W + w;
-            }
+            if (single)
+                register_successors(a, ws, b, w, min(cnt, k), s_br[w]);
+            else
+                part[0] = min(cnt, k);
+        }
+    }
+    if (!single) {
+        __threadfence();
+        __syncthreads();
+        if (t == 0) s_misc[2] = atomicAdd(ws.ticket4 + b, 1) == (int)gridDim.x - 1;
+        __syncthreads();
+        if (!s_misc[2]) return;
+        __threadfence();
+        // last slice: merge, most recent first
+        for (int w = warp; w < nb; w += nwarps) {
+            const int32_t *pw = ws.part4 + ((int64_t)b * ws.S4 * ws.W + w) * kPart4Ints;
+            const int64_t stride = (int64_t)ws.W * kPart4Ints;  // next slice, same branch
+            const int total = warp_merge_desc(
+                (int)gridDim.x, k, [&](int s2) { return __ldcg(pw + s2 * stride); },
+                [&](int s2, int i) { return __ldcg(pw + s2 * stride + 1 + i); },
+                ws.succ + ((int64_t)b * ws.W + w) * kMaxK);
+            if (lane == 0) register_successors(a, ws, b, w, total, s_br[w]);
         }
     }
     if ((v.lex || v.rr) && t < v.nc) {
