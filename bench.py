@@ -292,23 +292,42 @@ def step_launches(flags, W, emb):
     return n
 
 
-def algorithmic_bytes(w, g, lengths, tokens, flags=0):
-    """Bytes the step must move at minimum (no re-reads), per kernel."""
+def algorithmic_bytes(w, g, lengths, tokens, flags=0, emb_dim=None):
+    """Bytes the step must move at minimum (no re-reads), per kernel.  With a
+    token-embedding table of dimension emb_dim (two-representation mode) a
+    fallback needs one table row per distinct token of the history (the
+    score depends only on the token) plus one pass over the token ids, and a
+    successor backoff the same for its sequence."""
     d, k = w.d, w.k
     hk = g["hit_kind"]
     semantic = not flags & FLAG_NAMES["no_semantic"]
     active = (hk != 1) & semantic
     lex_bytes = int(4 * lengths.sum())
-    sem_rows = int(sum(lengths[b] - 1 for b in range(w.B) if active[b] and lengths[b] >= 2))
-    n_active = int(active.sum())
-    sem_bytes = (sem_rows * d * 2 + n_active * d * 2 + 4 * w.B) if semantic else 0
+
+    def distinct(b):
+        L = int(lengths[b])
+        return int(np.unique(tokens[b, : L - 1]).size) if L >= 2 else 0
+
+    if emb_dim is None:
+        sem_rows = int(sum(lengths[b] - 1 for b in range(w.B) if active[b] and lengths[b] >= 2))
+        n_active = int(active.sum())
+        sem_bytes = (sem_rows * d * 2 + n_active * d * 2 + 4 * w.B) if semantic else 0
+    else:
+        sem_bytes = 0
+        for b in range(w.B):
+            if active[b] and lengths[b] >= 2:
+                sem_bytes += (distinct(b) + 1) * emb_dim * 2 + 4 * int(lengths[b])
+        sem_bytes += 4 * w.B if semantic else 0
     # tree kernel: rerank rows + query for lexical hits, successor scan + rows
     succ_on = w.W > 0 and not flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"])
     gathered = 0
     succ_scan = 0
+    backoff = 0
     for b in range(w.B):
         L = int(lengths[b])
         if hk[b] == 1 and not flags & FLAG_NAMES["no_lex_rerank"]:
+            gathered += int(g["n_cand"][b]) + 1
+        if emb_dim is not None and hk[b] == 2:     # Eq. 6 rerank of the fallback's list
             gathered += int(g["n_cand"][b]) + 1
         if succ_on and (hk[b] == 2 or (hk[b] == 1 and flags & FLAG_NAMES["succ_on_strict"])):
             n = int(g["n_nodes"][b])
@@ -319,10 +338,15 @@ def algorithmic_bytes(w, g, lengths, tokens, flags=0):
             gathered += 1
             for h in heads:
                 t = int(g["draft_tokens"][b, h])
-                gathered += min(k, int((tokens[b, : L - 1] == t).sum()))
+                occ = int((tokens[b, : L - 1] == t).sum())
+                if occ == 0 and emb_dim is not None:   # backoff: the branch token's row
+                    backoff += (distinct(b) + 1) * emb_dim * 2 + 4 * L
+                    gathered += min(k, L - 1)
+                else:
+                    gathered += min(k, occ)
     N = g["draft_tokens"].shape[1]
     out_bytes = w.B * (N * 12 + N * N + k * 8 + 32)
-    tree_bytes = gathered * d * 2 + succ_scan + out_bytes
+    tree_bytes = gathered * d * 2 + succ_scan + backoff + out_bytes
     return {"lexical": lex_bytes, "semantic": sem_bytes, "tree": tree_bytes,
             "step": lex_bytes + sem_bytes + tree_bytes}
 
@@ -364,7 +388,8 @@ def run_native(args):
     g = eng.out.to_host()
     lengths = w.lengths.cpu().numpy()
     tokens = w.tokens.cpu().numpy()
-    nbytes = algorithmic_bytes(w, g, lengths, tokens, flags)
+    nbytes = algorithmic_bytes(w, g, lengths, tokens, flags,
+                               emb_dim=None if emb is None else int(emb.shape[1]))
 
     # Timed region A (the headline): K steps back to back, CUDA events only at
     # the two ends, so consecutive kernels keep their programmatic-launch
@@ -408,7 +433,9 @@ def run_native(args):
              for i, name in enumerate(("lexical", "semantic", "tree"))
              if name != "semantic" or semantic_on}
     # the dominant kernel: the semantic top-k, or without it the tree stage
-    dom_name, dom_kernel = (("semantic", "semantic_kernel") if semantic_on
+    dom_name, dom_kernel = (("semantic", "semantic_kernel" if emb is None else
+                             "rep_insert/count/scatter + semantic_kernel (gather) + expand")
+                            if semantic_on
                             else ("tree", "succ_scan_kernel + tree_kernel"))
     sem_ms = stage[dom_name]
     total_ms = max_over_ranks(total_ms, dev)

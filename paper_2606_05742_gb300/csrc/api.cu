@@ -153,12 +153,21 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, 1);
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
-    SemLaunch a{emb->table, ld, emb->dim, nullptr, lengths, active, B, k, tau, cand, score, n_cand,
-                nullptr, false};
-    a.tokens = tokens;
+    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
+    // the distinct tokens of the selected histories and the plan over them,
+    // the scores of the distinct tokens, then their positions
+    DedupeLaunch da{tokens, ld, lengths, B, emb->vocab, active, status, false, true, nullptr,
+                    true,   k,  cand,    score, n_cand};
+    ADAPLD_TRY(cuda_status(launch_dedupe(da, w, s)));
+    SemLaunch a{emb->table, ld, emb->dim, nullptr, w.rep_len, active, B, k, tau, cand, score, n_cand,
+                nullptr, true};
+    a.tokens = w.rep_tok;
     a.vocab = emb->vocab;
     a.status = status;
-    return cuda_status(launch_semantic(a, w, s));
+    ADAPLD_TRY(cuda_status(launch_semantic(a, w, s)));
+    ExpandLaunch ea{tokens, ld,     lengths, emb->vocab, B, nullptr, nullptr, nullptr, cand,
+                    score,  n_cand, k,       k,          nullptr, active, w.xticket};
+    return cuda_status(launch_expand(ea, w, s));
 }
 
 int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *lengths,
@@ -183,6 +192,7 @@ int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *le
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    if (emb) ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
     TreeLaunch a{tokens, ld, lengths, reps, d, query, B, hit_kind, cand, score, n_cand,
                  next_topk, next_topk ? Kn : 0, *p, *out, status};
     if (emb) a.emb = *emb;
@@ -212,10 +222,13 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     const bool semantic = !(p->flags & ADAPLD_NO_SEMANTIC);
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    if (emb) ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
 
     ADAPLD_TRY(record(ev ? ev->lexical_begin : nullptr, s));
+    // with a token-embedding table the plan is built over the distinct-token
+    // lists instead
     LexLaunch la{tokens, ld, lengths, B, p->n_max, p->k, out->hit_kind, out->match_n, out->cand,
-                 out->n_cand, out->score, out->status, to.stats, semantic};
+                 out->n_cand, out->score, out->status, to.stats, semantic && !emb};
     ADAPLD_TRY(cuda_status(launch_lexical(la, w, s)));
     ADAPLD_TRY(record(ev ? ev->lexical_end : nullptr, s));
 
@@ -223,15 +236,25 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
         ADAPLD_TRY(record(ev ? ev->semantic_begin : nullptr, s));
         SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
                      out->n_cand, out->hit_kind, true};
-        if (emb) {  // Eq. 4 over token embeddings
+        if (emb) {  // Eq. 4 over token embeddings, scored once per distinct token
+            DedupeLaunch da{tokens, ld, lengths, B, emb->vocab, nullptr, out->status, true, true,
+                            out->hit_kind, false, p->k, nullptr, nullptr, nullptr};
+            ADAPLD_TRY(cuda_status(launch_dedupe(da, w, s)));
             sa.reps = emb->table;
             sa.d = emb->dim;
             sa.query = nullptr;
-            sa.tokens = tokens;
+            sa.lengths = w.rep_len;
+            sa.tokens = w.rep_tok;
             sa.vocab = emb->vocab;
             sa.status = out->status;
         }
         ADAPLD_TRY(cuda_status(launch_semantic(sa, w, s)));
+        if (emb) {
+            ExpandLaunch ea{tokens, ld, lengths, emb->vocab, B, nullptr, nullptr, nullptr,
+                            out->cand, out->score, out->n_cand, p->k, p->k, out->hit_kind,
+                            nullptr, w.xticket};
+            ADAPLD_TRY(cuda_status(launch_expand(ea, w, s)));
+        }
         ADAPLD_TRY(record(ev ? ev->semantic_end : nullptr, s));
     }
 
@@ -239,6 +262,7 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
     TreeLaunch ta{tokens, ld, lengths, reps, d, query, B, out->hit_kind, out->cand, out->score,
                   out->n_cand, next_topk, next_topk ? Kn : 0, *p, to, out->status};
     if (emb) ta.emb = *emb;
+    ta.lists_ready = emb && semantic;  // the distinct-token lists exist for every sequence
     ADAPLD_TRY(cuda_status(launch_tree(ta, w, s)));
     return record(ev ? ev->tree_end : nullptr, s);
 }

@@ -35,9 +35,12 @@ struct Workspace {
     int32_t *ticket4;        // [B]  successor scan: slices done per sequence
     int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
     int32_t *npairs;         // [1]  successor backoff: (sequence, branch) pairs
-    int32_t *gticket4;       // [1]  successor scan: sequences done
+    int32_t *gticket_rep;    // [1]  distinct-token lists: sequences done (plan)
     int32_t *vticket;        // [B]  verification: CTAs done per sequence
     int32_t *done3;          // [B*W] successor backoff: CTAs done per pair
+    int32_t *rticket;        // [B]  distinct-token lists: chunks counted per sequence
+    int32_t *xticket;        // [B]  expansion of the fallback lists: slices done
+    int32_t *xticket2;       // [B*W] expansion of the backoff lists: slices done
     int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
     int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
     int32_t *slots2;         // [B + kMaxGrid2][kSlotInts] partial top-k lists
@@ -55,6 +58,16 @@ struct Workspace {
     float *succ_es;          // [B*W][kMaxK] backoff candidates' embedding scores
     unsigned long long *vpart;  // [B][N][S], N*S <= kMaxNodes: verification, packed
                                 //   (logit, index) maximum per node and row split
+    // distinct-token lists (two-representation mode): a row of the token-
+    // embedding fallback depends only on the token, so each token of a
+    // history is scored once
+    unsigned long long *htab;   // [B][H] hash of (token + 1) << 32 | latest position
+    int32_t *rep_tok;        // [B][ld] distinct tokens by latest position, then the anchor
+    int32_t *rep_len;        // [B] distinct tokens + 1 (a length: rows = rep_len - 1)
+    int32_t *rep_cnt;        // [B][C1] distinct tokens per chunk, then chunk offsets
+    int32_t *xpart;          // [B*W][S4][kMaxK][kPart4Ints] expansion: per-slice lists
+    int64_t H;               // hash slots per sequence (a power of two >= 2 (ld-1))
+    size_t htab_bytes;
     size_t counters_bytes;
     size_t total_bytes;
     int C1, S4, W;
@@ -64,6 +77,14 @@ __host__ __device__ inline size_t align_up(size_t x, size_t a) { return (x + a -
 
 __host__ __device__ inline int chunks_of(int64_t n, int64_t per) {
     return (int)((n < 1 ? 1 : n + per - 1) / per);
+}
+
+// Hash slots per sequence for the distinct-token lists: a power of two of at
+// least twice the candidate positions, so the load factor stays <= 1/2.
+__host__ __device__ inline int64_t hash_slots(int64_t ld) {
+    int64_t h = 64;
+    while (h < 2 * (ld - 1)) h <<= 1;
+    return h;
 }
 
 // Lays the workspace out at `base` (NULL: sizing only).
@@ -80,18 +101,21 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         return r;
     };
     const size_t BW = (size_t)B * w.W;
-    w.counters_bytes = sizeof(int32_t) * (4 + 5 * (size_t)B + BW);
+    w.counters_bytes = sizeof(int32_t) * (4 + 7 * (size_t)B + 2 * BW);
     w.dev_status = (int32_t *)take(w.counters_bytes);
     if (p) {
         w.global_ticket = w.dev_status + 1;
         w.npairs = w.dev_status + 2;
-        w.gticket4 = w.dev_status + 3;
+        w.gticket_rep = w.dev_status + 3;
         w.ticket1 = w.dev_status + 4;
         w.done2 = w.ticket1 + B;
         w.ticket4 = w.done2 + B;
         w.ticket5 = w.ticket4 + B;
         w.vticket = w.ticket5 + B;
         w.done3 = w.vticket + B;
+        w.rticket = w.done3 + BW;
+        w.xticket = w.rticket + B;
+        w.xticket2 = w.xticket + B;
     }
     w.part1 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1 * kPart1Ints);
     w.plan = (int64_t *)take(sizeof(int64_t) * ((size_t)B + 1));
@@ -109,6 +133,13 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.pair_out = (int32_t *)take(sizeof(int32_t) * BW);
     w.succ_es = (float *)take(sizeof(float) * BW * kMaxK);
     w.vpart = (unsigned long long *)take(sizeof(unsigned long long) * (size_t)B * kMaxNodes);
+    w.H = hash_slots(ld);
+    w.htab_bytes = sizeof(unsigned long long) * (size_t)B * w.H;
+    w.htab = (unsigned long long *)take(w.htab_bytes);
+    w.rep_tok = (int32_t *)take(sizeof(int32_t) * (size_t)B * ld);
+    w.rep_len = (int32_t *)take(sizeof(int32_t) * (size_t)B);
+    w.rep_cnt = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1);
+    w.xpart = (int32_t *)take(sizeof(int32_t) * BW * w.S4 * kMaxK * kPart4Ints);
     w.total_bytes = off;
     return w;
 }
@@ -312,6 +343,66 @@ __device__ __forceinline__ int warp_merge_desc(int nparts, int k, CountF count_o
     return total;
 }
 
+// Block-wide exclusive scan of one int64 per thread (blockDim.x <= 1024).
+__device__ inline int64_t block_exclusive_scan(int64_t v, int64_t *total, int64_t *scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int64_t incl = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int64_t u = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += u;
+    }
+    if (lane == 31) scratch[warp] = incl;
+    __syncthreads();
+    int64_t before = 0, all = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+        if (w < warp) before += scratch[w];
+        all += scratch[w];
+    }
+    __syncthreads();
+    *total = all;
+    return before + incl - v;
+}
+
+// One CTA builds the semantic plan plan[0..B]: prefix sums of the rows
+// (len - 1) of the selected sequences with a valid length (selection:
+// hit_kind != LEX when hit_kind is given, else active[b] != 0, NULL = all);
+// with init_out, selected sequences get default outputs (no candidates).
+// Lengths are read through L2 (they may come from the same kernel's CTAs).
+__device__ inline void build_plan_cta(const int32_t *lengths, int64_t ld, int32_t B,
+                                      const int32_t *hit_kind, const uint8_t *active,
+                                      int64_t *plan, bool init_out, int32_t k, int32_t *cand,
+                                      float *score, int32_t *n_cand) {
+    __shared__ int64_t scratch[32];
+    int64_t carry = 0;
+    for (int base = 0; base < B; base += blockDim.x) {
+        const int b = base + threadIdx.x;
+        int64_t rows = 0;
+        if (b < B) {
+            const int len = __ldcg(lengths + b);
+            const bool valid = len >= 1 && (int64_t)len <= ld;
+            bool sel;
+            if (hit_kind)
+                sel = __ldcg(hit_kind + b) != ADAPLD_HIT_LEX;
+            else
+                sel = active ? active[b] != 0 : true;
+            if (sel && valid) rows = len - 1;
+            if (sel && init_out) {
+                n_cand[b] = 0;
+                for (int i = 0; i < k; ++i) {
+                    cand[(int64_t)b * k + i] = -1;
+                    score[(int64_t)b * k + i] = 0.f;
+                }
+            }
+        }
+        int64_t total;
+        const int64_t ex = block_exclusive_scan(rows, &total, scratch);
+        if (b < B) plan[b] = carry + ex;
+        carry += total;
+    }
+    if (threadIdx.x == 0) plan[B] = carry;
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
     for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -416,8 +507,64 @@ struct TreeLaunch {
     adapld_tree_out out;
     int32_t *status;
     adapld_embeddings emb = {nullptr, 0, 0};  // token embeddings (two-representation mode)
+    bool lists_ready = false;  // the distinct-token lists were built by this call already
 };
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s);
+
+// Distinct-token lists of the histories (two-representation mode; csrc/
+// dedupe.cu).  For every selected sequence with a valid length:
+// rep_tok[b][0..n) = the distinct tokens of positions [0, len-2] (ids outside
+// [0, vocab) count as token 0, whose table row they read), ordered by their
+// latest position; rep_tok[b][n] = the anchor token M[len-1] (as stored);
+// rep_len[b] = n + 1, or 0 for an invalid length or an unselected sequence.
+// Scoring rep rows r < n against a query scores every position of the token
+// at once, and rank order r follows the latest position, so a top-k over the
+// lists ranks tokens exactly as the per-position top-k would rank their
+// latest occurrences.  Needs ws.htab zeroed beforehand.
+struct DedupeLaunch {
+    const int32_t *tokens;
+    int64_t ld;
+    const int32_t *lengths;
+    int32_t B, vocab;
+    const uint8_t *active;   // selection (NULL = every sequence)
+    int32_t *status;         // ADAPLD_SEQ_BAD_TOKEN bits (nullable)
+    bool pdl;                // launched as a programmatic dependent of a kernel
+    // semantic plan over the lists (built by the last sequence), selection as
+    // in build_plan_cta
+    bool build_plan;
+    const int32_t *hit_kind;
+    bool init_out;
+    int32_t k;
+    int32_t *cand;
+    float *score;
+    int32_t *n_cand;
+};
+cudaError_t launch_dedupe(const DedupeLaunch &a, const Workspace &ws, cudaStream_t s);
+
+// Expansion of top-k lists over distinct tokens (rep indices, as written by
+// the semantic kernel over the lists) into the top-k positions under (score
+// desc, position desc): every position of a listed token has that token's
+// score.  Virtual sequence p (real sequence vseq_b[p], output row
+// vseq_out[p]; identity when NULL, count *nvseq when given) rewrites its row
+// of cand / score / n_cand (row stride `stride`) in place.  Real sequences
+// are expanded when hit_kind[b] == SEM (hit_kind given) or active[b] != 0.
+struct ExpandLaunch {
+    const int32_t *tokens;
+    int64_t ld;
+    const int32_t *lengths;
+    int32_t vocab;
+    int32_t P;               // virtual sequences the grid covers
+    const int32_t *nvseq;    // device count (nullable: P)
+    const int32_t *vseq_b, *vseq_out;
+    int32_t *cand;
+    float *score;
+    int32_t *n_cand;
+    int32_t stride, k;
+    const int32_t *hit_kind;
+    const uint8_t *active;
+    int32_t *ticket;         // [P] slices done
+};
+cudaError_t launch_expand(const ExpandLaunch &a, const Workspace &ws, cudaStream_t s);
 
 struct VerifyLaunch {
     const uint16_t *logits;  // [B][N][V] bf16

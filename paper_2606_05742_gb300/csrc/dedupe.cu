@@ -1,0 +1,366 @@
+// Distinct-token lists for the token-embedding fallback (Eq. 4 as printed:
+// cos(e_{M_j}, e_a)) and their expansion back to positions.
+//
+// Under Eq. 4 the score of position j depends only on the token M[j], so a
+// history of len positions needs only as many table rows as it has distinct
+// tokens (about a sixth to a quarter of the positions on Zipf-like text).
+// Exactness is kept by ranking tokens by their latest position: the top-k
+// positions under (score desc, position desc) all belong to tokens among the
+// top-k of that token list, and expansion recovers their positions.
+//
+//  rep_insert_kernel  grid (C1 chunks of 4096 positions, B), 256 threads:
+//      inserts (token, position) into the sequence's open-addressing hash
+//      (key token + 1 in the high word, the latest position in the low word:
+//      atomicCAS to claim a slot, atomicMax to keep the latest position);
+//      lanes holding the same token in a warp insert once (__match_any_sync).
+//  rep_count_kernel   same grid: counts the positions that are the latest
+//      occurrence of their token per chunk; the last chunk of a sequence
+//      turns the counts into offsets and writes rep_len and the anchor; the
+//      last sequence builds the semantic plan over the lists.
+//  rep_scatter_kernel same grid: writes each chunk's latest occurrences'
+//      tokens in position order at the chunk's offset.
+//  expand_kernel      grid (S4 slices of 8192 positions, P), 512 threads: per
+//      listed token (a warp each) the k most recent positions in the slice;
+//      the last slice merges per token, then over tokens by (score desc,
+//      position desc) and rewrites the list as positions.
+//
+// Every probe loop is bounded by the table size (the load factor is at most
+// 1/2, so it never comes close); running past it would raise
+// ADAPLD_DEV_INTERNAL.
+#include "common.cuh"
+
+namespace adapld {
+
+namespace {
+
+struct DedupeArgs {
+    DedupeLaunch p;
+    Workspace ws;
+};
+
+struct ExpandArgs {
+    ExpandLaunch p;
+    Workspace ws;
+};
+
+// The table row a token id reads: ids outside [0, vocab) read row 0.
+__device__ __forceinline__ int canon(int tok, int vocab) {
+    return tok >= 0 && tok < vocab ? tok : 0;
+}
+
+// lowbias32, an integer hash published by C. Wellons (hash-prospector).
+__device__ __forceinline__ uint32_t hash32(uint32_t x) {
+    x ^= x >> 16;
+    x *= 0x7feb352du;
+    x ^= x >> 15;
+    x *= 0x846ca68bu;
+    x ^= x >> 16;
+    return x;
+}
+
+__device__ __forceinline__ bool seq_selected(const DedupeLaunch &a, int b, int &len) {
+    len = a.lengths[b];
+    if (len < 1 || (int64_t)len > a.ld) return false;
+    return a.active ? a.active[b] != 0 : true;
+}
+
+// Latest position stored for token u (-1 if absent or past the probe bound).
+__device__ __forceinline__ int hash_lookup(const unsigned long long *T, int64_t H, int u) {
+    const unsigned long long key = (unsigned long long)(uint32_t)(u + 1);
+    uint64_t h = hash32((uint32_t)u) & (uint64_t)(H - 1);
+    for (int64_t probe = 0; probe < H; ++probe) {
+        const unsigned long long cur = __ldcg(T + h);
+        if (cur == 0ull) return -1;
+        if ((cur >> 32) == key) return (int)(uint32_t)(cur & 0xffffffffull);
+        h = (h + 1) & (uint64_t)(H - 1);
+    }
+    return -1;
+}
+
+__global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) {
+    const DedupeLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int s_bad;
+    pdl_wait_then_release();
+    const int t = threadIdx.x, lane = t & 31;
+    const int b = blockIdx.y, c = blockIdx.x;
+    int len;
+    if (!seq_selected(a, b, len)) return;
+    const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);  // positions <= len-2
+    if (j0 >= j1) return;
+    if (t == 0) s_bad = 0;
+    __syncthreads();
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    unsigned long long *T = ws.htab + (int64_t)b * ws.H;
+    const int64_t H = ws.H;
+    bool bad = false, lost = false;
+    for (int base = j0; base < j1; base += kThreads1) {
+        const int j = base + t;
+        const bool in = j < j1;
+        const int raw = in ? M[j] : 0;
+        const int u = canon(raw, a.vocab);
+        bad |= in && raw != u;
+        const unsigned act = __ballot_sync(0xffffffffu, in);
+        if (!in) continue;
+        // lanes hold consecutive positions: the highest lane of a group of
+        // equal tokens has the latest one and inserts for the group
+        const unsigned same = __match_any_sync(act, u);
+        if (lane != 31 - __clz(same)) continue;
+        const unsigned long long mine =
+            ((unsigned long long)(uint32_t)(u + 1) << 32) | (unsigned long long)(uint32_t)j;
+        uint64_t h = hash32((uint32_t)u) & (uint64_t)(H - 1);
+        int64_t probe = 0;
+        for (; probe < H; ++probe) {
+            const unsigned long long old = atomicCAS(T + h, 0ull, mine);
+            if (old == 0ull) break;
+            if ((old >> 32) == (mine >> 32)) {
+                if ((uint32_t)old < (uint32_t)j) atomicMax(T + h, mine);
+                break;
+            }
+            h = (h + 1) & (uint64_t)(H - 1);
+        }
+        lost |= probe == H;
+    }
+    if (bad) s_bad = 1;
+    if (lost) atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
+    __syncthreads();
+    if (t == 0 && s_bad && a.status) atomicOr(a.status + b, ADAPLD_SEQ_BAD_TOKEN);
+}
+
+// Whether position j (token u) is the latest occurrence of its token.
+__device__ __forceinline__ bool is_latest(const unsigned long long *T, int64_t H, int u, int j) {
+    return hash_lookup(T, H, u) == j;
+}
+
+__global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
+    const DedupeLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int s_flag;
+    __shared__ int64_t s_scan[32];
+    pdl_wait_then_release();
+    const int t = threadIdx.x;
+    const int b = blockIdx.y, c = blockIdx.x;
+    int len;
+    const bool sel = seq_selected(a, b, len);
+    bool seq_done = false;  // this CTA finishes sequence b (then takes the global ticket)
+    if (!sel) {
+        if (c != 0) return;
+        if (t == 0) ws.rep_len[b] = 0;
+        seq_done = true;
+    } else {
+        const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);
+        const int32_t *M = a.tokens + (int64_t)b * a.ld;
+        const unsigned long long *T = ws.htab + (int64_t)b * ws.H;
+        int mine = 0;
+        for (int j = j0 + t; j < j1; j += kThreads1)
+            mine += is_latest(T, ws.H, canon(M[j], a.vocab), j);
+        int64_t total;  // the block's sum
+        (void)block_exclusive_scan(mine, &total, s_scan);
+        if (t == 0) ws.rep_cnt[(int64_t)b * ws.C1 + c] = (int)total;
+        __threadfence();
+        __syncthreads();
+        if (t == 0) s_flag = atomicAdd(ws.rticket + b, 1) == (int)gridDim.x - 1;
+        __syncthreads();
+        if (!s_flag) return;
+        __threadfence();
+        // last chunk of b: chunk counts -> offsets, n = distinct tokens
+        int64_t carry = 0;
+        for (int base = 0; base < (int)gridDim.x; base += kThreads1) {
+            const int cc = base + t;
+            const int64_t v =
+                cc < (int)gridDim.x ? __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + cc) : 0;
+            int64_t all;
+            const int64_t ex = block_exclusive_scan(v, &all, s_scan);
+            if (cc < (int)gridDim.x) ws.rep_cnt[(int64_t)b * ws.C1 + cc] = (int)(carry + ex);
+            carry += all;
+        }
+        if (t == 0) {
+            ws.rep_len[b] = (int)carry + 1;
+            ws.rep_tok[(int64_t)b * a.ld + carry] = M[len - 1];  // the anchor (as stored)
+        }
+        seq_done = true;
+    }
+    if (!seq_done || !a.build_plan) return;
+    // ---- the last sequence overall: the semantic plan over the lists
+    __threadfence();
+    __syncthreads();
+    if (t == 0) s_flag = atomicAdd(ws.gticket_rep, 1) == a.B - 1;
+    __syncthreads();
+    if (!s_flag) return;
+    __threadfence();
+    build_plan_cta(ws.rep_len, a.ld, a.B, a.hit_kind, a.hit_kind ? nullptr : a.active, ws.plan,
+                   a.init_out, a.k, a.cand, a.score, a.n_cand);
+}
+
+__global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args) {
+    const DedupeLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int64_t s_scan[32];
+    pdl_wait_then_release();
+    const int t = threadIdx.x;
+    const int b = blockIdx.y, c = blockIdx.x;
+    int len;
+    if (!seq_selected(a, b, len)) return;
+    const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);
+    if (j0 >= j1) return;
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const unsigned long long *T = ws.htab + (int64_t)b * ws.H;
+    int32_t *out = ws.rep_tok + (int64_t)b * a.ld + __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c);
+    int64_t carry = 0;
+    for (int base = j0; base < j1; base += kThreads1) {
+        const int j = base + t;
+        int u = 0;
+        bool keep = false;
+        if (j < j1) {
+            u = canon(M[j], a.vocab);
+            keep = is_latest(T, ws.H, u, j);
+        }
+        int64_t all;
+        const int64_t ex = block_exclusive_scan(keep ? 1 : 0, &all, s_scan);
+        if (keep) out[carry + ex] = u;
+        carry += all;
+    }
+}
+
+// ---------------------------------------------------------------- expansion
+constexpr int kExpandThreads = kThreads4;  // 16 warps
+constexpr int kExpandWarps = kExpandThreads / 32;
+
+struct ExpandShared {
+    int tok[kSlice4];         // canonical tokens of the slice
+    int key[kMaxK];           // listed tokens
+    float sc[kMaxK];          // their scores
+    int lst[kMaxK][kMaxK];    // per token: the k most recent positions
+    int cnt[kMaxK];
+    int flag;
+};
+
+// Slice sl of virtual sequence p (the whole CTA; every branch is uniform).
+__device__ void expand_one(const ExpandLaunch &a, const Workspace &ws, ExpandShared &sh, int p,
+                           int sl) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int b = a.vseq_b ? a.vseq_b[p] : p;
+    const int64_t row = a.vseq_out ? a.vseq_out[p] : p;
+    if (!a.vseq_b) {
+        if (a.hit_kind && a.hit_kind[b] != ADAPLD_HIT_SEM) return;
+        if (!a.hit_kind && a.active && !a.active[b]) return;
+    }
+    const int len = a.lengths[b];
+    if (len < 2 || (int64_t)len > a.ld) return;
+    const int n = min(a.n_cand[row], a.k);
+    if (n <= 0) return;
+    const int k = a.k;
+    int32_t *crow = a.cand + row * a.stride;
+    float *srow = a.score + row * a.stride;
+    if (t < n) {
+        const int r = crow[t];
+        const int rl = ws.rep_len[b];
+        sh.key[t] = r >= 0 && r < rl - 1 ? ws.rep_tok[(int64_t)b * a.ld + r] : -1;
+        sh.sc[t] = srow[t];
+    }
+    const int p0 = sl * kSlice4, p1 = min(p0 + kSlice4, len - 1);
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    for (int i = t; i < p1 - p0; i += kExpandThreads) sh.tok[i] = canon(M[p0 + i], a.vocab);
+    __syncthreads();
+
+    // the k most recent positions of each listed token in this slice
+    const bool single = gridDim.x == 1;
+    constexpr int U = 8;
+    for (int i = warp; i < n; i += kExpandWarps) {
+        const int key = sh.key[i];
+        int32_t *part = single ? nullptr
+                               : ws.xpart + (((int64_t)p * ws.S4 + sl) * kMaxK + i) * kPart4Ints;
+        int cnt = 0;
+        for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32 * U) {
+            unsigned m[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = top - 32 * u - lane;
+                m[u] = __ballot_sync(0xffffffffu, q >= p0 && sh.tok[q - p0] == key);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = top - 32 * u - lane;
+                const int rank = cnt + __popc(m[u] & ((1u << lane) - 1u));
+                if (((m[u] >> lane) & 1u) && rank < k) {
+                    if (single)
+                        sh.lst[i][rank] = q;
+                    else
+                        part[1 + rank] = q;
+                }
+                cnt += __popc(m[u]);
+            }
+        }
+        if (lane == 0) {
+            if (single)
+                sh.cnt[i] = min(cnt, k);
+            else
+                part[0] = min(cnt, k);
+        }
+    }
+    if (!single) {
+        __threadfence();
+        __syncthreads();
+        if (t == 0) sh.flag = atomicAdd(a.ticket + p, 1) == (int)gridDim.x - 1;
+        __syncthreads();
+        if (!sh.flag) return;
+        __threadfence();
+        // per token: merge the slices, most recent first
+        for (int i = warp; i < n; i += kExpandWarps) {
+            const int32_t *pw = ws.xpart + ((int64_t)p * ws.S4 * kMaxK + i) * kPart4Ints;
+            const int64_t stride = (int64_t)kMaxK * kPart4Ints;  // next slice, same token
+            const int total = warp_merge_desc(
+                (int)gridDim.x, k, [&](int s2) { return __ldcg(pw + s2 * stride); },
+                [&](int s2, int e) { return __ldcg(pw + s2 * stride + 1 + e); }, sh.lst[i]);
+            if (lane == 0) sh.cnt[i] = total;
+        }
+    }
+    __syncthreads();
+    // over tokens: (score desc, position desc), the first k
+    if (warp == 0) {
+        WarpTopK tk;
+        tk.reset();
+        for (int i = 0; i < n; ++i) {
+            const int c = sh.cnt[i];
+            tk.insert(lane < c, sh.sc[i], lane < c ? sh.lst[i][lane] : -1, k);
+        }
+        if (lane < k) {
+            crow[lane] = lane < tk.n ? tk.j : -1;
+            srow[lane] = lane < tk.n ? tk.s : 0.f;
+        }
+        if (lane == 0) a.n_cand[row] = tk.n;
+    }
+}
+
+__global__ void __launch_bounds__(kExpandThreads) expand_kernel(ExpandArgs args) {
+    __shared__ ExpandShared sh;
+    pdl_wait_then_release();
+    const ExpandLaunch &a = args.p;
+    const int P = a.nvseq ? min(*a.nvseq, a.P) : a.P;
+    // virtual sequences blockIdx.y, + gridDim.y, ... (the y extent is capped)
+    for (int p = blockIdx.y; p < P; p += gridDim.y) {
+        expand_one(a, args.ws, sh, p, blockIdx.x);
+        __syncthreads();  // before the next p reuses the shared state
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_dedupe(const DedupeLaunch &a, const Workspace &ws, cudaStream_t s) {
+    DedupeArgs args{a, ws};
+    const dim3 grid(ws.C1, a.B);
+    cudaError_t e = a.pdl ? launch_dependent(rep_insert_kernel, grid, dim3(kThreads1), 0, s, args)
+                          : (rep_insert_kernel<<<grid, kThreads1, 0, s>>>(args), cudaGetLastError());
+    if (e != cudaSuccess) return e;
+    e = launch_dependent(rep_count_kernel, grid, dim3(kThreads1), 0, s, args);
+    if (e != cudaSuccess) return e;
+    return launch_dependent(rep_scatter_kernel, grid, dim3(kThreads1), 0, s, args);
+}
+
+cudaError_t launch_expand(const ExpandLaunch &a, const Workspace &ws, cudaStream_t s) {
+    ExpandArgs args{a, ws};
+    const int gy = a.P < 65535 ? (a.P < 1 ? 1 : a.P) : 65535;
+    return launch_dependent(expand_kernel, dim3(ws.S4, gy), dim3(kExpandThreads), 0, s, args);
+}
+
+}  // namespace adapld

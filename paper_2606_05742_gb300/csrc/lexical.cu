@@ -22,62 +22,6 @@ struct LexArgs {
     Workspace ws;
 };
 
-// Block-wide exclusive scan of one int64 per thread (256 threads).
-__device__ int64_t block_exclusive_scan(int64_t v, int64_t *total, int64_t *scratch) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    int64_t incl = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        int64_t u = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += u;
-    }
-    if (lane == 31) scratch[warp] = incl;
-    __syncthreads();
-    int64_t before = 0, all = 0;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-        if (w < warp) before += scratch[w];
-        all += scratch[w];
-    }
-    __syncthreads();
-    *total = all;
-    return before + incl - v;
-}
-
-// One CTA builds plan[0..B] (see launch_plan in common.cuh).
-__device__ void build_plan_cta(const int32_t *lengths, int64_t ld, int32_t B,
-                               const int32_t *hit_kind, const uint8_t *active, int64_t *plan,
-                               bool init_out, int32_t k, int32_t *cand, float *score,
-                               int32_t *n_cand) {
-    __shared__ int64_t scratch[32];
-    int64_t carry = 0;
-    for (int base = 0; base < B; base += blockDim.x) {
-        const int b = base + threadIdx.x;
-        int64_t rows = 0;
-        if (b < B) {
-            const int len = lengths[b];
-            const bool valid = len >= 1 && (int64_t)len <= ld;
-            bool sel;
-            if (hit_kind)
-                sel = __ldcg(hit_kind + b) != ADAPLD_HIT_LEX;
-            else
-                sel = active ? active[b] != 0 : true;
-            if (sel && valid) rows = len - 1;
-            if (sel && init_out) {
-                n_cand[b] = 0;
-                for (int i = 0; i < k; ++i) {
-                    cand[(int64_t)b * k + i] = -1;
-                    score[(int64_t)b * k + i] = 0.f;
-                }
-            }
-        }
-        int64_t total;
-        const int64_t ex = block_exclusive_scan(rows, &total, scratch);
-        if (b < B) plan[b] = carry + ex;
-        carry += total;
-    }
-    if (threadIdx.x == 0) plan[B] = carry;
-}
-
 __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
     const LexLaunch &a = args.p;
     const Workspace &ws = args.ws;

@@ -366,8 +366,8 @@ __global__ void __launch_bounds__(256) backoff_plan_kernel(TreeArgs args) {
     for (int base = 0; base < n; base += 256) {
         const int p = base + threadIdx.x;
         int64_t rows = 0;
-        if (p < n) {
-            const int len = a.lengths[ws.pair_b[p]];
+        if (p < n) {  // the pair scores its sequence's distinct tokens
+            const int len = __ldcg(ws.rep_len + ws.pair_b[p]);
             rows = len >= 2 ? len - 1 : 0;
         }
         int64_t incl = rows;
@@ -605,15 +605,21 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
     const int tasks = succ_possible ? (W * k > k ? W * k : k) : k;
     TreeArgs args{a, ws, (tasks + kRowsPerCta5 - 1) / kRowsPerCta5};
     if (succ_possible) {
-        cudaError_t e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), 0, s,
-                                         args);
+        cudaError_t e;
+        if (a.emb.table && !a.lists_ready) {  // distinct-token lists for the backoff
+            DedupeLaunch da{a.tokens, a.ld, a.lengths, a.B, a.emb.vocab, nullptr, a.status, true,
+                            false, nullptr, false, k, nullptr, nullptr, nullptr};
+            e = launch_dedupe(da, ws, s);
+            if (e != cudaSuccess) return e;
+        }
+        e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), 0, s, args);
         if (e != cudaSuccess) return e;
         if (a.emb.table) {  // successor backoff over token embeddings
             e = launch_dependent(backoff_plan_kernel, dim3(1), dim3(256), 0, s, args);
             if (e != cudaSuccess) return e;
-            SemLaunch sl{a.emb.table, a.ld, a.emb.dim, nullptr, a.lengths, nullptr, a.B, k,
+            SemLaunch sl{a.emb.table, a.ld, a.emb.dim, nullptr, ws.rep_len, nullptr, a.B, k,
                          a.p.tau, ws.succ, ws.succ_es, ws.succ_n, nullptr, true};
-            sl.tokens = a.tokens;
+            sl.tokens = ws.rep_tok;
             sl.vocab = a.emb.vocab;
             sl.vseq_b = ws.pair_b;
             sl.vseq_tok = ws.pair_tok;
@@ -622,6 +628,12 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
             sl.out_stride = kMaxK;
             sl.status = a.status;
             e = launch_semantic(sl, ws, s);
+            if (e != cudaSuccess) return e;
+            // the best distinct tokens back to their k most recent positions
+            ExpandLaunch ea{a.tokens, a.ld,     a.lengths, a.emb.vocab, a.B * ws.W, ws.npairs,
+                            ws.pair_b, ws.pair_out, ws.succ,  ws.succ_es,  ws.succ_n, kMaxK,
+                            k,         nullptr,     nullptr,  ws.xticket2};
+            e = launch_expand(ea, ws, s);
             if (e != cudaSuccess) return e;
         }
     }

@@ -71,3 +71,24 @@ def test_reference_arm_prints_one_line(capsys):
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"] == {"value": line["value"], "unit": line["unit"],
                            "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
+def test_algorithmic_bytes_embedding_mode():
+    """With a token-embedding table the fallback counts one row per distinct
+    token (plus the anchor's) and one pass over the ids."""
+    L = 10
+    tokens = np.tile(np.arange(L, dtype=np.int32) % 5, (3, 1))   # 5 distinct in 0..8
+    lengths = np.full(3, L, np.int32)
+    g = {"hit_kind": np.array([1, 2, 0]), "n_cand": np.array([3, 2, 0]),
+         "n_nodes": np.array([4, 3, 1]),
+         "parents": np.array([[-1, 0, 1, 0], [-1, 0, 0, -1], [-1, -1, -1, -1]]),
+         "draft_tokens": np.array([[4, 0, 1, 2], [4, 1, 7, -1], [4, -1, -1, -1]])}
+    de = 8
+    x = bench.algorithmic_bytes(_W, g, lengths, tokens, emb_dim=de)
+    assert x["semantic"] == 2 * ((5 + 1) * de * 2 + 4 * L) + 4 * 3
+    base = bench.algorithmic_bytes(_W, g, lengths, tokens)
+    # the semantic hit adds its Eq. 6 rerank rows (2 + query); its branch
+    # token 7 never occurs: the backoff gathers the 5 distinct rows + anchor
+    # and scores min(k, L-1) positions instead of none
+    extra = (2 + 1) * 16 * 2 + (5 + 1) * de * 2 + 4 * L + 4 * 16 * 2
+    assert x["tree"] - base["tree"] == extra

@@ -417,6 +417,7 @@ EMB_CASES = [  # (cfg, B, L, d, de, V, seed)
     (2, 8, 1500, 128, 64, 4096, 0), (5, 4, 3000, 256, 4096, 8192, 1),
     (3, 6, 2000, 640, 136, 3000, 2), (4, 20, 500, 64, 8, 2048, 3),
     (5, 3, 1200, 64, 8192, 2048, 4),
+    (5, 3, 20000, 64, 256, 4096, 5),    # several chunks and slices per history
 ]
 
 
@@ -479,6 +480,83 @@ def test_embedding_topk_standalone():
             parity.check_semantic_list(cand[b].cpu().numpy(), score[b].cpu().numpy(), int(n[b]),
                                        s_all, eps, w.k, tau, rep, f"seq {b}")
         assert int(status.sum()) == 0
+
+
+def _emb_topk(w, E, tau, active=None):
+    tok, ln, _, _ = to_dev(w)
+    Ed = torch.from_numpy(E.view(np.int16)).cuda().view(torch.bfloat16)
+    ws = native.allocate_workspace(w.B, w.ld, w.d, params(P_of(w)))
+    cand = torch.full((w.B, w.k), -7, dtype=torch.int32, device="cuda")
+    score = torch.zeros((w.B, w.k), dtype=torch.float32, device="cuda")
+    n = torch.full((w.B,), -7, dtype=torch.int32, device="cuda")
+    native.embedding_topk(tok, ln, Ed, w.k, tau, cand, score, n, ws, active=active)
+    torch.cuda.synchronize()
+    assert native.read_device_status(ws) == 0
+    return cand.cpu().numpy(), score.cpu().numpy(), n.cpu().numpy()
+
+
+def test_embedding_equal_rows_interleave_by_recency():
+    """Tokens with bitwise equal table rows score exactly alike, so their
+    positions interleave by recency in the Eq. 4 ranking; a frequent token
+    whose row equals the anchor's fills the whole list with its most recent
+    positions.  The GPU scores each distinct token once and expands the
+    tokens back to positions: the lists must equal the oracle's."""
+    V, de = 600, 64
+    w = synth.make_workload(2, B=3, L=900, d=32, V=V, nohit=1.0, seed=81)
+    E = synth.make_embeddings(w, V, de, 81)
+    a0 = int(w.tokens[0, w.lengths[0] - 1])
+    a1 = int(w.tokens[1, w.lengths[1] - 1])
+    for t in (7, 11):
+        assert t not in (a0, a1)
+    E[7] = E[a0]
+    E[11] = E[a0]
+    w.tokens[0, [100, 250, 400, 600, 880]] = 7
+    w.tokens[0, [150, 300, 620, 890]] = 11
+    E[3] = E[a1]                        # token 3 is frequent under the Zipf draw
+    assert (w.tokens[1, : w.lengths[1] - 1] == 3).sum() > w.k
+    for tau in (0.1, NEG_INF):
+        cand, score, n = _emb_topk(w, E, tau)
+        for b in range(w.B):
+            L_b = int(w.lengths[b])
+            oc, _ = oracle.semantic_emb(w.tokens[b], L_b, E, w.k, tau)
+            assert cand[b, : n[b]].tolist() == oc, (b, tau)
+        want0 = sorted([j for j in range(w.lengths[0] - 1) if w.tokens[0, j] in (7, 11)],
+                       reverse=True)[: w.k]
+        assert cand[0, : w.k].tolist() == want0
+        assert (w.tokens[1, cand[1, : w.k]] == 3).all()
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P, emb=E), P, emb=E)
+
+
+def test_embedding_standalone_calls_match_the_step():
+    """lexical -> embedding fallback -> tree with the table (the tree call
+    builds the distinct-token lists for the backoff itself) gives the step's
+    trees."""
+    V = 3000
+    w = synth.make_workload(3, B=6, L=2500, d=64, V=V, nohit=0.7, seed=82)
+    E = synth.make_embeddings(w, V, 64, 82)
+    Ed = torch.from_numpy(E.view(np.int16)).cuda().view(torch.bfloat16)
+    P = P_of(w)
+    p = params(P)
+    g_step = run_step(w, P, emb=E)
+    tok, ln, reps, q = to_dev(w)
+    out = native.Outputs.allocate(w.B, p)
+    ws = native.allocate_workspace(w.B, w.ld, w.d, p)
+    native.lexical_match(tok, ln, w.n_max, w.k, out.hit_kind, out.match_n, out.cand, out.n_cand, ws)
+    active = (out.hit_kind != 1).to(torch.uint8)
+    native.embedding_topk(tok, ln, Ed, w.k, w.tau, out.cand, out.score, out.n_cand, ws,
+                          active=active)
+    out.hit_kind.copy_(torch.where(out.hit_kind == 1, out.hit_kind,
+                                   torch.where(out.n_cand > 0, 2, 0).to(torch.int32)))
+    out.status.zero_()
+    out.stats.zero_()
+    native.build_draft_tree(tok, ln, reps, q, out.hit_kind, out.cand, out.score, out.n_cand, p,
+                            out, ws, emb=Ed)
+    torch.cuda.synchronize()
+    assert native.read_device_status(ws) == 0
+    g = out.to_host()
+    for key in ("hit_kind", "anchor", "draft_tokens", "parents", "positions", "mask", "n_nodes"):
+        assert np.array_equal(g[key], g_step[key]), key
 
 
 def test_embedding_mode_token_out_of_table():
