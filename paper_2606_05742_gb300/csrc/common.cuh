@@ -65,6 +65,7 @@ struct Workspace {
     int32_t *rep_tok;        // [B][ld] distinct tokens by latest position, then the anchor
     int32_t *rep_len;        // [B] distinct tokens + 1 (a length: rows = rep_len - 1)
     int32_t *rep_cnt;        // [B][C1] distinct tokens per chunk, then chunk offsets
+    uint32_t *rep_bits;      // [B][C1][128] one bit per position: latest occurrence
     int32_t *xpart;          // [B*W][S4][kMaxK][kPart4Ints] expansion: per-slice lists
     int64_t H;               // hash slots per sequence (a power of two >= 2 (ld-1))
     size_t htab_bytes;
@@ -139,6 +140,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.rep_tok = (int32_t *)take(sizeof(int32_t) * (size_t)B * ld);
     w.rep_len = (int32_t *)take(sizeof(int32_t) * (size_t)B);
     w.rep_cnt = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1);
+    w.rep_bits = (uint32_t *)take(sizeof(uint32_t) * (size_t)B * w.C1 * (kChunk1 / 32));
     w.xpart = (int32_t *)take(sizeof(int32_t) * BW * w.S4 * kMaxK * kPart4Ints);
     w.total_bytes = off;
     return w;

@@ -13,12 +13,16 @@
 //      (key token + 1 in the high word, the latest position in the low word:
 //      atomicCAS to claim a slot, atomicMax to keep the latest position);
 //      lanes holding the same token in a warp insert once (__match_any_sync).
-//  rep_count_kernel   same grid: counts the positions that are the latest
-//      occurrence of their token per chunk; the last chunk of a sequence
-//      turns the counts into offsets and writes rep_len and the anchor; the
-//      last sequence builds the semantic plan over the lists.
-//  rep_scatter_kernel same grid: writes each chunk's latest occurrences'
+//  rep_count_kernel   same grid: marks the positions that are the latest
+//      occurrence of their token (a bit each) and counts them per chunk; the
+//      last chunk of a sequence turns the counts into offsets and writes
+//      rep_len and the anchor; the last sequence builds the semantic plan
+//      over the lists.
+//  rep_scatter_kernel same grid: writes each chunk's marked positions'
 //      tokens in position order at the chunk's offset.
+//  The three kernels issue a thread's 16 token loads, then its 16 first
+//  hash probes, before using any (the load factor keeps nearly every lookup
+//  at its first slot), so a chunk costs a few memory round trips.
 //  expand_kernel      grid (S4 slices of 8192 positions, P), 512 threads: per
 //      listed token (a warp each) the k most recent positions in the slice;
 //      the last slice merges per token, then over tokens by (score desc,
@@ -77,6 +81,9 @@ __device__ __forceinline__ int hash_lookup(const unsigned long long *T, int64_t 
     return -1;
 }
 
+constexpr int kPerThread = kChunk1 / kThreads1;  // positions per thread and chunk (16)
+constexpr int kWordsPerChunk = kChunk1 / 32;        // latest-occurrence bit words (128)
+
 __global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) {
     const DedupeLaunch &a = args.p;
     const Workspace &ws = args.ws;
@@ -92,34 +99,54 @@ __global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) 
     __syncthreads();
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     unsigned long long *T = ws.htab + (int64_t)b * ws.H;
-    const int64_t H = ws.H;
+    const uint64_t mask = (uint64_t)(ws.H - 1);
     bool bad = false, lost = false;
-    for (int base = j0; base < j1; base += kThreads1) {
-        const int j = base + t;
-        const bool in = j < j1;
-        const int raw = in ? M[j] : 0;
-        const int u = canon(raw, a.vocab);
-        bad |= in && raw != u;
-        const unsigned act = __ballot_sync(0xffffffffu, in);
-        if (!in) continue;
-        // lanes hold consecutive positions: the highest lane of a group of
-        // equal tokens has the latest one and inserts for the group
-        const unsigned same = __match_any_sync(act, u);
-        if (lane != 31 - __clz(same)) continue;
+    // all token loads, then all first-probe loads, in flight together
+    int u[kPerThread];
+#pragma unroll
+    for (int e = 0; e < kPerThread; ++e) {
+        const int j = j0 + e * kThreads1 + t;
+        const int raw = j < j1 ? M[j] : 0;
+        u[e] = canon(raw, a.vocab);
+        bad |= j < j1 && raw != u[e];
+    }
+    bool lead[kPerThread];
+    unsigned long long seen[kPerThread];
+#pragma unroll
+    for (int e = 0; e < kPerThread; ++e) {
+        const int j = j0 + e * kThreads1 + t;
+        const unsigned act = __ballot_sync(0xffffffffu, j < j1);
+        lead[e] = false;
+        if (j < j1) {
+            // lanes hold consecutive positions: the highest lane of a group
+            // of equal tokens has the latest one and inserts for the group
+            const unsigned same = __match_any_sync(act, u[e]);
+            lead[e] = lane == 31 - __clz(same);
+        }
+        seen[e] = lead[e] ? __ldcg(T + (hash32((uint32_t)u[e]) & mask)) : 0ull;
+    }
+#pragma unroll
+    for (int e = 0; e < kPerThread; ++e) {
+        if (!lead[e]) continue;
+        const int j = j0 + e * kThreads1 + t;
         const unsigned long long mine =
-            ((unsigned long long)(uint32_t)(u + 1) << 32) | (unsigned long long)(uint32_t)j;
-        uint64_t h = hash32((uint32_t)u) & (uint64_t)(H - 1);
+            ((unsigned long long)(uint32_t)(u[e] + 1) << 32) | (unsigned long long)(uint32_t)j;
+        uint64_t h = hash32((uint32_t)u[e]) & mask;
+        if ((seen[e] >> 32) == (mine >> 32)) {  // the token's slot: keep the latest position
+            if ((uint32_t)seen[e] < (uint32_t)j) atomicMax(T + h, mine);
+            continue;
+        }
         int64_t probe = 0;
-        for (; probe < H; ++probe) {
+        for (; probe < ws.H; ++probe) {
             const unsigned long long old = atomicCAS(T + h, 0ull, mine);
             if (old == 0ull) break;
             if ((old >> 32) == (mine >> 32)) {
                 if ((uint32_t)old < (uint32_t)j) atomicMax(T + h, mine);
                 break;
             }
-            h = (h + 1) & (uint64_t)(H - 1);
+            h = (h + 1) & mask;
         }
-        lost |= probe == H;
+        lost |= probe == ws.H;
     }
     if (bad) s_bad = 1;
     if (lost) atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
@@ -127,18 +154,17 @@ __global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) 
     if (t == 0 && s_bad && a.status) atomicOr(a.status + b, ADAPLD_SEQ_BAD_TOKEN);
 }
 
-// Whether position j (token u) is the latest occurrence of its token.
-__device__ __forceinline__ bool is_latest(const unsigned long long *T, int64_t H, int u, int j) {
-    return hash_lookup(T, H, u) == j;
-}
-
+// rep_count_kernel: marks the latest occurrences (one bit per position,
+// ws.rep_bits) and counts them per chunk; the last chunk of a sequence turns
+// the counts into offsets, writes rep_len and the anchor; the last sequence
+// builds the plan.
 __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
     const DedupeLaunch &a = args.p;
     const Workspace &ws = args.ws;
     __shared__ int s_flag;
     __shared__ int64_t s_scan[32];
     pdl_wait_then_release();
-    const int t = threadIdx.x;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int b = blockIdx.y, c = blockIdx.x;
     int len;
     const bool sel = seq_selected(a, b, len);
@@ -151,9 +177,35 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
         const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);
         const int32_t *M = a.tokens + (int64_t)b * a.ld;
         const unsigned long long *T = ws.htab + (int64_t)b * ws.H;
+        const uint64_t mask = (uint64_t)(ws.H - 1);
+        uint32_t *bits = ws.rep_bits + ((int64_t)b * ws.C1 + c) * kWordsPerChunk;
+        int u[kPerThread];
+#pragma unroll
+        for (int e = 0; e < kPerThread; ++e) {
+            const int j = j0 + e * kThreads1 + t;
+            u[e] = j < j1 ? canon(M[j], a.vocab) : 0;
+        }
+        unsigned long long seen[kPerThread];
+#pragma unroll
+        for (int e = 0; e < kPerThread; ++e) {
+            const int j = j0 + e * kThreads1 + t;
+            seen[e] = j < j1 ? __ldcg(T + (hash32((uint32_t)u[e]) & mask)) : 0ull;
+        }
         int mine = 0;
-        for (int j = j0 + t; j < j1; j += kThreads1)
-            mine += is_latest(T, ws.H, canon(M[j], a.vocab), j);
+#pragma unroll
+        for (int e = 0; e < kPerThread; ++e) {
+            const int j = j0 + e * kThreads1 + t;
+            bool latest = false;
+            if (j < j1) {
+                const unsigned long long key = (unsigned long long)(uint32_t)(u[e] + 1);
+                const int pos = (seen[e] >> 32) == key ? (int)(uint32_t)seen[e]
+                                                       : hash_lookup(T, ws.H, u[e]);
+                latest = pos == j;
+            }
+            const unsigned word = __ballot_sync(0xffffffffu, latest);
+            if (lane == 0) bits[e * (kThreads1 / 32) + warp] = word;
+            mine += latest;
+        }
         int64_t total;  // the block's sum
         (void)block_exclusive_scan(mine, &total, s_scan);
         if (t == 0) ws.rep_cnt[(int64_t)b * ws.C1 + c] = (int)total;
@@ -192,33 +244,42 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
                    a.init_out, a.k, a.cand, a.score, a.n_cand);
 }
 
+// rep_scatter_kernel: the chunk's latest occurrences, in position order, at
+// the chunk's offset.  Word i of the chunk's bits covers positions
+// j0 + 32 i .. +32; one scan over the 128 word counts gives every offset.
 __global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args) {
     const DedupeLaunch &a = args.p;
     const Workspace &ws = args.ws;
     __shared__ int64_t s_scan[32];
+    __shared__ int s_off[kWordsPerChunk];
+    __shared__ uint32_t s_word[kWordsPerChunk];
     pdl_wait_then_release();
-    const int t = threadIdx.x;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int b = blockIdx.y, c = blockIdx.x;
     int len;
     if (!seq_selected(a, b, len)) return;
     const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);
     if (j0 >= j1) return;
+    const uint32_t *bits = ws.rep_bits + ((int64_t)b * ws.C1 + c) * kWordsPerChunk;
+    const uint32_t w = t < kWordsPerChunk ? __ldcg(bits + t) : 0u;
+    int64_t all;
+    const int64_t ex = block_exclusive_scan(__popc(w), &all, s_scan);
+    if (t < kWordsPerChunk) {
+        s_off[t] = (int)ex;
+        s_word[t] = w;
+    }
+    __syncthreads();
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
-    const unsigned long long *T = ws.htab + (int64_t)b * ws.H;
     int32_t *out = ws.rep_tok + (int64_t)b * a.ld + __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c);
-    int64_t carry = 0;
-    for (int base = j0; base < j1; base += kThreads1) {
-        const int j = base + t;
-        int u = 0;
-        bool keep = false;
-        if (j < j1) {
-            u = canon(M[j], a.vocab);
-            keep = is_latest(T, ws.H, u, j);
+    // word i = e * 8 + warp holds positions j0 + e * 256 + warp * 32 + lane
+#pragma unroll 4
+    for (int e = 0; e < kPerThread; ++e) {
+        const int i = e * (kThreads1 / 32) + warp;
+        const uint32_t wi = s_word[i];
+        if ((wi >> lane) & 1u) {
+            const int j = j0 + e * kThreads1 + t;
+            out[s_off[i] + __popc(wi & ((1u << lane) - 1u))] = canon(M[j], a.vocab);
         }
-        int64_t all;
-        const int64_t ex = block_exclusive_scan(keep ? 1 : 0, &all, s_scan);
-        if (keep) out[carry + ex] = u;
-        carry += all;
     }
 }
 
