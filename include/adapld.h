@@ -216,7 +216,10 @@ int32_t adapld_tree_nodes(const adapld_params *p);
 /* Workspace bytes needed by any entry point for B sequences of capacity ld and
  * dimension d under parameters p (0 if the arguments are invalid).  The
  * workspace is device memory, 256-byte aligned, with no initialisation
- * required; one workspace may be reused by consecutive calls on one stream. */
+ * required; one workspace may be reused by consecutive calls on one stream.
+ * About 21 of the ~23 bytes per history position (B*ld) hold the distinct-token
+ * lists of the token-embedding mode (a hash of 2*ld slots of 8 bytes, the
+ * lists and a bit per position); the rest is a few KB per sequence. */
 size_t adapld_workspace_bytes(int32_t B, int64_t ld, int32_t d, const adapld_params *p);
 
 /* Human-readable text for a status code (static storage). */
