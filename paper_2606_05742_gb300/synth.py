@@ -299,7 +299,7 @@ def make_embeddings(w: Workload, V: int, de: int, seed: int = 0, synonyms: int =
     plants = []
     for b in w.forced:
         ln = int(lengths[b])
-        if ln < 3:
+        if ln < 3 or ln > tokens.shape[1]:   # too short, or an invalid length
             continue
         a = int(tokens[b, ln - 1])
         hist = tokens[b, : ln - 1]

@@ -559,6 +559,39 @@ def test_embedding_standalone_calls_match_the_step():
         assert np.array_equal(g[key], g_step[key]), key
 
 
+@pytest.mark.parametrize("lengths", [[0, 1, 2, 3, 50, 51], [2, 2, 3, 3, 4, 4]])
+def test_embedding_mode_edge_lengths(lengths):
+    """Empty, one- and two-token histories and a length past ld in
+    two-representation mode (the distinct-token lists of such histories are
+    empty or a single token)."""
+    V = 300
+    w = synth.make_workload(4, B=6, L=50, d=16, ld=50, V=V, seed=83, nohit=0.5,
+                            lengths=[min(x, 50) for x in lengths])
+    w.lengths = np.asarray(lengths, np.int32)   # 51 > ld: invalid on purpose
+    E = synth.make_embeddings(w, V, 16, 83)
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P, emb=E), P, emb=E)
+
+
+@pytest.mark.parametrize("kind", ["one_token", "all_distinct"])
+def test_embedding_mode_extreme_histories(kind):
+    """A history of one repeated token (one list entry, every position tied)
+    and a history of all-distinct tokens (the list is the whole history)."""
+    V = 9000
+    w = synth.make_workload(2, B=2, L=5000, d=32, V=V, seed=84, nohit=1.0)
+    L = int(w.lengths[0])
+    if kind == "one_token":
+        w.tokens[0, : L - 1] = 17
+        w.tokens[0, L - 1] = 18
+    else:
+        w.tokens[0, :L] = np.random.default_rng(84).permutation(V)[:L]
+    E = synth.make_embeddings(w, V, 32, 84)
+    for tau in (0.1, NEG_INF):
+        P = P_of(w, tau=tau)
+        check_all(w, run_step(w, P, emb=E), P, emb=E)
+
+
 def test_embedding_mode_token_out_of_table():
     """A token id outside the table reads row 0 and is flagged, no fault."""
     w = synth.make_workload(2, B=3, L=400, d=32, V=1000, nohit=1.0, seed=73)
