@@ -309,7 +309,7 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
  * One full draft-construction step for B sequences: lexical anchoring, the
  * semantic fallback for the sequences without a lexical hit (unless
  * ADAPLD_NO_SEMANTIC), then rerank and draft-tree construction, enqueued as
- * three kernels with no host synchronisation.  Arguments as above;
+ * a chain of kernels with no host synchronisation.  Arguments as above;
  * next_topk may be NULL (then Kn is ignored).
  */
 int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const uint16_t *reps,

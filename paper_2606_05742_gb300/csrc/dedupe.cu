@@ -20,9 +20,9 @@
 //      over the lists.
 //  rep_scatter_kernel same grid: writes each chunk's marked positions'
 //      tokens in position order at the chunk's offset.
-//  The three kernels issue a thread's 16 token loads, then its 16 first
-//  hash probes, before using any (the load factor keeps nearly every lookup
-//  at its first slot), so a chunk costs a few memory round trips.
+//  The list kernels issue a thread's 16 token loads, then its 16 first hash
+//  probes, before using any (the load factor keeps nearly every lookup at
+//  its first slot), so a chunk costs a few memory round trips.
 //  expand_kernel      grid (S4 slices of 8192 positions, P), 512 threads: per
 //      listed token (a warp each) the k most recent positions in the slice;
 //      the last slice merges per token, then over tokens by (score desc,
