@@ -33,46 +33,13 @@ struct TreeArgs {
     int rows_ctas;  // gridDim.x of tree_kernel
 };
 
-// cos(row, ref) of two bf16 rows in global memory (one warp).  The norm of
-// ref is recomputed by every warp in the same order, so it is bit-identical.
-__device__ __forceinline__ float warp_cosine(const uint16_t *row, const uint16_t *ref, int d) {
-    const int lane = threadIdx.x & 31;
-    const int nch = d >> 3;
-    float dot = 0.f, sx = 0.f, sy = 0.f;
-    for (int base = 0; base < nch; base += 32 * 8) {
-        uint4 wx[8], wy[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            const int ch = base + u * 32 + lane;
-            wx[u] = ch < nch ? ldg_nc_v4(row + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
-            wy[u] = ch < nch ? ldg_nc_v4(ref + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            const uint32_t xs[4] = {wx[u].x, wx[u].y, wx[u].z, wx[u].w};
-            const uint32_t ys[4] = {wy[u].x, wy[u].y, wy[u].z, wy[u].w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float x0 = bf16lo(xs[e]), x1 = bf16hi(xs[e]);
-                const float y0 = bf16lo(ys[e]), y1 = bf16hi(ys[e]);
-                dot = fmaf(x0, y0, dot);
-                dot = fmaf(x1, y1, dot);
-                sx = fmaf(x0, x0, sx);
-                sx = fmaf(x1, x1, sx);
-                sy = fmaf(y0, y0, sy);
-                sy = fmaf(y1, y1, sy);
-            }
-        }
-    }
-    return cosine_from(warp_sum(dot), warp_sum(sx), warp_sum(sy));
-}
-
 // <row, ref> and |row|^2 of one bf16 row in global memory against an fp32
-// vector in shared memory (one warp, 16 independent 16-byte loads per lane
-// in flight).
+// vector in shared memory (one warp, U independent 16-byte loads per lane in
+// flight).  A lane sums its chunks lane, lane + 32, ... in the same order
+// whatever U, so the result does not depend on U.
+template <int U = 16>
 __device__ __forceinline__ void warp_row_dot(const uint16_t *row, const float *ref, int d,
                                              float &dot_out, float &ss_out) {
-    constexpr int U = 16;
     const int lane = threadIdx.x & 31;
     const int nch = d >> 3;
     float dot = 0.f, ss = 0.f;
@@ -263,6 +230,8 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     __shared__ int s_next[kMaxW];
     __shared__ int s_br[kMaxW];
     __shared__ int s_misc[4];
+    __shared__ float s_red[32];
+    extern __shared__ __align__(16) float s_q[];  // [d] the query (fp32) for a rerank here
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int nwarps = kThreads4 / 32;
@@ -279,11 +248,13 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
         s_score[t] = a.score[(int64_t)b * k + t];
     }
     __syncthreads();
-    if (v.rr) {  // the ranking the branches depend on (each slice alike)
-        const uint16_t *q = a.query + (int64_t)b * d;
+    if (v.rr) {  // the ranking the branches depend on (each slice alike; the
+                 // arithmetic of the tree kernel's rerank, so the scores agree)
+        const float qss = block_load_vec(a.query + (int64_t)b * d, s_q, d, s_red);
         for (int ci = warp; ci < v.nc; ci += nwarps) {
-            const float cs = warp_cosine(R + (int64_t)s_cand[ci] * d, q, d);
-            if (lane == 0) s_score[ci] = cs;
+            float dot, ss;
+            warp_row_dot<8>(R + (int64_t)s_cand[ci] * d, s_q, d, dot, ss);
+            if (lane == 0) s_score[ci] = cosine_from(dot, ss, qss);
         }
         __syncthreads();
         if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc);
@@ -612,7 +583,11 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
             e = launch_dedupe(da, ws, s);
             if (e != cudaSuccess) return e;
         }
-        e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), 0, s, args);
+        const size_t qsmem = (size_t)a.d * sizeof(float);
+        e = cudaFuncSetAttribute(succ_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)qsmem);
+        if (e != cudaSuccess) return e;
+        e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), qsmem, s, args);
         if (e != cudaSuccess) return e;
         if (a.emb.table) {  // successor backoff over token embeddings
             e = launch_dependent(backoff_plan_kernel, dim3(1), dim3(256), 0, s, args);

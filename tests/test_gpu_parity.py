@@ -170,6 +170,17 @@ def test_rows_spread_over_all_ctas():
         check_all(w, run_step(w, P), P)
 
 
+def test_many_short_sequences():
+    """Thousands of short sequences: plans and tickets over B far above the
+    CTA count and a block's width, in both retrieval modes."""
+    V = 2000
+    w = synth.make_workload(4, B=3000, L=40, d=16, V=V, nohit=0.5, seed=7)
+    P = P_of(w)
+    check_all(w, run_step(w, P), P)
+    E = synth.make_embeddings(w, V, 16, 7)
+    check_all(w, run_step(w, P, emb=E), P, emb=E)
+
+
 def test_fewer_rows_than_ctas():
     w = synth.make_workload(2, B=3, L=9, d=16, nohit=1.0, seed=6, lengths=[9, 4, 2])
     for tau in (0.1, NEG_INF):
