@@ -286,9 +286,15 @@ def parse_flags(text):
 def step_launches(flags, W, emb):
     """Kernels one step launches (mirrors the launch sequence of adapld_step)."""
     succ = W > 0 and not (flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"]))
-    n = 2 + (0 if flags & FLAG_NAMES["no_semantic"] else 1) + (1 if succ else 0)
-    if emb and succ:
-        n += 2                              # backoff plan + gathered semantic pass
+    semantic = not flags & FLAG_NAMES["no_semantic"]
+    n = 2                                   # lexical, tree
+    if semantic:
+        n += 1 + (4 if emb else 0)          # semantic (+ three list kernels, expansion)
+    if succ:
+        n += 1                              # successor scan
+        if emb:
+            n += 3 if semantic else 6       # backoff plan, gathered pass, expansion
+                                            # (+ the lists, built by the tree stage)
     return n
 
 

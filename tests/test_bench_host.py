@@ -20,9 +20,12 @@ def test_flag_names_match_the_library():
 
 def test_step_launches():
     assert bench.step_launches(0, 4, False) == 4          # lexical, semantic, scan, tree
-    assert bench.step_launches(0, 4, True) == 6           # + backoff plan + gathered pass
+    # + three distinct-token list kernels, the expansion, the backoff plan,
+    # the backoff's gathered pass and its expansion
+    assert bench.step_launches(0, 4, True) == 11
     assert bench.step_launches(native.NO_SEMANTIC, 4, False) == 3
-    assert bench.step_launches(native.NO_SUCC, 4, True) == 3
+    assert bench.step_launches(native.NO_SUCC, 4, True) == 7
+    assert bench.step_launches(native.NO_SEMANTIC, 4, True) == 9
     assert bench.step_launches(native.NO_BRANCH | native.NO_SEMANTIC, 4, False) == 2
     assert bench.step_launches(0, 0, False) == 3
 
