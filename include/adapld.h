@@ -24,6 +24,10 @@
  *    stream has been synchronised.  No entry point synchronises the host
  *    except adapld_read_device_status().  Calls on different streams are
  *    independent provided they use different workspaces and outputs.
+ *  - adapld_step(), adapld_step_ex() (without events) and
+ *    adapld_accept_greedy() enqueue device work only: a decode loop may
+ *    capture them into a CUDA graph once and replay it, since every size
+ *    the kernels act on (lengths, tree sizes) is read on the device.
  *  - Sequence b (0 <= b < B) of the token history is tokens[b*ld .. b*ld+len_b)
  *    with len_b = lengths[b]; the query anchor is tokens[b*ld + len_b - 1].
  *  - Representations are bf16, passed as uint16_t bit patterns.  Row j of

@@ -397,6 +397,51 @@ def test_semantic_wait_timeout_is_reported_and_recoverable(monkeypatch):
     check_all(w, g, P)
 
 
+@pytest.mark.parametrize("mode", ["plain", "embeddings"])
+def test_step_replays_from_a_cuda_graph(mode):
+    """A step (and the verification after it) captured once in a CUDA graph
+    and replayed gives the eager outputs: the calls enqueue device work only
+    (no host synchronisation, no allocation), so a serving loop can capture
+    them with its decode step."""
+    V = 4000
+    w = synth.make_workload(2, B=6, L=1500, d=64, V=V, nohit=0.5, seed=91)
+    E = synth.make_embeddings(w, V, 64, 91) if mode == "embeddings" else None
+    P = P_of(w)
+    ref = run_step(w, P, emb=E)
+    tok, ln, reps, q = to_dev(w)
+    Ed = torch.from_numpy(E.view(np.int16)).cuda().view(torch.bfloat16) if E is not None else None
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    N = eng.out.draft_tokens.shape[1]
+    lg = torch.randn((w.B, N, 512), device="cuda").to(torch.bfloat16)
+    n_acc = torch.zeros(w.B, dtype=torch.int32, device="cuda")
+    new = torch.zeros((w.B, N), dtype=torch.int32, device="cuda")
+    n_new = torch.zeros(w.B, dtype=torch.int32, device="cuda")
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):            # warm-up outside the capture
+        eng.run(tok, ln, reps, q, emb=Ed)
+        native.accept_greedy(lg, eng.out.draft_tokens, eng.out.parents, eng.out.n_nodes, n_acc,
+                             new, n_new, eng.ws)
+    torch.cuda.synchronize()
+    want_acc = n_acc.clone()
+    for t in eng.out.tensors():
+        t.zero_()
+    n_acc.zero_()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        eng.run(tok, ln, reps, q, emb=Ed)
+        native.accept_greedy(lg, eng.out.draft_tokens, eng.out.parents, eng.out.n_nodes, n_acc,
+                             new, n_new, eng.ws)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    assert native.read_device_status(eng.ws) == 0
+    got = eng.out.to_host()
+    for key in ref:
+        assert np.array_equal(ref[key], got[key], equal_nan=True), key
+    assert torch.equal(n_acc, want_acc)
+
+
 def test_end_to_end_from_host_matches_device_path():
     """The public end-to-end call (pinned host inputs, copies on side streams,
     outputs copied back) returns what the device-resident call returns."""
