@@ -362,7 +362,11 @@ __global__ void __launch_bounds__(256) backoff_plan_kernel(TreeArgs args) {
 }
 
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
+// U: row loads in flight per lane.  U = 16 (one CTA per SM by registers)
+// when the grid fits one wave, U = 8 (two CTAs per SM) otherwise; the
+// scores are the same either way (see warp_row_dot).
+template <int U>
+__global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArgs args) {
     const TreeLaunch &a = args.p;
     const Workspace &ws = args.ws;
     __shared__ int s_cand[kMaxK];
@@ -436,7 +440,7 @@ __global__ void __launch_bounds__(kThreads4) tree_kernel(TreeArgs args) {
         const int row = s_row[warp];
         if (row >= 0) {
             float dot, ss;
-            warp_row_dot(R + (int64_t)row * d, s_ref, d, dot, ss);
+            warp_row_dot<U>(R + (int64_t)row * d, s_ref, d, dot, ss);
             if (lane == 0) score5[task0 + warp] = cosine_from(dot, ss, rss);
         }
         if (nctas > 1) {
@@ -613,11 +617,15 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
         }
     }
     const size_t smem = (size_t)a.d * sizeof(float);
-    cudaError_t e = cudaFuncSetAttribute(tree_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    int sms = 0, dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return cudaErrorInvalidDevice;
+    auto kern = (int64_t)args.rows_ctas * a.B <= sms ? tree_kernel<16> : tree_kernel<8>;
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_dependent(tree_kernel, dim3(args.rows_ctas, a.B), dim3(kThreads4), smem, s,
-                            args);
+    return launch_dependent(kern, dim3(args.rows_ctas, a.B), dim3(kThreads4), smem, s, args);
 }
 
 }  // namespace adapld
