@@ -325,6 +325,18 @@ def read_device_status(ws, stream=None) -> int:
     return int(v.value)
 
 
+class BoundCall:
+    """A library call with its arguments marshalled once (see Engine.bind)."""
+
+    def __init__(self, fn, args, keep, name):
+        self._fn, self._args, self._keep, self._name = fn, args, keep, name
+
+    def __call__(self) -> None:
+        rc = self._fn(*self._args)
+        if rc:
+            _check(rc, self._name)
+
+
 class Engine:
     """Owns the device buffers for repeated steps over B sequences of capacity
     ld and dimension d, and offers the end-to-end call from host tensors."""
@@ -341,6 +353,28 @@ class Engine:
         step(tokens, lengths, reps, query, self.p, self.out, self.ws, next_topk, events, stream,
              emb)
         return self.out
+
+    def bind(self, tokens, lengths, reps, query, next_topk=None, stream=None, emb=None):
+        """The step on fixed buffers with its arguments marshalled once: the
+        returned callable enqueues one step per call (a decode loop updates
+        the buffers' contents in place between calls)."""
+        B, ld, d = reps.shape
+        so = self.out.c_struct()
+        kn = next_topk.shape[2] if next_topk is not None else 0
+        lib = load()
+        args = [_ptr(tokens), ld, _ptr(lengths), _ptr(reps), d, _ptr(query), _ptr(next_topk),
+                kn, B, ctypes.byref(self.p), ctypes.byref(so), _ptr(self.ws),
+                self.ws.numel() * self.ws.element_size()]
+        keep = [so, self.p]
+        if emb is None:
+            fn = lib.adapld_step
+        else:
+            e = Embeddings.of(emb)
+            keep.append(e)
+            fn = lib.adapld_step_ex
+            args += [ctypes.byref(e), None]
+        args.append(_stream(stream))
+        return BoundCall(fn, tuple(args), keep, "adapld_step")
 
     def run_from_host(self, tokens_h, lengths_h, reps_h, query_h, dev_inputs, host_out,
                       stream=None, copy_streams: int = 4):

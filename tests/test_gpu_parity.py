@@ -398,6 +398,35 @@ def test_semantic_wait_timeout_is_reported_and_recoverable(monkeypatch):
 
 
 @pytest.mark.parametrize("mode", ["plain", "embeddings"])
+def test_bound_step_matches_run(mode):
+    """Engine.bind marshals the arguments once; its calls give the step's
+    outputs, also after the buffers' contents change in place."""
+    V = 4000
+    w = synth.make_workload(2, B=6, L=1500, d=64, V=V, nohit=0.5, seed=92)
+    E = synth.make_embeddings(w, V, 64, 92) if mode == "embeddings" else None
+    P = P_of(w)
+    ref = run_step(w, P, emb=E)
+    tok, ln, reps, q = to_dev(w)
+    Ed = torch.from_numpy(E.view(np.int16)).cuda().view(torch.bfloat16) if E is not None else None
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    call = eng.bind(tok, ln, reps, q, emb=Ed)
+    call()
+    torch.cuda.synchronize()
+    got = eng.out.to_host()
+    for key in ref:
+        assert np.array_equal(ref[key], got[key], equal_nan=True), key
+    # a shorter history in place: the next call sees it
+    ln[0] = 700
+    w.lengths[0] = 700
+    ref2 = run_step(w, P, emb=E)
+    call()
+    torch.cuda.synchronize()
+    got2 = eng.out.to_host()
+    for key in ref2:
+        assert np.array_equal(ref2[key], got2[key], equal_nan=True), key
+
+
+@pytest.mark.parametrize("mode", ["plain", "embeddings"])
 def test_step_replays_from_a_cuda_graph(mode):
     """A step (and the verification after it) captured once in a CUDA graph
     and replayed gives the eager outputs: the calls enqueue device work only
