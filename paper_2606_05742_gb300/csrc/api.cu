@@ -156,8 +156,8 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
     // the distinct tokens of the selected histories and the plan over them,
     // the scores of the distinct tokens, then their positions
-    DedupeLaunch da{tokens, ld, lengths, B, emb->vocab, active, status, false, true, nullptr,
-                    true,   k,  cand,    score, n_cand};
+    DedupeLaunch da{tokens, ld,   lengths, B,       emb->vocab, active, nullptr, status,
+                    false,  true, nullptr, true,    k,          cand,   score,   n_cand};
     ADAPLD_TRY(cuda_status(launch_dedupe(da, w, s)));
     SemLaunch a{emb->table, ld, emb->dim, nullptr, w.rep_len, active, B, k, tau, cand, score, n_cand,
                 nullptr, true};
@@ -237,7 +237,11 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
         SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
                      out->n_cand, out->hit_kind, true};
         if (emb) {  // Eq. 4 over token embeddings, scored once per distinct token
-            DedupeLaunch da{tokens, ld, lengths, B, emb->vocab, nullptr, out->status, true, true,
+            // lists for the fallback sequences, and for lexical hits too when
+            // those draft successors (their backoff needs them)
+            const bool lex_lists = (p->flags & ADAPLD_SUCC_ON_STRICT) != 0;
+            DedupeLaunch da{tokens, ld, lengths, B, emb->vocab, nullptr,
+                            lex_lists ? nullptr : out->hit_kind, out->status, true, true,
                             out->hit_kind, false, p->k, nullptr, nullptr, nullptr};
             ADAPLD_TRY(cuda_status(launch_dedupe(da, w, s)));
             sa.reps = emb->table;

@@ -529,6 +529,9 @@ struct DedupeLaunch {
     const int32_t *lengths;
     int32_t B, vocab;
     const uint8_t *active;   // selection (NULL = every sequence)
+    // when given, sequences with a lexical hit are left out (their lists are
+    // needed only if lexical hits draft successors)
+    const int32_t *skip_lex_of;
     int32_t *status;         // ADAPLD_SEQ_BAD_TOKEN bits (nullable)
     bool pdl;                // launched as a programmatic dependent of a kernel
     // semantic plan over the lists (built by the last sequence), selection as

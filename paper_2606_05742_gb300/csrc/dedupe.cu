@@ -65,6 +65,7 @@ __device__ __forceinline__ uint32_t hash32(uint32_t x) {
 __device__ __forceinline__ bool seq_selected(const DedupeLaunch &a, int b, int &len) {
     len = a.lengths[b];
     if (len < 1 || (int64_t)len > a.ld) return false;
+    if (a.skip_lex_of && __ldcg(a.skip_lex_of + b) == ADAPLD_HIT_LEX) return false;
     return a.active ? a.active[b] != 0 : true;
 }
 

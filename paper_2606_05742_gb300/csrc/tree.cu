@@ -582,8 +582,9 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
     if (succ_possible) {
         cudaError_t e;
         if (a.emb.table && !a.lists_ready) {  // distinct-token lists for the backoff
-            DedupeLaunch da{a.tokens, a.ld, a.lengths, a.B, a.emb.vocab, nullptr, a.status, true,
-                            false, nullptr, false, k, nullptr, nullptr, nullptr};
+            DedupeLaunch da{a.tokens, a.ld,  a.lengths, a.B,     a.emb.vocab, nullptr, nullptr,
+                            a.status, true, false,     nullptr, false,       k,       nullptr,
+                            nullptr,  nullptr};
             e = launch_dedupe(da, ws, s);
             if (e != cudaSuccess) return e;
         }

@@ -529,6 +529,24 @@ def test_embedding_mode(cfg, B, L, d, de, V, seed):
     print("branches needing the backoff:", backoff)
 
 
+@pytest.mark.parametrize("flags,table", [
+    (oracle.SUCC_ON_STRICT, False), (oracle.SUCC_ON_STRICT, True),
+    (oracle.NO_SEMANTIC | oracle.SUCC_ON_STRICT, True), (oracle.NO_LEX_RERANK, False),
+    (oracle.NO_SUCC, False)])
+def test_embedding_mode_ablations(flags, table):
+    """Variants of the two-representation step: successors on lexical hits
+    (with the next-token table their branch tokens may never have occurred,
+    so their backoff needs the distinct-token lists of lexical-hit
+    sequences, which the tree stage builds itself when the fallback is off),
+    no rerank, no successors."""
+    V = 3000
+    w = synth.make_workload(2, B=10, L=1200, d=64, V=V, nohit=0.5, seed=85)
+    E = synth.make_embeddings(w, V, 64, 85)
+    tk = synth.make_next_topk(w.tokens, w.lengths, V, 5) if table else None
+    P = P_of(w, flags=flags)
+    check_all(w, run_step(w, P, next_topk=tk, emb=E), P, next_topk=tk, emb=E)
+
+
 def test_embedding_mode_with_next_token_table():
     w = synth.make_workload(2, B=6, L=700, d=64, V=4096, nohit=0.5, seed=71)
     E = synth.make_embeddings(w, 4096, 64, 71)
