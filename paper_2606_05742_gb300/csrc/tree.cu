@@ -1,6 +1,12 @@
-// Rerank and draft-tree construction (Sec. 3.4-3.6, Eq. 6-15, Algorithm 1),
-// as two kernels so that every gathered representation row is read by its
-// own warp somewhere on the GPU instead of queueing behind one CTA.
+// Rerank and draft-tree construction (Sec. 3.4-3.6, Eq. 6-15, Algorithm 1).
+//
+// With at most 16 successor rows per sequence (W*k <= 16) the stage is one
+// kernel: succ_scan_kernel<U, true>, where the CTA that completes a
+// sequence's scan (or CTA 0 of a sequence without successors) goes on to
+// build its tree (tree_body, every row in that CTA, one per warp).
+// With more rows, or in two-representation mode (the successor backoff runs
+// in between), it is two kernels so that every gathered row is read by its
+// own warp somewhere on the GPU instead of queueing behind one CTA:
 //
 // succ_scan_kernel, grid (S4 slices, B), 512 threads -- only for sequences
 // that draft successors (Algorithm 1: semantic hits; every hit under
@@ -31,6 +37,22 @@ struct TreeArgs {
     TreeLaunch p;
     Workspace ws;
     int rows_ctas;  // gridDim.x of tree_kernel
+};
+
+// Shared state of the tree stage (the candidates, the branch set and the
+// node layout of one sequence).
+struct TreeSmem {
+    int cand[kMaxK];
+    float score[kMaxK];
+    int next[kMaxW];
+    int br[kMaxW];
+    int succ[kMaxW];
+    int misc[4];
+    int node_par[kMaxNodes];
+    short node_depth[kMaxNodes];
+    short node_path[kMaxNodes];
+    int node_src[kMaxNodes];
+    float red[32];
 };
 
 // <row, ref> and |row|^2 of one bf16 row in global memory against an fp32
@@ -221,16 +243,26 @@ __device__ __forceinline__ void register_successors(const TreeLaunch &a, const W
     }
 }
 
-__global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
+template <int U>
+__device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const SeqView &v,
+                          int r5, bool fused, TreeSmem &sm, float *s_ref);
+
+// FUSED: the CTA that completes a sequence's scan (or CTA 0 of a sequence
+// without successors) then builds that sequence's tree itself (tree_body,
+// all scored rows in this CTA), so the tree stage is one kernel.  U: row
+// loads in flight in tree_body.
+template <int U, bool FUSED>
+__global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(TreeArgs args) {
     const TreeLaunch &a = args.p;
     const Workspace &ws = args.ws;
     __shared__ int s_tok[kSlice4];
-    __shared__ int s_cand[kMaxK];
-    __shared__ float s_score[kMaxK];
-    __shared__ int s_next[kMaxW];
-    __shared__ int s_br[kMaxW];
-    __shared__ int s_misc[4];
-    __shared__ float s_red[32];
+    __shared__ TreeSmem sm;
+    int *s_cand = sm.cand;
+    float *s_score = sm.score;
+    int *s_next = sm.next;
+    int *s_br = sm.br;
+    int *s_misc = sm.misc;
+    float *s_red = sm.red;
     extern __shared__ __align__(16) float s_q[];  // [d] the query (fp32) for a rerank here
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
@@ -239,7 +271,10 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     const int k = a.p.k, d = a.d;
     pdl_wait_then_release();
     const SeqView v = view_of(a, b);
-    if (!v.need_succ) return;
+    if (!v.need_succ) {
+        if (FUSED && sl == 0) tree_body<U>(a, ws, b, v, 0, true, sm, s_q);
+        return;
+    }
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
 
@@ -269,7 +304,7 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     const int p1 = min(p0 + kSlice4, v.len - 1);  // positions t <= len-2
     for (int i = t; i < p1 - p0; i += kThreads4) s_tok[i] = M[p0 + i];
     __syncthreads();
-    constexpr int U = 8;  // 32-position groups tested per pass (independent loads)
+    constexpr int G = 8;  // 32-position groups tested per pass (independent loads)
     // one slice: its lists are the merged result, written in place (no merge)
     const bool single = gridDim.x == 1;
     for (int w = warp; w < nb; w += nwarps) {
@@ -278,15 +313,15 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
             single ? nullptr : ws.part4 + (((int64_t)b * ws.S4 + sl) * ws.W + w) * kPart4Ints;
         int32_t *lst = single ? ws.succ + ((int64_t)b * ws.W + w) * kMaxK : part + 1;
         int cnt = 0;
-        for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32 * U) {
-            unsigned m[U];
+        for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32 * G) {
+            unsigned m[G];
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
+            for (int u = 0; u < G; ++u) {
                 const int p = top - 32 * u - lane;
                 m[u] = __ballot_sync(0xffffffffu, p >= p0 && s_tok[p - p0] == bt);
             }
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
+            for (int u = 0; u < G; ++u) {
                 const int p = top - 32 * u - lane;
                 const int rank = cnt + __popc(m[u] & ((1u << lane) - 1u));
                 if (((m[u] >> lane) & 1u) && rank < k) lst[rank] = p;
@@ -321,6 +356,10 @@ __global__ void __launch_bounds__(kThreads4) succ_scan_kernel(TreeArgs args) {
     if ((v.lex || v.rr) && t < v.nc) {
         ws.rr_cand[(int64_t)b * kMaxK + t] = s_cand[t];
         ws.rr_score[(int64_t)b * kMaxK + t] = s_score[t];
+    }
+    if (FUSED) {
+        __syncthreads();  // the lists and the ranking above are visible to the block
+        tree_body<U>(a, ws, b, v, 0, true, sm, s_q);
     }
 }
 
@@ -362,35 +401,30 @@ __global__ void __launch_bounds__(256) backoff_plan_kernel(TreeArgs args) {
 }
 
 // ---------------------------------------------------------------------------
-// U: row loads in flight per lane.  U = 16 (one CTA per SM by registers)
-// when the grid fits one wave, U = 8 (two CTAs per SM) otherwise; the
-// scores are the same either way (see warp_row_dot).
+// The tree stage of sequence b for one CTA (all threads): CTA r5 of the
+// sequence scores its share of rows (every row when `fused`); the CTA that
+// completes the sequence ranks, picks successors and emits the tree.  s_ref:
+// d floats of shared memory.
 template <int U>
-__global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArgs args) {
-    const TreeLaunch &a = args.p;
-    const Workspace &ws = args.ws;
-    __shared__ int s_cand[kMaxK];
-    __shared__ float s_score[kMaxK];
-    __shared__ int s_next[kMaxW];
-    __shared__ int s_br[kMaxW];
-    __shared__ int s_succ[kMaxW];
-    __shared__ int s_misc[4];
-    __shared__ int node_par[kMaxNodes];
-    __shared__ short node_depth[kMaxNodes];
-    __shared__ short node_path[kMaxNodes];
-    __shared__ int node_src[kMaxNodes];
-    __shared__ int s_row[kRowsPerCta5];
-    __shared__ float s_red[32];
-    extern __shared__ __align__(16) float s_ref[];  // [d] reference vector (fp32)
+__device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const SeqView &v,
+                          int r5, bool fused, TreeSmem &sm, float *s_ref) {
+    int *s_cand = sm.cand;
+    float *s_score = sm.score;
+    int *s_next = sm.next;
+    int *s_br = sm.br;
+    int *s_succ = sm.succ;
+    int *s_misc = sm.misc;
+    int *node_par = sm.node_par;
+    short *node_depth = sm.node_depth;
+    short *node_path = sm.node_path;
+    int *node_src = sm.node_src;
+    float *s_red = sm.red;
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int nwarps = kThreads4 / 32;
-    const int b = blockIdx.y, r5 = blockIdx.x;
     const int k = a.p.k, d = a.d, W = a.p.branch_width, D = a.p.draft_len;
     const int succ_len = a.p.succ_len;
     const uint32_t flags = a.p.flags;
-    pdl_wait_then_release();
-    const SeqView v = view_of(a, b);
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
 
@@ -412,36 +446,32 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
     // candidates against the query, or successor candidate (w, i) at w*k + i
     const bool rerank = v.rr && !v.need_succ;
     const int ntasks = v.need_succ ? nb * k : (rerank ? v.nc : 0);
-    const int nctas = max(1, (ntasks + kRowsPerCta5 - 1) / kRowsPerCta5);
+    const int nctas = fused ? 1 : max(1, (ntasks + kRowsPerCta5 - 1) / kRowsPerCta5);
     if (r5 >= nctas) return;
     const int js0 = (v.lex || v.sem) ? s_cand[0] : -1;
     float *score5 = ws.score5 + (int64_t)b * ws.W * kMaxK;
 
     // ---- this CTA's share of the scored rows
     if (ntasks > 0) {
-        const int task0 = r5 * kRowsPerCta5;
-        if (t < kRowsPerCta5) {  // row of each task of this CTA, -1 if none
-            const int task = task0 + t;
-            int row = -1;
-            if (task < ntasks) {
-                if (v.need_succ) {
-                    const int w = task / k, i = task % k;
-                    const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
-                    const int pos = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i);
-                    row = i < n ? pos : -1;
-                } else {
-                    row = s_cand[task];
-                }
-            }
-            s_row[t] = row;
-        }
+        // this CTA's tasks: 16 (one per warp), or all of them when fused
+        const int task0 = fused ? 0 : r5 * kRowsPerCta5;
+        const int task1 = fused ? ntasks : min(ntasks, task0 + kRowsPerCta5);
         const uint16_t *ref = v.need_succ ? R + (int64_t)(js0 + 1) * d : a.query + (int64_t)b * d;
         const float rss = block_load_vec(ref, s_ref, d, s_red);  // syncs the block
-        const int row = s_row[warp];
-        if (row >= 0) {
-            float dot, ss;
-            warp_row_dot<U>(R + (int64_t)row * d, s_ref, d, dot, ss);
-            if (lane == 0) score5[task0 + warp] = cosine_from(dot, ss, rss);
+        for (int task = task0 + warp; task < task1; task += nwarps) {
+            int row;
+            if (v.need_succ) {
+                const int w = task / k, i = task % k;
+                const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
+                row = i < n ? __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i) : -1;
+            } else {
+                row = s_cand[task];
+            }
+            if (row >= 0) {
+                float dot, ss;
+                warp_row_dot<U>(R + (int64_t)row * d, s_ref, d, dot, ss);
+                if (lane == 0) score5[task] = cosine_from(dot, ss, rss);
+            }
         }
         if (nctas > 1) {
             __threadfence();
@@ -571,7 +601,26 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
     }
 }
 
+// U: row loads in flight per lane.  U = 16 (one CTA per SM by registers)
+// when the grid fits one wave, U = 8 (two CTAs per SM) otherwise; the
+// scores are the same either way (see warp_row_dot).
+template <int U>
+__global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArgs args) {
+    __shared__ TreeSmem sm;
+    extern __shared__ __align__(16) float s_ref[];  // [d] reference vector (fp32)
+    pdl_wait_then_release();
+    const SeqView v = view_of(args.p, blockIdx.y);
+    tree_body<U>(args.p, args.ws, blockIdx.y, v, blockIdx.x, false, sm, s_ref);
+}
+
 }  // namespace
+
+// Successor rows per sequence up to which the fused kernel scores them in the
+// CTA that completes the scan (one row per warp, as a tree-kernel CTA would)
+// instead of a tree kernel spreading them over CTAs.  Measured on GB300: with
+// 16 rows (configs 1 and 4) fusing saves 2.4-2.7 us per step; with 24 or 64
+// rows (configs 2 and 3) the second kernel's parallel rows win by 4-14 us.
+constexpr int kMaxFusedTasks = kRowsPerCta5;
 
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s) {
     const int W = a.p.branch_width, k = a.p.k;
@@ -579,8 +628,21 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
         W > 0 && !(a.p.flags & (ADAPLD_NO_SUCC | ADAPLD_NO_BRANCH));
     const int tasks = succ_possible ? (W * k > k ? W * k : k) : k;
     TreeArgs args{a, ws, (tasks + kRowsPerCta5 - 1) / kRowsPerCta5};
+    int sms = 0, dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        return cudaErrorInvalidDevice;
+    const size_t vsmem = (size_t)a.d * sizeof(float);  // the staged query / reference row
     if (succ_possible) {
         cudaError_t e;
+        if (!a.emb.table && W * k <= kMaxFusedTasks) {  // scan and tree in one kernel
+            auto kern = (int64_t)ws.S4 * a.B <= sms ? succ_scan_kernel<16, true>
+                                                    : succ_scan_kernel<8, true>;
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)vsmem);
+            if (e != cudaSuccess) return e;
+            return launch_dependent(kern, dim3(ws.S4, a.B), dim3(kThreads4), vsmem, s, args);
+        }
         if (a.emb.table && !a.lists_ready) {  // distinct-token lists for the backoff
             DedupeLaunch da{a.tokens, a.ld,  a.lengths, a.B,     a.emb.vocab, nullptr, nullptr,
                             a.status, true, false,     nullptr, false,       k,       nullptr,
@@ -588,11 +650,11 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
             e = launch_dedupe(da, ws, s);
             if (e != cudaSuccess) return e;
         }
-        const size_t qsmem = (size_t)a.d * sizeof(float);
-        e = cudaFuncSetAttribute(succ_scan_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)qsmem);
+        e = cudaFuncSetAttribute(succ_scan_kernel<8, false>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)vsmem);
         if (e != cudaSuccess) return e;
-        e = launch_dependent(succ_scan_kernel, dim3(ws.S4, a.B), dim3(kThreads4), qsmem, s, args);
+        e = launch_dependent(succ_scan_kernel<8, false>, dim3(ws.S4, a.B), dim3(kThreads4), vsmem,
+                             s, args);
         if (e != cudaSuccess) return e;
         if (a.emb.table) {  // successor backoff over token embeddings
             e = launch_dependent(backoff_plan_kernel, dim3(1), dim3(256), 0, s, args);
@@ -617,16 +679,11 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
             if (e != cudaSuccess) return e;
         }
     }
-    const size_t smem = (size_t)a.d * sizeof(float);
-    int sms = 0, dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        return cudaErrorInvalidDevice;
     auto kern = (int64_t)args.rows_ctas * a.B <= sms ? tree_kernel<16> : tree_kernel<8>;
     cudaError_t e =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)vsmem);
     if (e != cudaSuccess) return e;
-    return launch_dependent(kern, dim3(args.rows_ctas, a.B), dim3(kThreads4), smem, s, args);
+    return launch_dependent(kern, dim3(args.rows_ctas, a.B), dim3(kThreads4), vsmem, s, args);
 }
 
 }  // namespace adapld
