@@ -135,6 +135,8 @@ struct SeqView {
     bool valid, cand_ok, lex, sem, branch_on, need_succ;
     bool rr;  // the candidates are (re)ranked by Eq. 6 in this stage
     int nc;
+    int cand_t;      // this thread's candidate cand[b][t] (t < k) and its score
+    float score_t;
 };
 
 // Block-wide (every thread must call, before any early exit).
@@ -142,17 +144,19 @@ __device__ __forceinline__ SeqView view_of(const TreeLaunch &a, int b) {
     SeqView v;
     const int k = a.p.k, W = a.p.branch_width, t = threadIdx.x;
     const uint32_t flags = a.p.flags;
+    // independent loads first (one memory round trip), then the checks
     v.len = a.lengths[b];
+    const int nc_raw = a.n_cand[b];
+    const int hk_raw = a.hit_kind[b];
+    const int c = t < k ? a.cand[(int64_t)b * k + t] : 0;
+    v.score_t = t < k ? a.score[(int64_t)b * k + t] : 0.f;
+    v.cand_t = c;
     v.valid = v.len >= 1 && (int64_t)v.len <= a.ld;
     // candidates come from the caller on the standalone path: check the range
-    const int nc0 = v.valid ? min(a.n_cand[b], k) : 0;
-    bool ok = true;
-    if (t < nc0) {
-        const int c = a.cand[(int64_t)b * k + t];
-        ok = c >= 0 && c <= v.len - 2;
-    }
+    const int nc0 = v.valid ? min(nc_raw, k) : 0;
+    const bool ok = t >= nc0 || (c >= 0 && c <= v.len - 2);
     v.cand_ok = __syncthreads_and(ok) != 0;
-    const int hk = (v.valid && v.cand_ok) ? a.hit_kind[b] : ADAPLD_HIT_NONE;
+    const int hk = (v.valid && v.cand_ok) ? hk_raw : ADAPLD_HIT_NONE;
     v.nc = v.cand_ok ? max(nc0, 0) : 0;
     v.lex = hk == ADAPLD_HIT_LEX && v.nc > 0;
     v.sem = hk == ADAPLD_HIT_SEM && v.nc > 0;
@@ -279,8 +283,8 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
 
     if (t < v.nc) {
-        s_cand[t] = a.cand[(int64_t)b * k + t];
-        s_score[t] = a.score[(int64_t)b * k + t];
+        s_cand[t] = v.cand_t;
+        s_score[t] = v.score_t;
     }
     __syncthreads();
     if (v.rr) {  // the ranking the branches depend on (each slice alike; the
@@ -434,8 +438,8 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
             s_cand[t] = __ldcg(ws.rr_cand + (int64_t)b * kMaxK + t);
             s_score[t] = __ldcg(ws.rr_score + (int64_t)b * kMaxK + t);
         } else {
-            s_cand[t] = a.cand[(int64_t)b * k + t];
-            s_score[t] = a.score[(int64_t)b * k + t];
+            s_cand[t] = v.cand_t;
+            s_score[t] = v.score_t;
         }
     }
     __syncthreads();
