@@ -431,6 +431,9 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
     const uint32_t flags = a.p.flags;
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
+    // the status word is rewritten at the end; its token bit comes from
+    // earlier kernels, so it is read now, off the tail's critical path
+    const int status0 = (a.status && t == 0) ? a.status[b] : 0;
 
     // ---- ranked candidates (the successor scan reranked a strict hit already)
     if (t < v.nc) {
@@ -467,7 +470,8 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
             if (v.need_succ) {
                 const int w = task / k, i = task % k;
                 const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
-                row = i < n ? __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i) : -1;
+                const int pos = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i);
+                row = i < n ? pos : -1;
             } else {
                 row = s_cand[task];
             }
@@ -505,11 +509,12 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
     if (v.branch_on && !v.need_succ) nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc);
     if (v.need_succ) {
         for (int w = warp; w < nb; w += nwarps) {  // Eq. 14: argmax per branch
+            // all three loads at once (lanes past the count are masked after)
             const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
-            const float *sc = score5 + w * k;
-            const int32_t *ps = ws.succ + ((int64_t)b * ws.W + w) * kMaxK;
-            float bs = lane < n ? __ldcg(sc + lane) : -INFINITY;
-            int bj = lane < n ? __ldcg(ps + lane) : -1;
+            const float sl = __ldcg(score5 + w * k + lane);
+            const int pl = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + lane);
+            float bs = lane < n ? sl : -INFINITY;
+            int bj = lane < n ? pl : -1;
 #pragma unroll
             for (int o = 16; o; o >>= 1) {
                 const float os = __shfl_xor_sync(0xffffffffu, bs, o);
@@ -599,7 +604,7 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
             if (s_misc[3]) atomicAdd(a.out.stats + 3, s_misc[3]);
         }
         if (a.status)  // the embedding fallback may have flagged a token id
-            a.status[b] = (a.status[b] & ADAPLD_SEQ_BAD_TOKEN) |
+            a.status[b] = (status0 & ADAPLD_SEQ_BAD_TOKEN) |
                           (v.valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) |
                           (v.cand_ok ? 0 : ADAPLD_SEQ_BAD_CANDIDATE);
     }
