@@ -45,9 +45,10 @@ def parse():
                     help="two-representation mode: token-embedding fallback (vocab x d table)")
     ap.add_argument("--batch", type=int, default=None,
                     help="override B (profiling of small cases; not the headline workload)")
-    ap.add_argument("--verify", action="store_true",
-                    help="also time greedy verification of the step's trees against "
+    ap.add_argument("--no-verify", dest="verify", action="store_false",
+                    help="skip timing greedy verification of the step's trees against "
                          "synthetic target logits [B][nodes][V]")
+    ap.add_argument("--verify", dest="verify", action="store_true", help=argparse.SUPPRESS)
     ap.add_argument("--flags", default="",
                     help="ablation variants (Table 4), comma-separated: no_lex_rerank, "
                          "succ_on_strict, no_semantic, no_branch, no_succ")
