@@ -302,6 +302,39 @@ def test_repeated_calls_reuse_workspace():
     check_all(w, first, P)
 
 
+# ------------------------------------------------ randomised configurations
+@pytest.mark.parametrize("case", range(24))
+def test_random_configurations(case):
+    """Random parameter combinations (n_max, k, W, D, succ_len, tau, ablation
+    flags, ragged lengths, d, the next-token table, the embedding table)
+    against the oracle, so rarely combined paths (the fused tree stage with
+    a table and flags, several slices with few rows, ...) meet it too."""
+    rng = np.random.default_rng(5000 + case)
+    cfg = int(rng.integers(1, 6))
+    B = int(rng.integers(1, 24))
+    L = int(rng.choice([2, 7, 300, 1500, 5000, 9000]))
+    d = int(rng.choice([8, 64, 136, 512, 1024]))
+    V = int(rng.choice([300, 4000, 20000]))
+    lengths = [int(x) for x in rng.integers(1, L + 1, size=B)]
+    lengths[0] = L
+    w = synth.make_workload(cfg, B=B, L=L, d=d, V=V, nohit=float(rng.choice([0.0, 0.5, 1.0])),
+                            seed=case, lengths=lengths)
+    flags = 0
+    for f in (oracle.NO_LEX_RERANK, oracle.SUCC_ON_STRICT, oracle.NO_SEMANTIC, oracle.NO_BRANCH,
+              oracle.NO_SUCC):
+        if rng.random() < 0.2:
+            flags |= f
+    P = P_of(w, tau=float(rng.choice([NEG_INF, 0.0, 0.1, 0.5])), flags=flags,
+             n_max=int(rng.integers(1, 9)), k=int(rng.integers(1, 33)),
+             W=int(rng.integers(0, 9)), D=int(rng.integers(1, 41)),
+             succ_len=int(rng.integers(1, 5)))
+    tk = synth.make_next_topk(w.tokens, w.lengths, V, int(rng.integers(1, 9)),
+                              seed=case) if rng.random() < 0.3 else None
+    E = synth.make_embeddings(w, V, int(rng.choice([8, 64, 200])), case) \
+        if rng.random() < 0.4 else None
+    check_all(w, run_step(w, P, next_topk=tk, emb=E), P, next_topk=tk, emb=E)
+
+
 # ----------------------------------------------------- full-size workloads
 @pytest.mark.parametrize("cfg", [1, 2, 3, 4, 5])
 def test_full_size_config(cfg):
