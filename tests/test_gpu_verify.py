@@ -325,3 +325,38 @@ def test_full_size_config5():
     assert (n_new.cpu().numpy() == o.n_new).all()
     assert (new.cpu().numpy() == o.new_tokens).all()
     assert o.n_accept.max() >= 1
+
+
+@pytest.mark.parametrize("case", range(16))
+def test_random_trees(case):
+    """Random trees (every parent before its child, random fan-out), tie-heavy
+    logits with planted choices, random lengths and capacities, the append
+    with and without hidden states, against the oracle."""
+    rng = np.random.default_rng(700 + case)
+    B = int(rng.integers(1, 12))
+    N = int(rng.integers(1, 80))
+    V = int(rng.choice([8, 64, 1000, 20000]))
+    ld = int(rng.integers(4, 200))
+    d = int(rng.choice([8, 32, 136]))
+    draft = np.full((B, N), -1, np.int32)
+    par = np.full((B, N), -1, np.int32)
+    nn = rng.integers(0, N + 1, size=B).astype(np.int32)
+    for b in range(B):
+        for i in range(1, int(nn[b])):
+            par[b, i] = int(rng.integers(0, i))
+        draft[b, : nn[b]] = rng.integers(0, V, size=int(nn[b]))
+    lg = planted_logits(draft, par, nn, V, rng, p_accept=float(rng.uniform(0.3, 0.95)),
+                        spread=int(rng.integers(1, 4)))
+    mode = case % 3  # 0: verification only, 1: append tokens, 2: append tokens and rows
+    mem, node_reps = None, None
+    if mode:
+        tokens = rng.integers(0, V, size=(B, ld)).astype(np.int32)
+        lengths = rng.integers(0, ld + 1, size=B).astype(np.int32)
+        reps = synth.f32_to_bf16_bits(rng.standard_normal((B, ld, d)).astype(np.float32))
+        query = synth.f32_to_bf16_bits(rng.standard_normal((B, d)).astype(np.float32))
+        mem = (tokens, lengths, reps, query)
+        if mode == 2:
+            node_reps = synth.f32_to_bf16_bits(
+                rng.standard_normal((B, N, d)).astype(np.float32))
+    gpu, o, o_mem = run_both(lg, draft, par, nn, mem, node_reps)
+    assert_same(gpu, o, o_mem)
