@@ -85,19 +85,11 @@ __device__ __forceinline__ int hash_lookup(const unsigned long long *T, int64_t 
 constexpr int kPerThread = kChunk1 / kThreads1;  // positions per thread and chunk (16)
 constexpr int kWordsPerChunk = kChunk1 / 32;        // latest-occurrence bit words (128)
 
-__global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) {
-    const DedupeLaunch &a = args.p;
-    const Workspace &ws = args.ws;
-    __shared__ int s_bad;
-    pdl_wait_then_release();
+// Inserts positions [j0, j1) of sequence b into its hash (all threads of the
+// CTA).  A token id outside the table sets *s_bad.
+__device__ void insert_chunk(const DedupeLaunch &a, const Workspace &ws, int b, int j0, int j1,
+                             int *s_bad) {
     const int t = threadIdx.x, lane = t & 31;
-    const int b = blockIdx.y, c = blockIdx.x;
-    int len;
-    if (!seq_selected(a, b, len)) return;
-    const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);  // positions <= len-2
-    if (j0 >= j1) return;
-    if (t == 0) s_bad = 0;
-    __syncthreads();
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     unsigned long long *T = ws.htab + (int64_t)b * ws.H;
     const uint64_t mask = (uint64_t)(ws.H - 1);
@@ -149,23 +141,106 @@ __global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) 
         }
         lost |= probe == ws.H;
     }
-    if (bad) s_bad = 1;
+    if (bad) *s_bad = 1;
     if (lost) atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
+}
+
+// Marks the positions of [j0, j1) that are the latest occurrence of their
+// token: bit lane of words[e * 8 + warp] for position j0 + e*256 + warp*32 +
+// lane (every word of the chunk is written).  Returns this thread's count.
+__device__ int mark_chunk(const DedupeLaunch &a, const Workspace &ws, int b, int j0, int j1,
+                          uint32_t *words) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const unsigned long long *T = ws.htab + (int64_t)b * ws.H;
+    const uint64_t mask = (uint64_t)(ws.H - 1);
+    int u[kPerThread];
+#pragma unroll
+    for (int e = 0; e < kPerThread; ++e) {
+        const int j = j0 + e * kThreads1 + t;
+        u[e] = j < j1 ? canon(M[j], a.vocab) : 0;
+    }
+    unsigned long long seen[kPerThread];
+#pragma unroll
+    for (int e = 0; e < kPerThread; ++e) {
+        const int j = j0 + e * kThreads1 + t;
+        seen[e] = j < j1 ? __ldcg(T + (hash32((uint32_t)u[e]) & mask)) : 0ull;
+    }
+    int mine = 0;
+#pragma unroll
+    for (int e = 0; e < kPerThread; ++e) {
+        const int j = j0 + e * kThreads1 + t;
+        bool latest = false;
+        if (j < j1) {
+            const unsigned long long key = (unsigned long long)(uint32_t)(u[e] + 1);
+            const int pos = (seen[e] >> 32) == key ? (int)(uint32_t)seen[e]
+                                                   : hash_lookup(T, ws.H, u[e]);
+            latest = pos == j;
+        }
+        const unsigned word = __ballot_sync(0xffffffffu, latest);
+        if (lane == 0) words[e * (kThreads1 / 32) + warp] = word;
+        mine += latest;
+    }
+    return mine;
+}
+
+// Writes the marked positions' tokens of the chunk starting at j0 in
+// position order to out (s_word: the chunk's 128 words in shared memory).
+// One scan over the word counts gives every offset.
+__device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32_t *s_word,
+                              int *s_off, int64_t *s_scan, int32_t *out) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const uint32_t w = t < kWordsPerChunk ? s_word[t] : 0u;
+    int64_t all;
+    const int64_t ex = block_exclusive_scan(__popc(w), &all, s_scan);
+    if (t < kWordsPerChunk) s_off[t] = (int)ex;
+    __syncthreads();
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    // word i = e * 8 + warp holds positions j0 + e * 256 + warp * 32 + lane
+#pragma unroll 4
+    for (int e = 0; e < kPerThread; ++e) {
+        const int i = e * (kThreads1 / 32) + warp;
+        const uint32_t wi = s_word[i];
+        if ((wi >> lane) & 1u) {
+            const int j = j0 + e * kThreads1 + t;
+            out[s_off[i] + __popc(wi & ((1u << lane) - 1u))] = canon(M[j], a.vocab);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kThreads1) rep_insert_kernel(DedupeArgs args) {
+    const DedupeLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int s_bad;
+    pdl_wait_then_release();
+    const int t = threadIdx.x;
+    const int b = blockIdx.y, c = blockIdx.x;
+    int len;
+    if (!seq_selected(a, b, len)) return;
+    const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);  // positions <= len-2
+    if (j0 >= j1) return;
+    if (t == 0) s_bad = 0;
+    __syncthreads();
+    insert_chunk(a, ws, b, j0, j1, &s_bad);
     __syncthreads();
     if (t == 0 && s_bad && a.status) atomicOr(a.status + b, ADAPLD_SEQ_BAD_TOKEN);
 }
 
-// rep_count_kernel: marks the latest occurrences (one bit per position,
-// ws.rep_bits) and counts them per chunk; the last chunk of a sequence turns
-// the counts into offsets, writes rep_len and the anchor; the last sequence
-// builds the plan.
+// rep_count_kernel: marks the latest occurrences (ws.rep_bits) and counts
+// them per chunk; the last chunk of a sequence turns the counts into
+// offsets, writes rep_len and the anchor; the last sequence builds the plan.
+// SINGLE (every history fits one chunk, C1 == 1): the kernel also inserts
+// the chunk first and scatters it after, so the lists take one kernel.
+template <bool SINGLE>
 __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
     const DedupeLaunch &a = args.p;
     const Workspace &ws = args.ws;
-    __shared__ int s_flag;
+    __shared__ int s_flag, s_bad;
     __shared__ int64_t s_scan[32];
+    __shared__ uint32_t s_word[SINGLE ? kWordsPerChunk : 1];
+    __shared__ int s_off[SINGLE ? kWordsPerChunk : 1];
     pdl_wait_then_release();
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int t = threadIdx.x;
     const int b = blockIdx.y, c = blockIdx.x;
     int len;
     const bool sel = seq_selected(a, b, len);
@@ -177,59 +252,47 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
     } else {
         const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);
         const int32_t *M = a.tokens + (int64_t)b * a.ld;
-        const unsigned long long *T = ws.htab + (int64_t)b * ws.H;
-        const uint64_t mask = (uint64_t)(ws.H - 1);
-        uint32_t *bits = ws.rep_bits + ((int64_t)b * ws.C1 + c) * kWordsPerChunk;
-        int u[kPerThread];
-#pragma unroll
-        for (int e = 0; e < kPerThread; ++e) {
-            const int j = j0 + e * kThreads1 + t;
-            u[e] = j < j1 ? canon(M[j], a.vocab) : 0;
+        if (SINGLE) {
+            if (t == 0) s_bad = 0;
+            __syncthreads();
+            insert_chunk(a, ws, b, j0, j1, &s_bad);
+            __syncthreads();  // this CTA's inserts are the whole sequence's
+            if (t == 0 && s_bad && a.status) atomicOr(a.status + b, ADAPLD_SEQ_BAD_TOKEN);
         }
-        unsigned long long seen[kPerThread];
-#pragma unroll
-        for (int e = 0; e < kPerThread; ++e) {
-            const int j = j0 + e * kThreads1 + t;
-            seen[e] = j < j1 ? __ldcg(T + (hash32((uint32_t)u[e]) & mask)) : 0ull;
-        }
-        int mine = 0;
-#pragma unroll
-        for (int e = 0; e < kPerThread; ++e) {
-            const int j = j0 + e * kThreads1 + t;
-            bool latest = false;
-            if (j < j1) {
-                const unsigned long long key = (unsigned long long)(uint32_t)(u[e] + 1);
-                const int pos = (seen[e] >> 32) == key ? (int)(uint32_t)seen[e]
-                                                       : hash_lookup(T, ws.H, u[e]);
-                latest = pos == j;
-            }
-            const unsigned word = __ballot_sync(0xffffffffu, latest);
-            if (lane == 0) bits[e * (kThreads1 / 32) + warp] = word;
-            mine += latest;
-        }
+        uint32_t *words =
+            SINGLE ? s_word : ws.rep_bits + ((int64_t)b * ws.C1 + c) * kWordsPerChunk;
+        const int mine = mark_chunk(a, ws, b, j0, j1, words);
         int64_t total;  // the block's sum
         (void)block_exclusive_scan(mine, &total, s_scan);
-        if (t == 0) ws.rep_cnt[(int64_t)b * ws.C1 + c] = (int)total;
-        __threadfence();
-        __syncthreads();
-        if (t == 0) s_flag = atomicAdd(ws.rticket + b, 1) == (int)gridDim.x - 1;
-        __syncthreads();
-        if (!s_flag) return;
-        __threadfence();
-        // last chunk of b: chunk counts -> offsets, n = distinct tokens
-        int64_t carry = 0;
-        for (int base = 0; base < (int)gridDim.x; base += kThreads1) {
-            const int cc = base + t;
-            const int64_t v =
-                cc < (int)gridDim.x ? __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + cc) : 0;
-            int64_t all;
-            const int64_t ex = block_exclusive_scan(v, &all, s_scan);
-            if (cc < (int)gridDim.x) ws.rep_cnt[(int64_t)b * ws.C1 + cc] = (int)(carry + ex);
-            carry += all;
-        }
-        if (t == 0) {
-            ws.rep_len[b] = (int)carry + 1;
-            ws.rep_tok[(int64_t)b * a.ld + carry] = M[len - 1];  // the anchor (as stored)
+        if (SINGLE) {  // one chunk: offset 0, no ticket
+            scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld);
+            if (t == 0) {
+                ws.rep_len[b] = (int)total + 1;
+                ws.rep_tok[(int64_t)b * a.ld + total] = M[len - 1];  // the anchor (as stored)
+            }
+        } else {
+            if (t == 0) ws.rep_cnt[(int64_t)b * ws.C1 + c] = (int)total;
+            __threadfence();
+            __syncthreads();
+            if (t == 0) s_flag = atomicAdd(ws.rticket + b, 1) == (int)gridDim.x - 1;
+            __syncthreads();
+            if (!s_flag) return;
+            __threadfence();
+            // last chunk of b: chunk counts -> offsets, n = distinct tokens
+            int64_t carry = 0;
+            for (int base = 0; base < (int)gridDim.x; base += kThreads1) {
+                const int cc = base + t;
+                const int64_t v =
+                    cc < (int)gridDim.x ? __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + cc) : 0;
+                int64_t all;
+                const int64_t ex = block_exclusive_scan(v, &all, s_scan);
+                if (cc < (int)gridDim.x) ws.rep_cnt[(int64_t)b * ws.C1 + cc] = (int)(carry + ex);
+                carry += all;
+            }
+            if (t == 0) {
+                ws.rep_len[b] = (int)carry + 1;
+                ws.rep_tok[(int64_t)b * a.ld + carry] = M[len - 1];  // the anchor (as stored)
+            }
         }
         seq_done = true;
     }
@@ -246,8 +309,7 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
 }
 
 // rep_scatter_kernel: the chunk's latest occurrences, in position order, at
-// the chunk's offset.  Word i of the chunk's bits covers positions
-// j0 + 32 i .. +32; one scan over the 128 word counts gives every offset.
+// the chunk's offset.
 __global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args) {
     const DedupeLaunch &a = args.p;
     const Workspace &ws = args.ws;
@@ -255,33 +317,17 @@ __global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args)
     __shared__ int s_off[kWordsPerChunk];
     __shared__ uint32_t s_word[kWordsPerChunk];
     pdl_wait_then_release();
-    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int t = threadIdx.x;
     const int b = blockIdx.y, c = blockIdx.x;
     int len;
     if (!seq_selected(a, b, len)) return;
     const int j0 = c * kChunk1, j1 = min(j0 + kChunk1, len - 1);
     if (j0 >= j1) return;
     const uint32_t *bits = ws.rep_bits + ((int64_t)b * ws.C1 + c) * kWordsPerChunk;
-    const uint32_t w = t < kWordsPerChunk ? __ldcg(bits + t) : 0u;
-    int64_t all;
-    const int64_t ex = block_exclusive_scan(__popc(w), &all, s_scan);
-    if (t < kWordsPerChunk) {
-        s_off[t] = (int)ex;
-        s_word[t] = w;
-    }
+    if (t < kWordsPerChunk) s_word[t] = __ldcg(bits + t);
     __syncthreads();
-    const int32_t *M = a.tokens + (int64_t)b * a.ld;
-    int32_t *out = ws.rep_tok + (int64_t)b * a.ld + __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c);
-    // word i = e * 8 + warp holds positions j0 + e * 256 + warp * 32 + lane
-#pragma unroll 4
-    for (int e = 0; e < kPerThread; ++e) {
-        const int i = e * (kThreads1 / 32) + warp;
-        const uint32_t wi = s_word[i];
-        if ((wi >> lane) & 1u) {
-            const int j = j0 + e * kThreads1 + t;
-            out[s_off[i] + __popc(wi & ((1u << lane) - 1u))] = canon(M[j], a.vocab);
-        }
-    }
+    scatter_chunk(a, b, j0, s_word, s_off, s_scan,
+                  ws.rep_tok + (int64_t)b * a.ld + __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c));
 }
 
 // ---------------------------------------------------------------- expansion
@@ -411,10 +457,14 @@ __global__ void __launch_bounds__(kExpandThreads) expand_kernel(ExpandArgs args)
 cudaError_t launch_dedupe(const DedupeLaunch &a, const Workspace &ws, cudaStream_t s) {
     DedupeArgs args{a, ws};
     const dim3 grid(ws.C1, a.B);
+    if (ws.C1 == 1)  // every history is one chunk: one kernel builds the lists
+        return a.pdl ? launch_dependent(rep_count_kernel<true>, grid, dim3(kThreads1), 0, s, args)
+                     : (rep_count_kernel<true><<<grid, kThreads1, 0, s>>>(args),
+                        cudaGetLastError());
     cudaError_t e = a.pdl ? launch_dependent(rep_insert_kernel, grid, dim3(kThreads1), 0, s, args)
                           : (rep_insert_kernel<<<grid, kThreads1, 0, s>>>(args), cudaGetLastError());
     if (e != cudaSuccess) return e;
-    e = launch_dependent(rep_count_kernel, grid, dim3(kThreads1), 0, s, args);
+    e = launch_dependent(rep_count_kernel<false>, grid, dim3(kThreads1), 0, s, args);
     if (e != cudaSuccess) return e;
     return launch_dependent(rep_scatter_kernel, grid, dim3(kThreads1), 0, s, args);
 }
