@@ -28,6 +28,7 @@ __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
     __shared__ int tok[kChunk1 + 8];
     __shared__ int suf[8];
     __shared__ int wval[kThreads1 / 32];
+    __shared__ int wcnt[(kChunk1 / kThreads1) * (kThreads1 / 32)];  // hits per (block, warp)
     __shared__ int list[kMaxK];
     __shared__ int flag;
 
@@ -71,28 +72,37 @@ __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
         for (int w = 0; w < kThreads1 / 32; ++w) cmax = max(cmax, wval[w]);
         __syncthreads();
         if (cmax > 0) {
-            // most recent first: position blocks from the top, within a block
-            // higher warps and then higher lanes first
+            // most recent first: position blocks e from the top, within a
+            // block higher warps and then higher lanes first.  Every
+            // (block, warp) count goes to shared memory at once, so one
+            // barrier ranks all positions.
+            constexpr int E = kChunk1 / kThreads1, NW = kThreads1 / 32;
+            unsigned bal[E];
 #pragma unroll
-            for (int e = kChunk1 / kThreads1 - 1; e >= 0; --e) {
+            for (int e = 0; e < E; ++e) {
                 const int p = j0 + e * kThreads1 + t;
-                const bool hit = p < j1 && m[e] == cmax;
-                const unsigned bal = __ballot_sync(0xffffffffu, hit);
-                if (lane == 0) wval[warp] = __popc(bal);
-                __syncthreads();
-                int above = 0, all = 0;
-                for (int w = 0; w < kThreads1 / 32; ++w) {
-                    if (w > warp) above += wval[w];
-                    all += wval[w];
-                }
-                const unsigned higher = lane == 31 ? 0u : (bal & (0xffffffffu << (lane + 1)));
-                const int rank = cnt + above + __popc(higher);
-                if (hit && rank < a.k) list[rank] = p;
-                cnt += all;
-                __syncthreads();
-                if (cnt >= a.k) break;
+                bal[e] = __ballot_sync(0xffffffffu, p < j1 && m[e] == cmax);
+                if (lane == 0) wcnt[e * NW + warp] = __popc(bal[e]);
             }
-            cnt = min(cnt, a.k);
+            __syncthreads();
+            // ranks: positions of higher blocks, then of higher warps and
+            // lanes in this block, come first
+            int before = 0;  // hits in blocks above e (filled from the top)
+#pragma unroll
+            for (int e = E - 1; e >= 0; --e) {
+                int above = 0, all = 0;
+#pragma unroll
+                for (int w = 0; w < NW; ++w) {
+                    const int cw = wcnt[e * NW + w];
+                    above += w > warp ? cw : 0;
+                    all += cw;
+                }
+                const unsigned higher = lane == 31 ? 0u : (bal[e] & (0xffffffffu << (lane + 1)));
+                const int rank = before + above + __popc(higher);
+                if (((bal[e] >> lane) & 1u) && rank < a.k) list[rank] = j0 + e * kThreads1 + t;
+                before += all;
+            }
+            cnt = min(before, a.k);
         }
     }
 
