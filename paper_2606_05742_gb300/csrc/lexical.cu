@@ -166,12 +166,17 @@ __global__ void __launch_bounds__(kThreads1) lexical_kernel(LexArgs args) {
     if (!a.build_plan) return;
 
     // ---- last sequence overall: semantic plan ---------------------------------
-    __threadfence();
-    __syncthreads();
-    if (t == 0) flag = atomicAdd(ws.global_ticket, 1) == a.B - 1;
-    __syncthreads();
-    if (!flag) return;
-    __threadfence();
+    // (a grid of one CTA is last by construction: no ticket)
+    if (gridDim.x * gridDim.y > 1) {
+        __threadfence();
+        __syncthreads();
+        if (t == 0) flag = atomicAdd(ws.global_ticket, 1) == a.B - 1;
+        __syncthreads();
+        if (!flag) return;
+        __threadfence();
+    } else {
+        __syncthreads();  // this CTA's outcome writes are visible to the block
+    }
     build_plan_cta(a.lengths, a.ld, a.B, a.hit_kind, nullptr, ws.plan, false, a.k, nullptr,
                    nullptr, nullptr);
 }
