@@ -490,8 +490,10 @@ def run_native(args):
     if not args.no_e2e and emb is None:
         tok_h = w.tokens.cpu().pin_memory()
         len_h = w.lengths.cpu().pin_memory()
-        reps_h = torch.empty(w.reps.shape, dtype=w.reps.dtype, pin_memory=True)
-        reps_h.copy_(w.reps)
+        # the host inputs are written by the CPU, as a host producer would
+        # write them (a pinned buffer last written by the GPU read back over
+        # the host link at a fraction of the rate in probes)
+        reps_h = w.reps.cpu().pin_memory()
         q_h = w.query.cpu().pin_memory()
         dev_in = (torch.empty_like(w.tokens), torch.empty_like(w.lengths),
                   torch.empty_like(w.reps), torch.empty_like(w.query))
