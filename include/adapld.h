@@ -322,6 +322,23 @@ int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const
                 adapld_stream_t stream);
 
 /*
+ * adapld_step() from HOST inputs to HOST outputs, all on `stream`: copies
+ * tokens_h, lengths_h, reps_h and query_h (host memory, page-locked for the
+ * copies to be asynchronous) into the caller's device buffers tokens_d,
+ * lengths_d, reps_d and query_d (same layouts), runs the step into out_d
+ * (device), then copies every non-NULL array of out_h (host; the same
+ * shapes as out_d) from out_d.  The host outputs are valid once the stream
+ * has been synchronised.  Nothing is allocated; argument errors as for
+ * adapld_step() (ADAPLD_ERR_NULL also for a missing host or device input).
+ */
+int adapld_step_from_host(const int32_t *tokens_h, int64_t ld, const int32_t *lengths_h,
+                          const uint16_t *reps_h, int32_t d, const uint16_t *query_h, int32_t B,
+                          const adapld_params *p, int32_t *tokens_d, int32_t *lengths_d,
+                          uint16_t *reps_d, uint16_t *query_d, const adapld_step_out *out_d,
+                          const adapld_step_out *out_h, void *ws, size_t ws_bytes,
+                          adapld_stream_t stream);
+
+/*
  * adapld_step() with two options.  emb (nullable) selects the
  * two-representation mode: the fallback scores token embeddings (Eq. 4 as
  * printed), semantic candidates are reranked by the hidden states (Eq. 6),

@@ -279,6 +279,53 @@ int adapld_step(const int32_t *tokens, int64_t ld, const int32_t *lengths, const
                           ws_bytes, nullptr, nullptr, stream);
 }
 
+int adapld_step_from_host(const int32_t *tokens_h, int64_t ld, const int32_t *lengths_h,
+                          const uint16_t *reps_h, int32_t d, const uint16_t *query_h, int32_t B,
+                          const adapld_params *p, int32_t *tokens_d, int32_t *lengths_d,
+                          uint16_t *reps_d, uint16_t *query_d, const adapld_step_out *out_d,
+                          const adapld_step_out *out_h, void *ws, size_t ws_bytes,
+                          adapld_stream_t stream) {
+    if (!tokens_h || !lengths_h || !reps_h || !query_h || !tokens_d || !lengths_d || !reps_d ||
+        !query_d || !out_d || !out_h)
+        return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_params(p));
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_dim(d));
+    cudaStream_t s = (cudaStream_t)stream;
+    auto h2d = [&](void *dst, const void *src, size_t bytes) {
+        return cuda_status(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, s));
+    };
+    const size_t rows = (size_t)B * (size_t)ld;
+    ADAPLD_TRY(h2d(tokens_d, tokens_h, sizeof(int32_t) * rows));
+    ADAPLD_TRY(h2d(lengths_d, lengths_h, sizeof(int32_t) * (size_t)B));
+    ADAPLD_TRY(h2d(reps_d, reps_h, sizeof(uint16_t) * rows * (size_t)d));
+    ADAPLD_TRY(h2d(query_d, query_h, sizeof(uint16_t) * (size_t)B * (size_t)d));
+    ADAPLD_TRY(adapld_step(tokens_d, ld, lengths_d, reps_d, d, query_d, nullptr, 0, B, p, out_d,
+                           ws, ws_bytes, stream));
+    // the outputs back, every array the caller asked for
+    const size_t N = (size_t)adapld_tree_nodes(p), k = (size_t)p->k, b = (size_t)B;
+    struct Copy {
+        void *dst;
+        const void *src;
+        size_t bytes;
+    };
+    const adapld_tree_out &th = out_h->tree, &td = out_d->tree;
+    const Copy copies[] = {
+        {out_h->hit_kind, out_d->hit_kind, 4 * b},     {out_h->match_n, out_d->match_n, 4 * b},
+        {out_h->cand, out_d->cand, 4 * b * k},         {out_h->score, out_d->score, 4 * b * k},
+        {out_h->n_cand, out_d->n_cand, 4 * b},         {out_h->status, out_d->status, 4 * b},
+        {th.anchor, td.anchor, 4 * b},                 {th.draft_tokens, td.draft_tokens, 4 * b * N},
+        {th.parents, td.parents, 4 * b * N},           {th.positions, td.positions, 4 * b * N},
+        {th.mask, td.mask, b * N * N},                 {th.n_nodes, td.n_nodes, 4 * b},
+        {th.stats, td.stats, 4 * 4},
+    };
+    for (const Copy &c : copies) {
+        if (!c.dst || !c.src) continue;
+        ADAPLD_TRY(cuda_status(cudaMemcpyAsync(c.dst, c.src, c.bytes, cudaMemcpyDeviceToHost, s)));
+    }
+    return ADAPLD_OK;
+}
+
 int adapld_accept_greedy(const uint16_t *logits, int32_t V, const int32_t *draft_tokens,
                          const int32_t *parents, const int32_t *n_nodes, int32_t B, int32_t N,
                          int32_t *n_accept, int32_t *new_tokens, int32_t *n_new,

@@ -36,6 +36,7 @@ EXPORTED = [
     "adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
     "adapld_step", "adapld_step_ex", "adapld_read_device_status",
     "adapld_semantic_topk_static", "adapld_embedding_topk", "adapld_accept_greedy",
+    "adapld_step_from_host",
 ]
 STATIC_MAX_B = 1024
 ERR_STATIC_LIMIT = -15
@@ -123,10 +124,12 @@ def load() -> ctypes.CDLL:
                                                     P, P]
         lib.adapld_accept_greedy.argtypes = [P, i32, P, P, P, i32, i32, P, P, P, P, i64, P, P,
                                              P, i32, P, P, P, sz, P]
+        lib.adapld_step_from_host.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, P, P, P,
+                                              sz, P]
         for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
                   "adapld_step", "adapld_step_ex", "adapld_read_device_status",
                   "adapld_semantic_topk_static", "adapld_embedding_topk",
-                  "adapld_accept_greedy"):
+                  "adapld_accept_greedy", "adapld_step_from_host"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -241,17 +244,19 @@ class Outputs:
     stats: object
 
     @staticmethod
-    def allocate(B: int, p: Params, device="cuda") -> "Outputs":
+    def allocate(B: int, p: Params, device="cuda", pin_memory=False) -> "Outputs":
+        """Buffers on `device` ("cpu" with pin_memory=True: page-locked host
+        buffers for adapld_step_from_host)."""
         import torch
         N = 1 + p.draft_len + p.branch_width * (1 + p.succ_len)
-        i32 = dict(dtype=torch.int32, device=device)
+        i32 = dict(dtype=torch.int32, device=device, pin_memory=pin_memory)
         return Outputs(
             torch.empty(B, **i32), torch.empty(B, **i32), torch.empty((B, p.k), **i32),
-            torch.empty((B, p.k), dtype=torch.float32, device=device), torch.empty(B, **i32),
-            torch.empty(B, **i32), torch.empty(B, **i32), torch.empty((B, N), **i32),
-            torch.empty((B, N), **i32), torch.empty((B, N), **i32),
-            torch.empty((B, N, N), dtype=torch.uint8, device=device), torch.empty(B, **i32),
-            torch.empty(4, **i32))
+            torch.empty((B, p.k), dtype=torch.float32, device=device, pin_memory=pin_memory),
+            torch.empty(B, **i32), torch.empty(B, **i32), torch.empty(B, **i32),
+            torch.empty((B, N), **i32), torch.empty((B, N), **i32), torch.empty((B, N), **i32),
+            torch.empty((B, N, N), dtype=torch.uint8, device=device, pin_memory=pin_memory),
+            torch.empty(B, **i32), torch.empty(4, **i32))
 
     def c_struct(self) -> StepOut:
         return StepOut(_ptr(self.hit_kind), _ptr(self.match_n), _ptr(self.cand),
@@ -353,6 +358,27 @@ class Engine:
         step(tokens, lengths, reps, query, self.p, self.out, self.ws, next_topk, events, stream,
              emb)
         return self.out
+
+    def bind_from_host(self, tokens_h, lengths_h, reps_h, query_h, dev_inputs, host_out,
+                       stream=None):
+        """The end-to-end step through adapld_step_from_host, arguments
+        marshalled once: each call copies the host inputs (page-locked) into
+        `dev_inputs` (tokens, lengths, reps, query on the device), runs the
+        step into self.out and copies every output into `host_out` (an
+        Outputs of page-locked host tensors).  Returns (call, h2d bytes, d2h
+        bytes)."""
+        B, ld, d = reps_h.shape
+        tok_d, len_d, reps_d, q_d = dev_inputs
+        so_d = self.out.c_struct()
+        so_h = host_out.c_struct()
+        lib = load()
+        args = (_ptr(tokens_h), ld, _ptr(lengths_h), _ptr(reps_h), d, _ptr(query_h), B,
+                ctypes.byref(self.p), _ptr(tok_d), _ptr(len_d), _ptr(reps_d), _ptr(q_d),
+                ctypes.byref(so_d), ctypes.byref(so_h), _ptr(self.ws),
+                self.ws.numel() * self.ws.element_size(), _stream(stream))
+        h2d = sum(t.numel() * t.element_size() for t in (tokens_h, lengths_h, reps_h, query_h))
+        return (BoundCall(lib.adapld_step_from_host, args, [so_d, so_h, self.p],
+                          "adapld_step_from_host"), h2d, host_out.nbytes())
 
     def bind(self, tokens, lengths, reps, query, next_topk=None, stream=None, emb=None):
         """The step on fixed buffers with its arguments marshalled once: the

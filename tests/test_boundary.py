@@ -191,6 +191,24 @@ def test_accept_argument_errors(lib, kw, code):
     assert _accept(lib, **kw) == code
 
 
+def test_step_from_host_argument_errors(lib):
+    p = native.make_params(3, 8, 2, 8)
+    so = native.StepOut(FAKE, FAKE, FAKE, FAKE, FAKE, None,
+                        native.TreeOut(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None))
+    args = [FAKE, 64, FAKE, FAKE, 16, FAKE, 2, ctypes.byref(p), FAKE, FAKE, FAKE, FAKE,
+            ctypes.byref(so), ctypes.byref(so), FAKE, 1 << 30, None]
+    for i in (0, 2, 3, 5, 8, 9, 10, 11, 12, 13):     # each required pointer
+        bad = list(args)
+        bad[i] = None
+        assert lib.adapld_step_from_host(*bad) == -1, i
+    bad = list(args)
+    bad[6] = 0
+    assert lib.adapld_step_from_host(*bad) == -2
+    bad = list(args)
+    bad[4] = 12
+    assert lib.adapld_step_from_host(*bad) == -7
+
+
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(native, "LIB_PATH", str(tmp_path / "missing.so"))
     monkeypatch.setattr(native, "_lib", None)

@@ -504,6 +504,40 @@ def test_step_replays_from_a_cuda_graph(mode):
     assert torch.equal(n_acc, want_acc)
 
 
+def test_step_from_host_matches_device_path():
+    """adapld_step_from_host: host inputs in, host outputs out, in one call,
+    equal to the device-resident step; twice on the same buffers."""
+    w = synth.make_workload(2, B=7, L=900, d=64, nohit=0.5, seed=93)
+    P = P_of(w)
+    ref = run_step(w, P)
+    p = params(P)
+    eng = native.Engine(w.B, w.ld, w.d, p)
+    tok_h = torch.from_numpy(np.ascontiguousarray(w.tokens)).pin_memory()
+    len_h = torch.from_numpy(np.ascontiguousarray(w.lengths)).pin_memory()
+    reps_h = torch.from_numpy(np.ascontiguousarray(w.reps).view(np.int16)).view(
+        torch.bfloat16).pin_memory()
+    q_h = torch.from_numpy(np.ascontiguousarray(w.query).view(np.int16)).view(
+        torch.bfloat16).pin_memory()
+    dev = (torch.empty(tok_h.shape, dtype=torch.int32, device="cuda"),
+           torch.empty(len_h.shape, dtype=torch.int32, device="cuda"),
+           torch.empty(reps_h.shape, dtype=torch.bfloat16, device="cuda"),
+           torch.empty(q_h.shape, dtype=torch.bfloat16, device="cuda"))
+    host_out = native.Outputs.allocate(w.B, p, device="cpu", pin_memory=True)
+    call, h2d, d2h = eng.bind_from_host(tok_h, len_h, reps_h, q_h, dev, host_out)
+    assert h2d == w.tokens.nbytes + w.lengths.nbytes + w.reps.nbytes + w.query.nbytes
+    assert d2h == host_out.nbytes()
+    for _ in range(2):
+        for t in host_out.tensors():
+            t.zero_()
+        call()
+        torch.cuda.synchronize()
+        got = {n: t.numpy() for n, t in zip(
+            ["hit_kind", "match_n", "cand", "score", "n_cand", "status", "anchor", "draft_tokens",
+             "parents", "positions", "mask", "n_nodes", "stats"], host_out.tensors())}
+        for key in ref:
+            assert np.array_equal(ref[key], got[key], equal_nan=True), key
+
+
 def test_end_to_end_from_host_matches_device_path():
     """The public end-to-end call (pinned host inputs, copies on side streams,
     outputs copied back) returns what the device-resident call returns."""
