@@ -5,9 +5,10 @@
 // 4096 candidate positions (plus an n_max-1 token halo) in shared memory,
 // computes for each position j the length m(j) of the backward match
 // M[j-i] == M[len-1-i], i < m(j) <= min(n_max, len-1), reduces the chunk
-// maximum and collects the k most recent positions reaching it with warp
-// ballots.  The last CTA of a sequence (atomic ticket) merges the chunk
-// results: n* = max m, candidates = the k most recent positions with
+// maximum and ranks the positions reaching it, most recent first, with warp
+// ballots and one barrier.  A history of one chunk writes its result
+// directly; otherwise the last CTA of a sequence (atomic ticket) merges the
+// chunk results: n* = max m, candidates = the k most recent positions with
 // m(j) = n*.  On the step path the last sequence to finish also writes the
 // prefix sums of the semantic fallback's rows (the plan), so the semantic
 // kernel can balance rows over the whole GPU without a host round trip.

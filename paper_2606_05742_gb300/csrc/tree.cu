@@ -14,14 +14,15 @@
 // (lexical hits are reranked here in that mode), then scans its slice of
 // 8192 positions for the branch tokens, a warp per branch, backwards with
 // ballots, keeping the k most recent occurrences.  The last slice CTA
-// (atomic ticket) merges the slices, most recent first, into the successor
-// candidate lists.
+// (atomic ticket; none with one slice) merges the slices, most recent first,
+// into the successor candidate lists.
 //
 // tree_kernel, grid (R5, B), 512 threads.  Every sequence has a list of rows
 // to score: the lexical candidates against the query (Eq. 6), or every
 // successor candidate against R[j*+1] (Eq. 13).  CTA r scores rows
-// [16r, 16r+16), one warp per row, both operands streamed from global memory
-// with eight 16-byte loads per lane in flight.  The last CTA of the sequence
+// [16r, 16r+16), one warp per row against the reference vector staged once
+// per CTA in shared memory, with 16 (or 8) 16-byte row loads per lane in
+// flight.  The last CTA of the sequence
 // then ranks the lexical candidates (Eq. 7), picks each branch's successor
 // (Eq. 14), lays out the tree (root, main chain, branch paths with their
 // successors) and writes tokens, parents, position ids and the ancestor mask.
