@@ -151,7 +151,13 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
         s_par[i] = a.parents[(int64_t)b * N + i];
         const unsigned long long *kp = ws.vpart + ((int64_t)b * N + i) * S;
         unsigned long long key = 0ull;
-        for (int j = 0; j < S; ++j) key = max(key, __ldcg(kp + j));
+        for (int j0 = 0; j0 < S; j0 += 8) {  // eight partial keys in flight at a time
+            unsigned long long kk[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) kk[j] = j0 + j < S ? __ldcg(kp + j0 + j) : 0ull;
+#pragma unroll
+            for (int j = 0; j < 8; ++j) key = max(key, kk[j]);
+        }
         s_tgt[i] = key_index(key);
     }
     __syncthreads();
