@@ -430,6 +430,43 @@ def test_semantic_wait_timeout_is_reported_and_recoverable(monkeypatch):
     check_all(w, g, P)
 
 
+def test_concurrent_calls_from_threads():
+    """Two host threads, each with its own stream, workspace and outputs,
+    issue steps concurrently (the library keeps no shared state): each gets
+    the single-threaded result."""
+    import threading
+    V = 4000
+    ws_ = [synth.make_workload(2, B=5, L=2000, d=64, V=V, nohit=0.6, seed=94 + i)
+           for i in range(2)]
+    refs = [run_step(w, P_of(w)) for w in ws_]
+    results, errors = [None, None], []
+
+    def worker(i):
+        try:
+            w = ws_[i]
+            s = torch.cuda.Stream()
+            with torch.cuda.stream(s):
+                tok, ln, reps, q = to_dev(w)
+                eng = native.Engine(w.B, w.ld, w.d, params(P_of(w)))
+                call = eng.bind(tok, ln, reps, q, stream=s)
+                for _ in range(20):
+                    call()
+                s.synchronize()
+                results[i] = eng.out.to_host()
+        except Exception as e:  # reported below
+            errors.append(e)
+
+    th = [threading.Thread(target=worker, args=(i,)) for i in range(2)]
+    for t in th:
+        t.start()
+    for t in th:
+        t.join()
+    assert not errors, errors
+    for ref, got in zip(refs, results):
+        for key in ref:
+            assert np.array_equal(ref[key], got[key], equal_nan=True), key
+
+
 @pytest.mark.parametrize("mode", ["plain", "embeddings"])
 def test_bound_step_matches_run(mode):
     """Engine.bind marshals the arguments once; its calls give the step's
