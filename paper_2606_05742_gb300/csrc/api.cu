@@ -349,7 +349,6 @@ int adapld_accept_greedy(const uint16_t *logits, int32_t V, const int32_t *draft
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, 1, 1));
     const Workspace w = layout_workspace(ws, B, 1, 1);
     cudaStream_t s = (cudaStream_t)stream;
-    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
     VerifyLaunch a{logits, V, draft_tokens, parents, n_nodes, B, N, n_accept, new_tokens, n_new,
                    tokens, ld, lengths, node_reps, reps, d, query, status};
     return cuda_status(launch_verify(a, w, s));

@@ -9,15 +9,16 @@
 // verify_kernel, grid (S splits, N nodes, B), 256 threads.  CTA (s, i, b)
 // reads split s of node i's row in 32 KB groups (8 independent 16-byte
 // loads per thread, all issued before any is used; groups s, s + S, ...)
-// and keeps the first index of the maximum, stored as a 64-bit key that
-// orders by value, then by the smaller index (S <= 1024 / N keeps the
-// partial keys within the workspace).  CTAs of nodes >= n_nodes[b] exit at
-// once.  The last CTA of a sequence (atomic ticket over n_nodes[b] x S CTAs)
-// takes the largest key per node, loads the tree into shared memory,
-// walks from the root with warp ballots (the child whose token equals the
-// choice at the current node), writes the new tokens (accepted draft tokens,
-// then the choice after the last accepted node) and appends them, with the
-// hidden states of the root and the accepted nodes, to the memory.
+// and stores the first index of the maximum as a 64-bit key that orders by
+// value, then by the smaller index (S <= 1024 / N keeps the partial keys
+// within the workspace).  CTAs of nodes >= n_nodes[b] exit at once.  No
+// counters and no fences: walk_kernel, one CTA per sequence and launched as
+// a programmatic dependent (so every key is visible), takes the largest key
+// per node, loads the tree into shared memory, walks from the root with warp
+// ballots (the child whose token equals the choice at the current node),
+// writes the new tokens (accepted draft tokens, then the choice after the
+// last accepted node) and appends them, with the hidden states of the root
+// and the accepted nodes, to the memory.
 #include <climits>
 
 #include "common.cuh"
@@ -77,27 +78,14 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
     const Workspace &ws = args.ws;
     __shared__ float s_v[kThreadsV / 32];
     __shared__ int s_i[kThreadsV / 32];
-    __shared__ int s_tok[kMaxNodes], s_par[kMaxNodes], s_tgt[kMaxNodes];
-    __shared__ int s_path[kMaxNodes];
-    __shared__ int s_flag, s_nacc;
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int split = blockIdx.x, node = blockIdx.y, b = blockIdx.z;
     const int N = a.N, V = a.V, S = args.S;
+    // the walk kernel may be scheduled now; it waits for this grid to finish
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int n = min(a.n_nodes[b], N);
-    int32_t *new_b = a.new_tokens + (int64_t)b * N;
-    if (n <= 0) {  // an empty tree: nothing to verify or append
-        if (node == 0 && split == 0) {
-            for (int i = t; i < N; i += kThreadsV) new_b[i] = -1;
-            if (t == 0) {
-                a.n_accept[b] = 0;
-                a.n_new[b] = 0;
-                if (a.status) a.status[b] = 0;
-            }
-        }
-        return;
-    }
-    if (node >= n) return;
+    if (node >= n) return;  // (also every CTA of an empty tree)
 
     // ---- this split of the target's row after the node: first index of the maximum
     const uint16_t *row = a.logits + ((int64_t)b * N + node) * V;
@@ -138,12 +126,33 @@ __global__ void __launch_bounds__(kThreadsV) verify_kernel(VerifyArgs args) {
                 bi = s_i[k];
             }
         ws.vpart[((int64_t)b * N + node) * S + split] = bi < V ? choice_key(bv, bi) : 0ull;
-        __threadfence();
-        s_flag = atomicAdd(ws.vticket + b, 1) == n * S - 1;
     }
-    __syncthreads();
-    if (!s_flag) return;
-    __threadfence();
+}
+
+// walk_kernel, one CTA per sequence, launched as a programmatic dependent of
+// verify_kernel (so every partial key is visible): the largest key per node,
+// the walk, the new tokens and the append.
+__global__ void __launch_bounds__(kThreadsV) walk_kernel(VerifyArgs args) {
+    const VerifyLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ int s_tok[kMaxNodes], s_par[kMaxNodes], s_tgt[kMaxNodes];
+    __shared__ int s_path[kMaxNodes];
+    __shared__ int s_nacc;
+    pdl_wait_then_release();
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int b = blockIdx.x;
+    const int N = a.N, S = args.S;
+    const int n = min(a.n_nodes[b], N);
+    int32_t *new_b = a.new_tokens + (int64_t)b * N;
+    if (n <= 0) {  // an empty tree: nothing to verify or append
+        for (int i = t; i < N; i += kThreadsV) new_b[i] = -1;
+        if (t == 0) {
+            a.n_accept[b] = 0;
+            a.n_new[b] = 0;
+            if (a.status) a.status[b] = 0;
+        }
+        return;
+    }
 
     // ---- the last CTA of sequence b: walk the tree
     for (int i = t; i < n; i += kThreadsV) {
@@ -231,7 +240,9 @@ cudaError_t launch_verify(const VerifyLaunch &a, const Workspace &ws, cudaStream
     const int S = max(1, min(groups, kMaxNodes / a.N));
     VerifyArgs args{a, ws, S};
     verify_kernel<<<dim3(S, a.N, a.B), kThreadsV, 0, s>>>(args);
-    return cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return launch_dependent(walk_kernel, dim3(a.B), dim3(kThreadsV), 0, s, args);
 }
 
 }  // namespace adapld
