@@ -36,7 +36,6 @@ struct Workspace {
     int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
     int32_t *npairs;         // [1]  successor backoff: (sequence, branch) pairs
     int32_t *gticket_rep;    // [1]  distinct-token lists: sequences done (plan)
-    int32_t *vticket;        // [B]  verification: CTAs done per sequence
     int32_t *done3;          // [B*W] successor backoff: CTAs done per pair
     int32_t *rticket;        // [B]  distinct-token lists: chunks counted per sequence
     int32_t *xticket;        // [B]  expansion of the fallback lists: slices done
@@ -102,7 +101,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         return r;
     };
     const size_t BW = (size_t)B * w.W;
-    w.counters_bytes = sizeof(int32_t) * (4 + 7 * (size_t)B + 2 * BW);
+    w.counters_bytes = sizeof(int32_t) * (4 + 6 * (size_t)B + 2 * BW);
     w.dev_status = (int32_t *)take(w.counters_bytes);
     if (p) {
         w.global_ticket = w.dev_status + 1;
@@ -112,8 +111,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         w.done2 = w.ticket1 + B;
         w.ticket4 = w.done2 + B;
         w.ticket5 = w.ticket4 + B;
-        w.vticket = w.ticket5 + B;
-        w.done3 = w.vticket + B;
+        w.done3 = w.ticket5 + B;
         w.rticket = w.done3 + BW;
         w.xticket = w.rticket + B;
         w.xticket2 = w.xticket + B;
