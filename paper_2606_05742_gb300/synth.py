@@ -292,10 +292,13 @@ def make_embeddings(w: Workload, V: int, de: int, seed: int = 0, synonyms: int =
     embedding fallback (Eq. 4) finds them and a candidate right before the
     anchor makes the anchor itself a branch token with no earlier
     occurrence (the successor backoff of Sec. 3.5).  numpy uint16 bits on
-    the CPU, a torch bf16 tensor when the workload lives on a GPU."""
+    the CPU, a torch bf16 tensor when the workload lives on a GPU.  A forced
+    miss in a history that already holds all V ids takes id V
+    (`force_no_hit`), so the table gets max(V, largest id + 1) rows."""
     tokens = w.tokens if isinstance(w.tokens, np.ndarray) else w.tokens.cpu().numpy()
     lengths = w.lengths if isinstance(w.lengths, np.ndarray) else w.lengths.cpu().numpy()
     rng = np.random.default_rng([seed, 31337, V, de])
+    V = max(V, int(tokens.max()) + 1) if tokens.size else V
     plants = []
     for b in w.forced:
         ln = int(lengths[b])

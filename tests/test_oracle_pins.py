@@ -177,6 +177,19 @@ def test_forced_no_hit_sequences_miss():
             assert n == 0 and c == []
 
 
+def test_forced_miss_over_a_full_vocabulary():
+    """A history that holds every id of a small vocabulary can only miss
+    with id V; the embedding table then grows a row for it."""
+    V = 300
+    w = synth.make_workload(5, B=3, L=9000, d=8, V=V, nohit=1.0, seed=2064)
+    for b in range(w.B):
+        ln = int(w.lengths[b])
+        assert oracle.lexical(w.tokens[b, :ln], w.n_max, w.k)[0] == 0
+    assert int(w.tokens.max()) == V
+    E = synth.make_embeddings(w, V, 8, 1)
+    assert E.shape == (V + 1, 8)
+
+
 # --------------------------------------------------------------- semantic
 def test_cosine_closed_forms():
     rng = np.random.default_rng(1)
