@@ -49,6 +49,8 @@ struct Workspace {
     int32_t *rr_cand;        // [B][kMaxK] reranked lexical candidates (successor scan)
     float *rr_score;         // [B][kMaxK] their scores
     float *score5;           // [B][W*kMaxK] scores computed by the tree kernel
+    int32_t *tok5;           // [B][W*kMaxK] first successor token of each scored candidate
+    int32_t *brs;            // [B][1 + W] branch count and branch tokens (successor scan)
     int64_t *plan3;          // [B*W+1] successor backoff plan
     int32_t *slots3;         // [B*W + kMaxGrid2][kSlotInts] its partial lists
     int32_t *pair_b;         // [B*W] real sequence of each backoff pair
@@ -125,6 +127,8 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.rr_cand = (int32_t *)take(sizeof(int32_t) * (size_t)B * kMaxK);
     w.rr_score = (float *)take(sizeof(float) * (size_t)B * kMaxK);
     w.score5 = (float *)take(sizeof(float) * (size_t)B * w.W * kMaxK);
+    w.tok5 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.W * kMaxK);
+    w.brs = (int32_t *)take(sizeof(int32_t) * (size_t)B * (w.W + 1));
     w.plan3 = (int64_t *)take(sizeof(int64_t) * (BW + 1));
     w.slots3 = (int32_t *)take(sizeof(int32_t) * (BW + kMaxGrid2) * kSlotInts);
     w.pair_b = (int32_t *)take(sizeof(int32_t) * BW);

@@ -10,12 +10,13 @@
 //
 // succ_scan_kernel, grid (S4 slices, B), 512 threads -- only for sequences
 // that draft successors (Algorithm 1: semantic hits; every hit under
-// ADAPLD_SUCC_ON_STRICT).  Each CTA rebuilds the anchor and the branch set
-// (lexical hits are reranked here in that mode), then scans its slice of
-// 8192 positions for the branch tokens, a warp per branch, backwards with
-// ballots, keeping the k most recent occurrences.  The last slice CTA
+// ADAPLD_SUCC_ON_STRICT).  Each CTA stages its slice of 8192 positions (and
+// the one after it) while it reads the sequence's outcome, rebuilds the
+// anchor and the branch set (lexical hits are reranked here in that mode),
+// then scans the slice for the branch tokens, a warp per branch, backwards
+// with ballots, keeping the k most recent occurrences.  The last slice CTA
 // (atomic ticket; none with one slice) merges the slices, most recent first,
-// into the successor candidate lists.
+// into the successor candidate lists; slice 0 publishes the branch set.
 //
 // tree_kernel, grid (R5, B), 512 threads.  Every sequence has a list of rows
 // to score: the lexical candidates against the query (Eq. 6), or every
@@ -26,6 +27,14 @@
 // then ranks the lexical candidates (Eq. 7), picks each branch's successor
 // (Eq. 14), lays out the tree (root, main chain, branch paths with their
 // successors) and writes tokens, parents, position ids and the ancestor mask.
+//
+// Each of these CTAs moves a few KB, so its time is the number of dependent
+// memory round trips.  Loads that do not depend on one another are issued
+// together: the branch set, the ranked candidates and each warp's list entry
+// with the sequence's outcome; each warp's first row with the reference
+// vector, the candidates' continuation tokens and the token after each scored
+// row.  With one slice the fused kernel reads every history token it needs
+// from the staged slice.
 #include "common.cuh"
 
 namespace adapld {
@@ -33,6 +42,9 @@ namespace adapld {
 namespace {
 
 constexpr int kRowsPerCta5 = kThreads4 / 32;  // one warp per scored row
+constexpr int kWin = 16;  // continuation tokens staged per lexical candidate
+constexpr int kVecPer = 16384 / 8 / kThreads4;  // 16-byte chunks per thread of a staged vector
+static_assert(kMaxK * kWin == kThreads4, "one continuation token per thread");
 
 struct TreeArgs {
     TreeLaunch p;
@@ -45,10 +57,16 @@ struct TreeArgs {
 struct TreeSmem {
     int cand[kMaxK];
     float score[kMaxK];
+    int slot[kMaxK];  // window row (win) of each ranked candidate
     int next[kMaxW];
     int br[kMaxW];
-    int succ[kMaxW];
+    int succ[kMaxW];  // the successor picked for each branch (Eq. 14)
+    int stok[kMaxW];  // and the token after it
     int misc[4];
+    int lpos[kMaxK];  // rows of a CTA that scores all of its sequence's rows:
+    float lsc[kMaxK];  //   position, score and the token after the position
+    int ltok[kMaxK];
+    int win[kMaxK][kWin];  // M[c+1 .. c+kWin] of each lexical candidate c (-1 past len-1)
     int node_par[kMaxNodes];
     short node_depth[kMaxNodes];
     short node_path[kMaxNodes];
@@ -56,76 +74,136 @@ struct TreeSmem {
     float red[32];
 };
 
-// <row, ref> and |row|^2 of one bf16 row in global memory against an fp32
-// vector in shared memory (one warp, U independent 16-byte loads per lane in
-// flight).  A lane sums its chunks lane, lane + 32, ... in the same order
-// whatever U, so the result does not depend on U.
-template <int U = 16>
-__device__ __forceinline__ void warp_row_dot(const uint16_t *row, const float *ref, int d,
-                                             float &dot_out, float &ss_out) {
+// Where a CTA reads history tokens: the staged history (s_tok: positions
+// [0, ld) of the sequence), or global memory; wsm, when set, holds the
+// continuation windows of the candidates (M[s_cand[q]+1] = win[slot[q]][0]).
+struct TokSrc {
+    const int *s_tok;
+    const TreeSmem *wsm;
+};
+
+// Asynchronous global -> shared copies (no registers held while in flight).
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem));
+}
+__device__ __forceinline__ void cp_async4(void *smem, const void *gmem) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem)), "l"(gmem));
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+    asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+// One warp's dot product of a bf16 row in global memory with a bf16 vector
+// in shared memory (both widened exactly to fp32), in batches of U 16-byte
+// chunks per lane: chunk
+// base + 32u + lane for u < U.  A lane sums its chunks lane, lane + 32, ... in
+// increasing order whatever U, so the result does not depend on U or on where
+// the first batch was loaded.
+template <int U>
+__device__ __forceinline__ void row_batch_load(const uint16_t *row, int nch, int base,
+                                               uint4 (&w)[U]) {
     const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+        const int ch = base + u * 32 + lane;
+        w[u] = ch < nch ? ldg_nc_v4(row + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
+    }
+}
+
+template <int U>
+__device__ __forceinline__ void row_batch_acc(const uint4 (&w)[U], const uint16_t *ref, int nch,
+                                              int base, float &dot, float &ss) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+        const int ch = base + u * 32 + lane;
+        if (ch < nch) {
+            const uint4 rv = *(const uint4 *)(ref + ch * 8);
+            const float4 r0 = make_float4(bf16lo(rv.x), bf16hi(rv.x), bf16lo(rv.y), bf16hi(rv.y));
+            const float4 r1 = make_float4(bf16lo(rv.z), bf16hi(rv.z), bf16lo(rv.w), bf16hi(rv.w));
+            const float x0 = bf16lo(w[u].x), x1 = bf16hi(w[u].x);
+            const float x2 = bf16lo(w[u].y), x3 = bf16hi(w[u].y);
+            const float x4 = bf16lo(w[u].z), x5 = bf16hi(w[u].z);
+            const float x6 = bf16lo(w[u].w), x7 = bf16hi(w[u].w);
+            dot = fmaf(x0, r0.x, dot);
+            dot = fmaf(x1, r0.y, dot);
+            dot = fmaf(x2, r0.z, dot);
+            dot = fmaf(x3, r0.w, dot);
+            dot = fmaf(x4, r1.x, dot);
+            dot = fmaf(x5, r1.y, dot);
+            dot = fmaf(x6, r1.z, dot);
+            dot = fmaf(x7, r1.w, dot);
+            ss = fmaf(x0, x0, ss);
+            ss = fmaf(x1, x1, ss);
+            ss = fmaf(x2, x2, ss);
+            ss = fmaf(x3, x3, ss);
+            ss = fmaf(x4, x4, ss);
+            ss = fmaf(x5, x5, ss);
+            ss = fmaf(x6, x6, ss);
+            ss = fmaf(x7, x7, ss);
+        }
+    }
+}
+
+// <row, ref> and |row|^2 (warp totals); w holds the row's first batch.
+template <int U>
+__device__ __forceinline__ void warp_row_dot_from(const uint16_t *row, const uint16_t *ref, int d,
+                                                  uint4 (&w)[U], float &dot_out, float &ss_out) {
     const int nch = d >> 3;
     float dot = 0.f, ss = 0.f;
-    for (int base = 0; base < nch; base += 32 * U) {
-        uint4 w[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int ch = base + u * 32 + lane;
-            w[u] = ch < nch ? ldg_nc_v4(row + (size_t)ch * 8) : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int ch = base + u * 32 + lane;
-            if (ch < nch) {
-                const float4 r0 = *(const float4 *)(ref + ch * 8);
-                const float4 r1 = *(const float4 *)(ref + ch * 8 + 4);
-                const float x0 = bf16lo(w[u].x), x1 = bf16hi(w[u].x);
-                const float x2 = bf16lo(w[u].y), x3 = bf16hi(w[u].y);
-                const float x4 = bf16lo(w[u].z), x5 = bf16hi(w[u].z);
-                const float x6 = bf16lo(w[u].w), x7 = bf16hi(w[u].w);
-                dot = fmaf(x0, r0.x, dot);
-                dot = fmaf(x1, r0.y, dot);
-                dot = fmaf(x2, r0.z, dot);
-                dot = fmaf(x3, r0.w, dot);
-                dot = fmaf(x4, r1.x, dot);
-                dot = fmaf(x5, r1.y, dot);
-                dot = fmaf(x6, r1.z, dot);
-                dot = fmaf(x7, r1.w, dot);
-                ss = fmaf(x0, x0, ss);
-                ss = fmaf(x1, x1, ss);
-                ss = fmaf(x2, x2, ss);
-                ss = fmaf(x3, x3, ss);
-                ss = fmaf(x4, x4, ss);
-                ss = fmaf(x5, x5, ss);
-                ss = fmaf(x6, x6, ss);
-                ss = fmaf(x7, x7, ss);
-            }
-        }
+    row_batch_acc<U>(w, ref, nch, 0, dot, ss);
+    for (int base = 32 * U; base < nch; base += 32 * U) {
+        row_batch_load<U>(row, nch, base, w);
+        row_batch_acc<U>(w, ref, nch, base, dot, ss);
     }
     dot_out = warp_sum(dot);
     ss_out = warp_sum(ss);
 }
 
-// Loads a bf16 vector into shared memory as fp32 and returns its squared
-// norm (block-wide; every thread gets the same value).
-__device__ float block_load_vec(const uint16_t *v, float *dst, int d, float *scratch) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    float part = 0.f;
-    for (int ch = threadIdx.x; ch < (d >> 3); ch += blockDim.x) {
-        const uint4 w = ldg_nc_v4(v + (size_t)ch * 8);
-        const float x[8] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y),
-                            bf16lo(w.z), bf16hi(w.z), bf16lo(w.w), bf16hi(w.w)};
+template <int U>
+__device__ __forceinline__ void warp_row_dot(const uint16_t *row, const uint16_t *ref, int d,
+                                             float &dot_out, float &ss_out) {
+    uint4 w[U];
+    row_batch_load<U>(row, d >> 3, 0, w);
+    warp_row_dot_from<U>(row, ref, d, w, dot_out, ss_out);
+}
+
+// A bf16 vector of d <= 16384 elements staged in shared memory (16-byte
+// aligned, d bf16) by the 512-thread block: vec_issue starts its copies (at
+// most kVecPer per thread), vec_finish waits for every cp.async of the
+// thread and returns the squared norm to every thread (block-wide;
+// synchronises the block).
+__device__ __forceinline__ void vec_issue(const uint16_t *v, int d, uint16_t *dst) {
+    const int nch = d >> 3;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            dst[ch * 8 + e] = x[e];
-            part = fmaf(x[e], x[e], part);
+    for (int u = 0; u < kVecPer; ++u) {
+        const int ch = u * kThreads4 + threadIdx.x;
+        if (ch < nch) cp_async16(dst + ch * 8, v + (size_t)ch * 8);
+    }
+}
+
+__device__ float vec_finish(const uint16_t *dst, int d, float *scratch) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nch = d >> 3;
+    cp_async_wait_all();
+    __syncthreads();
+    float part = 0.f;
+#pragma unroll
+    for (int u = 0; u < kVecPer; ++u) {
+        const int ch = u * kThreads4 + threadIdx.x;
+        if (ch < nch) {
+            const uint4 w = *(const uint4 *)(dst + ch * 8);
+            const float x[8] = {bf16lo(w.x), bf16hi(w.x), bf16lo(w.y), bf16hi(w.y),
+                                bf16lo(w.z), bf16hi(w.z), bf16lo(w.w), bf16hi(w.w)};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) part = fmaf(x[e], x[e], part);
         }
     }
     part = warp_sum(part);
     if (lane == 0) scratch[warp] = part;
     __syncthreads();
     float tot = 0.f;
-    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += scratch[w];
+    for (int w = 0; w < kThreads4 / 32; ++w) tot += scratch[w];
     __syncthreads();
     return tot;
 }
@@ -171,21 +249,57 @@ __device__ __forceinline__ SeqView view_of(const TreeLaunch &a, int b) {
     return v;
 }
 
+// Values written by earlier kernels that a tree-kernel CTA may need, loaded
+// together with the sequence's outcome.  They are read in bounds but
+// speculatively (possibly stale) and used only where the outcome says the
+// successor scan wrote them.
+struct TreePrefetch {
+    int brs;       // thread t <= W: the branch count (t = 0), then the branch tokens
+    int rr_c;      // thread t < k: the candidates as ranked by the successor scan
+    float rr_s;
+    int task_pos;  // the first row of this thread's warp: its successor candidate
+    int task_n;    // and the candidate count of its branch
+};
+
+__device__ __forceinline__ TreePrefetch prefetch_tree(const TreeLaunch &a, const Workspace &ws,
+                                                      int b, int r5) {
+    TreePrefetch f;
+    const int t = threadIdx.x, k = a.p.k, W = ws.W;
+    f.brs = t <= W ? __ldcg(ws.brs + (int64_t)b * (W + 1) + t) : 0;
+    f.rr_c = t < k ? __ldcg(ws.rr_cand + (int64_t)b * kMaxK + t) : 0;
+    f.rr_s = t < k ? __ldcg(ws.rr_score + (int64_t)b * kMaxK + t) : 0.f;
+    const int task = r5 * kRowsPerCta5 + (t >> 5);
+    const int w = task / k, i = task - w * k;
+    const bool in = w < W;
+    f.task_pos = in ? __ldcg(ws.succ + ((int64_t)b * W + w) * kMaxK + i) : -1;
+    f.task_n = in ? __ldcg(ws.succ_n + (int64_t)b * W + w) : 0;
+    return f;
+}
+
+__device__ __forceinline__ int tok_at(const TokSrc &src, const int32_t *M, int p) {
+    return src.s_tok ? src.s_tok[p] : __ldg(M + p);
+}
+
 // Branch set (Eq. 10-11) into s_br, count returned; s_cand holds the ranked
 // candidates (s_cand[0] = j*).  Block-wide: every thread must call.
 __device__ __forceinline__ int branch_set(const TreeLaunch &a, int b, const SeqView &v,
-                                          const int *s_cand,
-                          int *s_next, int *s_br, int *s_misc) {
+                                          const int *s_cand, int *s_next, int *s_br,
+                                          int *s_misc, const TokSrc &src) {
     const int t = threadIdx.x, W = a.p.branch_width;
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
-    const int js = s_cand[0];
+    // M[s_cand[q] + 1], the continuation of ranked candidate q
+    auto next_of = [&](int q) {
+        if (src.s_tok) return src.s_tok[s_cand[q] + 1];
+        if (src.wsm) return src.wsm->win[src.wsm->slot[q]][0];
+        return __ldg(M + s_cand[q] + 1);
+    };
     if (a.next_topk) {
-        const int32_t *row = a.next_topk + ((int64_t)b * a.ld + js) * a.Kn;
+        const int32_t *row = a.next_topk + ((int64_t)b * a.ld + s_cand[0]) * a.Kn;
         if (t < a.Kn) s_next[t] = row[t];
     } else if (t < v.nc) {
-        s_next[t] = M[s_cand[t] + 1];
+        s_next[t] = next_of(t);
     }
-    if (t == kThreads4 - 1) s_misc[0] = v.lex ? M[js + 1] : -1;
+    if (t == kThreads4 - 1) s_misc[0] = v.lex ? next_of(0) : -1;
     __syncthreads();
     if (t == 0) {
         int nb = 0;
@@ -213,11 +327,13 @@ __device__ __forceinline__ int branch_set(const TreeLaunch &a, int b, const SeqV
 }
 
 // Warp 0 sorts n <= 32 (score, position) pairs in place by (score desc,
-// position desc).
-__device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int n) {
+// position desc); s_slot, when given, is permuted alongside.
+__device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int n,
+                                               int *s_slot) {
     const int lane = threadIdx.x & 31;
     const float sc = lane < n ? s_score[lane] : -INFINITY;
     const int cj = lane < n ? s_cand[lane] : -1;
+    const int sl = (s_slot && lane < n) ? s_slot[lane] : 0;
     int rank = 0;
     for (int m = 0; m < n; ++m) {
         const float os = __shfl_sync(0xffffffffu, sc, m);
@@ -228,6 +344,7 @@ __device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int 
     if (lane < n) {
         s_cand[rank] = cj;
         s_score[rank] = sc;
+        if (s_slot) s_slot[rank] = sl;
     }
     __syncwarp();
 }
@@ -250,38 +367,54 @@ __device__ __forceinline__ void register_successors(const TreeLaunch &a, const W
 
 template <int U>
 __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const SeqView &v,
-                          int r5, bool fused, TreeSmem &sm, float *s_ref);
+                          int r5, bool fused, TreeSmem &sm, uint16_t *s_ref, const TokSrc &src,
+                          const TreePrefetch *pf, int nb_known, bool lists_smem);
 
 // FUSED: the CTA that completes a sequence's scan (or CTA 0 of a sequence
 // without successors) then builds that sequence's tree itself (tree_body,
 // all scored rows in this CTA), so the tree stage is one kernel.  U: row
-// loads in flight in tree_body.
+// loads in flight in tree_body.  Dynamic shared memory: d bf16 (the query or
+// reference vector), then kSlice4 + 1 ints (this slice's tokens).
 template <int U, bool FUSED>
 __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(TreeArgs args) {
     const TreeLaunch &a = args.p;
     const Workspace &ws = args.ws;
-    __shared__ int s_tok[kSlice4];
     __shared__ TreeSmem sm;
+    extern __shared__ __align__(16) uint16_t s_dyn[];
+    uint16_t *s_q = s_dyn;
+    int *s_tok = (int *)(s_dyn + a.d);
     int *s_cand = sm.cand;
     float *s_score = sm.score;
     int *s_next = sm.next;
     int *s_br = sm.br;
     int *s_misc = sm.misc;
     float *s_red = sm.red;
-    extern __shared__ __align__(16) float s_q[];  // [d] the query (fp32) for a rerank here
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int nwarps = kThreads4 / 32;
     const int b = blockIdx.y, sl = blockIdx.x;
     const int k = a.p.k, d = a.d;
-    pdl_wait_then_release();
-    const SeqView v = view_of(a, b);
-    if (!v.need_succ) {
-        if (FUSED && sl == 0) tree_body<U>(a, ws, b, v, 0, true, sm, s_q);
-        return;
-    }
+    const bool single = gridDim.x == 1;
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
+    pdl_wait_then_release();
+    // this slice's tokens, positions [p0, p0 + kSlice4] clipped at ld, copied
+    // while the sequence's outcome is read (they do not depend on it)
+    const int p0 = sl * kSlice4;
+    const int nld = (int)min((int64_t)kSlice4 + 1, a.ld - p0);
+    for (int i = t; i < nld; i += kThreads4) cp_async4(s_tok + i, M + p0 + i);
+    const SeqView v = view_of(a, b);
+    cp_async_wait_all();  // (also before an exit: the copies target this CTA's memory)
+    if (!v.need_succ && !(FUSED && sl == 0)) return;
+    __syncthreads();
+    // with one slice the staged tokens are the whole history
+    const TokSrc src{single ? s_tok : nullptr, nullptr};
+    if constexpr (FUSED) {
+        if (!v.need_succ) {
+            tree_body<U>(a, ws, b, v, 0, true, sm, s_q, src, nullptr, -1, false);
+            return;
+        }
+    }
 
     if (t < v.nc) {
         s_cand[t] = v.cand_t;
@@ -290,33 +423,45 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
     __syncthreads();
     if (v.rr) {  // the ranking the branches depend on (each slice alike; the
                  // arithmetic of the tree kernel's rerank, so the scores agree)
-        const float qss = block_load_vec(a.query + (int64_t)b * d, s_q, d, s_red);
-        for (int ci = warp; ci < v.nc; ci += nwarps) {
+        uint4 w0[8];  // each warp's first candidate row, loaded with the query
+        if (warp < v.nc) row_batch_load<8>(R + (int64_t)s_cand[warp] * d, d >> 3, 0, w0);
+        vec_issue(a.query + (int64_t)b * d, d, s_q);
+        const float qss = vec_finish(s_q, d, s_red);
+        if (warp < v.nc) {
+            float dot, ss;
+            warp_row_dot_from<8>(R + (int64_t)s_cand[warp] * d, s_q, d, w0, dot, ss);
+            if (lane == 0) s_score[warp] = cosine_from(dot, ss, qss);
+        }
+        for (int ci = warp + nwarps; ci < v.nc; ci += nwarps) {
             float dot, ss;
             warp_row_dot<8>(R + (int64_t)s_cand[ci] * d, s_q, d, dot, ss);
             if (lane == 0) s_score[ci] = cosine_from(dot, ss, qss);
         }
         __syncthreads();
-        if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc);
+        if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc, nullptr);
         __syncthreads();
     } else if (v.lex) {
         if (t < v.nc) s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
         __syncthreads();
     }
-    const int nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc);
+    const int nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc, src);
+    if (!FUSED && sl == 0) {  // the branch set, for the tree kernel
+        int32_t *bo = ws.brs + (int64_t)b * (ws.W + 1);
+        if (t == 0) bo[0] = nb;
+        if (t < nb) bo[1 + t] = s_br[t];
+    }
 
-    const int p0 = sl * kSlice4;
     const int p1 = min(p0 + kSlice4, v.len - 1);  // positions t <= len-2
-    for (int i = t; i < p1 - p0; i += kThreads4) s_tok[i] = M[p0 + i];
-    __syncthreads();
     constexpr int G = 8;  // 32-position groups tested per pass (independent loads)
-    // one slice: its lists are the merged result, written in place (no merge)
-    const bool single = gridDim.x == 1;
+    // one slice: its lists are the merged result, written in place (no merge);
+    // the fused kernel keeps them in shared memory (W*k <= 16)
+    const bool lists_smem = FUSED && single;
     for (int w = warp; w < nb; w += nwarps) {
         const int bt = s_br[w];
         int32_t *part =
             single ? nullptr : ws.part4 + (((int64_t)b * ws.S4 + sl) * ws.W + w) * kPart4Ints;
-        int32_t *lst = single ? ws.succ + ((int64_t)b * ws.W + w) * kMaxK : part + 1;
+        int32_t *lst = lists_smem ? sm.lpos + w * k
+                                  : (single ? ws.succ + ((int64_t)b * ws.W + w) * kMaxK : part + 1);
         int cnt = 0;
         for (int top = p1 - 1; top >= p0 && cnt < k; top -= 32 * G) {
             unsigned m[G];
@@ -332,6 +477,10 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
                 if (((m[u] >> lane) & 1u) && rank < k) lst[rank] = p;
                 cnt += __popc(m[u]);
             }
+        }
+        if (lists_smem) {  // entries past the count read as "no row"
+            __syncwarp();
+            for (int i = min(cnt, k) + lane; i < k; i += 32) lst[i] = -1;
         }
         if (lane == 0) {
             if (single)
@@ -358,20 +507,19 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
             if (lane == 0) register_successors(a, ws, b, w, total, s_br[w]);
         }
     }
-    if ((v.lex || v.rr) && t < v.nc) {
+    if (!FUSED && (v.lex || v.rr) && t < v.nc) {
         ws.rr_cand[(int64_t)b * kMaxK + t] = s_cand[t];
         ws.rr_score[(int64_t)b * kMaxK + t] = s_score[t];
     }
-    if (FUSED) {
+    if constexpr (FUSED) {
         __syncthreads();  // the lists and the ranking above are visible to the block
-        tree_body<U>(a, ws, b, v, 0, true, sm, s_q);
+        tree_body<U>(a, ws, b, v, 0, true, sm, s_q, src, nullptr, nb, lists_smem);
     }
 }
 
 // The plan of the successor backoff pass: row prefix sums over the
 // (sequence, branch) pairs registered by succ_scan_kernel (one CTA).
 __global__ void __launch_bounds__(256) backoff_plan_kernel(TreeArgs args) {
-    const TreeLaunch &a = args.p;
     const Workspace &ws = args.ws;
     __shared__ int64_t scratch[8];
     pdl_wait_then_release();
@@ -409,10 +557,14 @@ __global__ void __launch_bounds__(256) backoff_plan_kernel(TreeArgs args) {
 // The tree stage of sequence b for one CTA (all threads): CTA r5 of the
 // sequence scores its share of rows (every row when `fused`); the CTA that
 // completes the sequence ranks, picks successors and emits the tree.  s_ref:
-// d floats of shared memory.
+// d bf16 of shared memory (16-byte aligned).  src: where history tokens are read.  pf: the
+// tree kernel's prefetched values (NULL in the fused kernel).  nb_known >= 0:
+// the fused scan left the ranked candidates and the branch set (nb_known
+// branches) in sm.  lists_smem: the successor lists are in sm.lpos.
 template <int U>
 __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const SeqView &v,
-                          int r5, bool fused, TreeSmem &sm, float *s_ref) {
+                          int r5, bool fused, TreeSmem &sm, uint16_t *s_ref, const TokSrc &src,
+                          const TreePrefetch *pf, int nb_known, bool lists_smem) {
     int *s_cand = sm.cand;
     float *s_score = sm.score;
     int *s_next = sm.next;
@@ -435,20 +587,25 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
     // the status word is rewritten at the end; its token bit comes from
     // earlier kernels, so it is read now, off the tail's critical path
     const int status0 = (a.status && t == 0) ? a.status[b] : 0;
+    if (t < kMaxK) sm.slot[t] = t;
 
-    // ---- ranked candidates (the successor scan reranked a strict hit already)
-    if (t < v.nc) {
-        if (v.need_succ && (v.lex || v.rr)) {
-            s_cand[t] = __ldcg(ws.rr_cand + (int64_t)b * kMaxK + t);
-            s_score[t] = __ldcg(ws.rr_score + (int64_t)b * kMaxK + t);
-        } else {
-            s_cand[t] = v.cand_t;
-            s_score[t] = v.score_t;
+    // ---- ranked candidates; with successors, the branch set
+    int nb = 0;
+    if (nb_known >= 0) {
+        nb = nb_known;
+    } else {
+        if (t < v.nc) {  // the successor scan ranked these already
+            const bool from_scan = pf && v.need_succ && (v.lex || v.rr);
+            s_cand[t] = from_scan ? pf->rr_c : v.cand_t;
+            s_score[t] = from_scan ? pf->rr_s : v.score_t;
         }
+        if (pf && v.need_succ) {  // published by the successor scan
+            if (t >= 1 && t <= ws.W) s_br[t - 1] = pf->brs;
+            if (t == 0) s_misc[1] = pf->brs;
+        }
+        __syncthreads();
+        if (v.need_succ) nb = s_misc[1];
     }
-    __syncthreads();
-    // with successors the ranking is final here, so the branch set is known
-    int nb = v.need_succ ? branch_set(a, b, v, s_cand, s_next, s_br, s_misc) : 0;
 
     // the rows this sequence scores, and the CTAs that share them: lexical
     // candidates against the query, or successor candidate (w, i) at w*k + i
@@ -456,33 +613,76 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
     const int ntasks = v.need_succ ? nb * k : (rerank ? v.nc : 0);
     const int nctas = fused ? 1 : max(1, (ntasks + kRowsPerCta5 - 1) / kRowsPerCta5);
     if (r5 >= nctas) return;
+    const bool local = nctas == 1;  // every row in this CTA: results stay in sm
     const int js0 = (v.lex || v.sem) ? s_cand[0] : -1;
     float *score5 = ws.score5 + (int64_t)b * ws.W * kMaxK;
+    int32_t *tok5 = ws.tok5 + (int64_t)b * ws.W * kMaxK;
+    // continuation windows of the candidates (branch tokens, main chain) when
+    // the history is not staged
+    const bool use_win = !src.s_tok && v.nc > 0 && (v.lex || (v.branch_on && !v.need_succ));
 
-    // ---- this CTA's share of the scored rows
+    // ---- this CTA's share of the scored rows, every independent load first
+    const int task0 = fused ? 0 : r5 * kRowsPerCta5;
+    const int task1 = fused ? ntasks : min(ntasks, task0 + kRowsPerCta5);
+    auto row_of = [&](int task, bool first) -> int {
+        if (!v.need_succ) return s_cand[task];
+        if (lists_smem) return sm.lpos[task];
+        const int w = task / k, i = task - w * k;
+        int n, pos;
+        if (first && pf) {
+            n = pf->task_n;
+            pos = pf->task_pos;
+        } else {
+            n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
+            pos = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i);
+        }
+        return i < n ? pos : -1;
+    };
+    const int first_task = task0 + warp;
+    const int row0 = first_task < task1 ? row_of(first_task, true) : -1;
+    uint4 w0[U];
+    if (row0 >= 0) row_batch_load<U>(R + (int64_t)row0 * d, d >> 3, 0, w0);
+    if (ntasks > 0)
+        vec_issue(v.need_succ ? R + (int64_t)(js0 + 1) * d : a.query + (int64_t)b * d, d, s_ref);
+    const int tk0 = (v.need_succ && row0 >= 0 && lane == 0) ? tok_at(src, M, row0 + 1) : -1;
+    if (use_win && t < v.nc * kWin) {
+        const int r = t / kWin, o = t - r * kWin;
+        const int p = s_cand[r] + 1 + o;
+        sm.win[r][o] = p <= v.len - 1 ? __ldg(M + p) : -1;
+    }
     if (ntasks > 0) {
-        // this CTA's tasks: 16 (one per warp), or all of them when fused
-        const int task0 = fused ? 0 : r5 * kRowsPerCta5;
-        const int task1 = fused ? ntasks : min(ntasks, task0 + kRowsPerCta5);
-        const uint16_t *ref = v.need_succ ? R + (int64_t)(js0 + 1) * d : a.query + (int64_t)b * d;
-        const float rss = block_load_vec(ref, s_ref, d, s_red);  // syncs the block
-        for (int task = task0 + warp; task < task1; task += nwarps) {
-            int row;
-            if (v.need_succ) {
-                const int w = task / k, i = task % k;
-                const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
-                const int pos = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + i);
-                row = i < n ? pos : -1;
+        const float rss = vec_finish(s_ref, d, s_red);  // syncs the block
+        auto record = [&](int task, int row, float sc, int tk) {  // lane 0
+            if (local) {
+                sm.lpos[task] = row;
+                sm.lsc[task] = sc;
+                sm.ltok[task] = tk;
             } else {
-                row = s_cand[task];
+                if (row >= 0) score5[task] = sc;
+                if (v.need_succ) tok5[task] = tk;
             }
+        };
+        if (first_task < task1) {  // the first row's loads are in flight already
+            float sc = 0.f;
+            if (row0 >= 0) {
+                float dot, ss;
+                warp_row_dot_from<U>(R + (int64_t)row0 * d, s_ref, d, w0, dot, ss);
+                sc = cosine_from(dot, ss, rss);
+            }
+            if (lane == 0) record(first_task, row0, sc, tk0);
+        }
+        for (int task = first_task + nwarps; task < task1; task += nwarps) {
+            const int row = row_of(task, false);
+            float sc = 0.f;
             if (row >= 0) {
                 float dot, ss;
                 warp_row_dot<U>(R + (int64_t)row * d, s_ref, d, dot, ss);
-                if (lane == 0) score5[task] = cosine_from(dot, ss, rss);
+                sc = cosine_from(dot, ss, rss);
             }
+            if (lane == 0)
+                record(task, row, sc, (v.need_succ && row >= 0) ? tok_at(src, M, row + 1) : -1);
         }
-        if (nctas > 1) {
+        if (!local) {
             __threadfence();
             __syncthreads();
             if (t == 0) s_misc[2] = atomicAdd(ws.ticket5 + b, 1) == nctas - 1;
@@ -492,14 +692,16 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
         } else {
             __syncthreads();
         }
+    } else {
+        __syncthreads();  // the windows are visible to the block
     }
 
     // ---- the last CTA of the sequence: rank, branch, pick successors, emit
     if (rerank) {
         if (warp == 0) {
-            if (lane < v.nc) s_score[lane] = __ldcg(score5 + lane);
+            if (lane < v.nc) s_score[lane] = local ? sm.lsc[lane] : __ldcg(score5 + lane);
             __syncwarp();
-            warp_sort_desc(s_cand, s_score, v.nc);
+            warp_sort_desc(s_cand, s_score, v.nc, sm.slot);
         }
         __syncthreads();
     } else if (v.lex && (flags & ADAPLD_NO_LEX_RERANK)) {
@@ -507,25 +709,43 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
         __syncthreads();
     }
     const int js = (v.lex || v.sem) ? s_cand[0] : -1;
-    if (v.branch_on && !v.need_succ) nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc);
+    if (v.branch_on && !v.need_succ)
+        nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc,
+                        TokSrc{src.s_tok, use_win ? &sm : nullptr});
     if (v.need_succ) {
         for (int w = warp; w < nb; w += nwarps) {  // Eq. 14: argmax per branch
-            // all three loads at once (lanes past the count are masked after)
-            const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
-            const float sl = __ldcg(score5 + w * k + lane);
-            const int pl = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + lane);
-            float bs = lane < n ? sl : -INFINITY;
-            int bj = lane < n ? pl : -1;
+            float bs;
+            int bj, btk;
+            if (local) {
+                const int pl = lane < k ? sm.lpos[w * k + lane] : -1;
+                bs = pl >= 0 ? sm.lsc[w * k + lane] : -INFINITY;
+                bj = pl;
+                btk = pl >= 0 ? sm.ltok[w * k + lane] : -1;
+            } else {
+                // all four loads at once (lanes past the count are masked after)
+                const int n = __ldcg(ws.succ_n + (int64_t)b * ws.W + w);
+                const float sl = __ldcg(score5 + w * k + lane);
+                const int pl = __ldcg(ws.succ + ((int64_t)b * ws.W + w) * kMaxK + lane);
+                const int tl = __ldcg(tok5 + w * k + lane);
+                bs = lane < n ? sl : -INFINITY;
+                bj = lane < n ? pl : -1;
+                btk = tl;
+            }
 #pragma unroll
             for (int o = 16; o; o >>= 1) {
                 const float os = __shfl_xor_sync(0xffffffffu, bs, o);
                 const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+                const int ot = __shfl_xor_sync(0xffffffffu, btk, o);
                 if (better(os, oj, bs, bj)) {
                     bs = os;
                     bj = oj;
+                    btk = ot;
                 }
             }
-            if (lane == 0) s_succ[w] = n > 0 ? bj : -1;
+            if (lane == 0) {
+                s_succ[w] = bj >= 0 ? bj : -1;
+                sm.stok[w] = btk;
+            }
         }
         __syncthreads();
     }
@@ -576,10 +796,19 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
     for (int i = t; i < N; i += kThreads4) {
         int tok = -1, par = -1, pos = -1;
         if (i < n) {
-            const int src = node_src[i];
-            tok = src >= 0 ? M[src] : s_br[-2 - src];
+            const int s = node_src[i], path = node_path[i], depth = node_depth[i];
+            if (s < 0)
+                tok = s_br[-2 - s];
+            else if (src.s_tok)
+                tok = src.s_tok[s];
+            else if (path == 1 && use_win && depth <= kWin)  // main chain: s = j* + depth
+                tok = sm.win[sm.slot[0]][depth - 1];
+            else if (path >= 2 && depth == 2)  // a branch's first successor token
+                tok = sm.stok[path - 2];
+            else
+                tok = __ldg(M + s);
             par = node_par[i];
-            pos = v.len - 1 + node_depth[i];
+            pos = v.len - 1 + depth;
         }
         a.out.draft_tokens[ob + i] = tok;
         a.out.parents[ob + i] = par;
@@ -613,14 +842,16 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
 
 // U: row loads in flight per lane.  U = 16 (one CTA per SM by registers)
 // when the grid fits one wave, U = 8 (two CTAs per SM) otherwise; the
-// scores are the same either way (see warp_row_dot).
+// scores are the same either way (see row_batch_acc).
 template <int U>
 __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArgs args) {
     __shared__ TreeSmem sm;
-    extern __shared__ __align__(16) float s_ref[];  // [d] reference vector (fp32)
+    extern __shared__ __align__(16) uint16_t s_ref[];  // [d] reference vector (bf16)
     pdl_wait_then_release();
+    const TreePrefetch pf = prefetch_tree(args.p, args.ws, blockIdx.y, blockIdx.x);
     const SeqView v = view_of(args.p, blockIdx.y);
-    tree_body<U>(args.p, args.ws, blockIdx.y, v, blockIdx.x, false, sm, s_ref);
+    tree_body<U>(args.p, args.ws, blockIdx.y, v, blockIdx.x, false, sm, s_ref,
+                 TokSrc{nullptr, nullptr}, &pf, -1, false);
 }
 
 }  // namespace
@@ -631,6 +862,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
 // 16 rows (configs 1 and 4) fusing saves 2.4-2.7 us per step; with 24 or 64
 // rows (configs 2 and 3) the second kernel's parallel rows win by 4-14 us.
 constexpr int kMaxFusedTasks = kRowsPerCta5;
+static_assert(kMaxFusedTasks <= kMaxK, "fused lists live in TreeSmem::lpos");
 
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s) {
     const int W = a.p.branch_width, k = a.p.k;
@@ -642,16 +874,17 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return cudaErrorInvalidDevice;
-    const size_t vsmem = (size_t)a.d * sizeof(float);  // the staged query / reference row
+    const size_t vsmem = (size_t)a.d * sizeof(uint16_t);  // the staged query / reference row
+    const size_t ssmem = vsmem + (size_t)(kSlice4 + 1) * sizeof(int);  // + a slice's tokens
     if (succ_possible) {
         cudaError_t e;
         if (!a.emb.table && W * k <= kMaxFusedTasks) {  // scan and tree in one kernel
             auto kern = (int64_t)ws.S4 * a.B <= sms ? succ_scan_kernel<16, true>
                                                     : succ_scan_kernel<8, true>;
             e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)vsmem);
+                                     (int)ssmem);
             if (e != cudaSuccess) return e;
-            return launch_dependent(kern, dim3(ws.S4, a.B), dim3(kThreads4), vsmem, s, args);
+            return launch_dependent(kern, dim3(ws.S4, a.B), dim3(kThreads4), ssmem, s, args);
         }
         if (a.emb.table && !a.lists_ready) {  // distinct-token lists for the backoff
             DedupeLaunch da{a.tokens, a.ld,  a.lengths, a.B,     a.emb.vocab, nullptr, nullptr,
@@ -661,9 +894,9 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
             if (e != cudaSuccess) return e;
         }
         e = cudaFuncSetAttribute(succ_scan_kernel<8, false>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)vsmem);
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ssmem);
         if (e != cudaSuccess) return e;
-        e = launch_dependent(succ_scan_kernel<8, false>, dim3(ws.S4, a.B), dim3(kThreads4), vsmem,
+        e = launch_dependent(succ_scan_kernel<8, false>, dim3(ws.S4, a.B), dim3(kThreads4), ssmem,
                              s, args);
         if (e != cudaSuccess) return e;
         if (a.emb.table) {  // successor backoff over token embeddings
