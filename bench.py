@@ -173,17 +173,24 @@ class OracleSample:
     lexical miss and one lexical-hit sequence, truncated to ``rows`` positions
     and generated on the host.  The oracle's cost is linear in the positions,
     so a full step is extrapolated as n_miss * t_miss * (L-1)/(rows-1) +
-    n_hit * t_hit * L/rows."""
+    n_hit * t_hit * L/rows, with n_miss the lexical misses (the sequences
+    that run the semantic fallback) of the timed workload's own histories
+    (generated from the same seed; the oracle's lexical step counts them)."""
 
-    def __init__(self, cfg_id: int, seed: int, rows: int):
+    def __init__(self, cfg_id: int, seed: int, rows: int, batch=None):
+        import oracle
         from paper_2606_05742_gb300 import synth
         c = synth.CONFIGS[cfg_id]
-        self.L, B = c["L"], c["B"]
+        self.L = c["L"]
+        B = c["B"] if batch is None else batch
         self.rows = min(rows, self.L)
         self.w = synth.make_workload(cfg_id, B=2, L=self.rows, nohit=0.5, seed=seed + 1000)
         self.miss = int(self.w.forced[0])
         self.hit = 1 - self.miss
-        self.n_miss = int(synth.forced_set(cfg_id, B, c["nohit"], seed).size)
+        tokens, lengths, _ = synth.make_tokens(cfg_id, B=B, seed=seed)
+        self.n_miss = sum(
+            1 for b in range(B)
+            if oracle.lexical(tokens[b, : lengths[b]], c["n_max"], c["k"])[0] == 0)
         self.n_hit = B - self.n_miss
         self.desc = (f"oracle (1 thread) on 1 forced-miss + 1 lexical-hit sequence of config "
                      f"{cfg_id} truncated to {self.rows} positions (d={c['d']}), extrapolated "
@@ -237,7 +244,7 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    sample = OracleSample(args.config, args.seed, rows=4096)
+    sample = OracleSample(args.config, args.seed, rows=4096, batch=args.batch)
     threads = host_threads(sample.n_miss + sample.n_hit)
     for _ in range(args.warmup):
         sample.rate_parallel(threads)
@@ -530,7 +537,7 @@ def run_native(args):
     step_gbs = nbytes["step"] / (ms_per_step / 1000.0) / 1e9
     cpu = None
     if not args.no_cpu_baseline:
-        sample = OracleSample(cfg, args.seed, rows=65536)
+        sample = OracleSample(cfg, args.seed, rows=65536, batch=args.batch)
         threads = host_threads(sample.n_miss + sample.n_hit)
         v1 = statistics.median([sample.rate() for _ in range(3)])
         vp = statistics.median([sample.rate_parallel(threads) for _ in range(3)])

@@ -144,6 +144,34 @@ class Workload:
     device: str = "cpu"
 
 
+def make_tokens(cfg_id: int, *, B: Optional[int] = None, L: Optional[int] = None,
+                ld: Optional[int] = None, lengths=None, seed: int = 0,
+                nohit: Optional[float] = None, V: Optional[int] = None):
+    """The token histories of ``make_workload`` with the same arguments (the
+    same seeds), without the representation cache: (tokens [B][ld] int32,
+    lengths [B] int32, forced misses)."""
+    c = CONFIGS[cfg_id]
+    B = c["B"] if B is None else B
+    L = c["L"] if L is None else L
+    V = c["V"] if V is None else V
+    ld = L if ld is None else ld
+    frac = c["nohit"] if nohit is None else nohit
+    if lengths is None:
+        lengths = np.full(B, L, dtype=np.int32)
+    lengths = np.asarray(lengths, dtype=np.int32)
+    assert lengths.shape == (B,) and int(lengths.max()) <= ld
+    tokens = np.zeros((B, ld), dtype=np.int32)
+    forced = forced_set(cfg_id, B, frac, seed)
+    fset = set(forced.tolist())
+    for b in range(B):
+        rng = np.random.default_rng([seed, cfg_id, b])
+        tokens[b] = gen_tokens(rng, ld, V, c["copy"])
+        ln = int(lengths[b])
+        if b in fset and ln >= 1:
+            force_no_hit(tokens[b], ln, V)
+    return tokens, lengths, forced
+
+
 def make_workload(cfg_id: int, *, device: str = "cpu", B: Optional[int] = None,
                   L: Optional[int] = None, d: Optional[int] = None, ld: Optional[int] = None,
                   lengths=None, seed: int = 0, nohit: Optional[float] = None,
@@ -158,24 +186,10 @@ def make_workload(cfg_id: int, *, device: str = "cpu", B: Optional[int] = None,
     B = c["B"] if B is None else B
     L = c["L"] if L is None else L
     d = c["d"] if d is None else d
-    V = c["V"] if V is None else V
     ld = L if ld is None else ld
-    frac = c["nohit"] if nohit is None else nohit
     n_plant = c["planted"] if planted == -1 else planted
-    if lengths is None:
-        lengths = np.full(B, L, dtype=np.int32)
-    lengths = np.asarray(lengths, dtype=np.int32)
-    assert lengths.shape == (B,) and int(lengths.max()) <= ld
-
-    tokens = np.zeros((B, ld), dtype=np.int32)
-    forced = forced_set(cfg_id, B, frac, seed)
-    fset = set(forced.tolist())
-    for b in range(B):
-        rng = np.random.default_rng([seed, cfg_id, b])
-        tokens[b] = gen_tokens(rng, ld, V, c["copy"])
-        ln = int(lengths[b])
-        if b in fset and ln >= 1:
-            force_no_hit(tokens[b], ln, V)
+    tokens, lengths, forced = make_tokens(cfg_id, B=B, L=L, ld=ld, lengths=lengths, seed=seed,
+                                          nohit=nohit, V=V)
 
     planted_rows = []
     if device == "cpu":

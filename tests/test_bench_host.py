@@ -65,7 +65,7 @@ def test_reference_arm_prints_one_line(capsys):
     the contract's JSON line (small workload: config 1)."""
     import json
     import argparse
-    args = argparse.Namespace(config=1, seed=0, steps=2, warmup=1, gpus=1)
+    args = argparse.Namespace(config=1, seed=0, steps=2, warmup=1, gpus=1, batch=None)
     bench.run_reference(args)
     out = [ln for ln in capsys.readouterr().out.splitlines() if ln.startswith("{")]
     assert len(out) == 1
@@ -95,3 +95,15 @@ def test_algorithmic_bytes_embedding_mode():
     # and scores min(k, L-1) positions instead of none
     extra = (2 + 1) * 16 * 2 + (5 + 1) * de * 2 + 4 * L + 4 * 16 * 2
     assert x["tree"] - base["tree"] == extra
+
+
+def test_oracle_sample_counts_the_workloads_misses():
+    """The CPU baseline extrapolates to the timed workload's own lexical
+    misses: every forced miss, plus histories that miss naturally."""
+    from paper_2606_05742_gb300 import synth
+    sample = bench.OracleSample(2, 0, rows=256)
+    tokens, lengths, forced = synth.make_tokens(2, seed=0)
+    assert sample.n_miss + sample.n_hit == synth.CONFIGS[2]["B"]
+    assert sample.n_miss >= len(forced)
+    small = bench.OracleSample(2, 0, rows=256, batch=4)
+    assert small.n_miss + small.n_hit == 4
