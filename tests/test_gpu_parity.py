@@ -231,6 +231,36 @@ def test_longer_successors(succ_len):
     check_all(w, run_step(w, P), P)
 
 
+@pytest.mark.parametrize("flags", [0, oracle.SUCC_ON_STRICT])
+def test_maximum_tree(flags):
+    """The largest tree the boundary takes: 1 + D + W(1 + succ_len) = 1024
+    nodes (D = 255, W = 64, succ_len = 11, k = 32, n_max = 8), 64 branches from
+    a 64-wide next-token table, so every branch scans for successors and
+    2048 successor rows per sequence are scored."""
+    V = 4000
+    w = synth.make_workload(2, B=4, L=2000, d=64, V=V, nohit=0.5, seed=91)
+    tk = synth.make_next_topk(w.tokens, w.lengths, V, 64, seed=91)
+    P = P_of(w, n_max=8, k=32, W=64, D=255, succ_len=11, flags=flags, tau=NEG_INF)
+    g = run_step(w, P, next_topk=tk)
+    assert g["draft_tokens"].shape[1] == 1024
+    assert int(g["n_nodes"].max()) > 300
+    check_all(w, g, P, next_topk=tk)
+
+
+def test_maximum_batch():
+    """B = 65535, the largest batch (every kernel's grid y at its limit), of
+    short ragged histories; the oracle checks the first and last sequences
+    and a seeded sample, the statistics cover every sequence."""
+    B = 65535
+    rng = np.random.default_rng(65535)
+    lengths = rng.integers(1, 13, size=B).astype(np.int32)
+    w = synth.make_workload(4, B=B, L=12, d=8, V=50, nohit=0.3, seed=5, lengths=lengths)
+    P = P_of(w, tau=NEG_INF)
+    g = run_step(w, P)
+    sample = sorted({0, 1, B - 2, B - 1, *rng.choice(B, 1500, replace=False).tolist()})
+    check_all(w, g, P, seqs=sample)
+
+
 def test_next_token_table():
     w = synth.make_workload(2, B=6, L=400, d=64, nohit=0.5, seed=13)
     tk = synth.make_next_topk(w.tokens, w.lengths, 32000, 6)

@@ -228,6 +228,31 @@ def test_choice_across_row_splits():
     assert gpu["new"][0].tolist() == [100, 0, 50, V - 1]
 
 
+def test_maximum_trees_from_a_step():
+    """Trees of the largest size (1024 nodes: D = 255, W = 64, succ_len = 11,
+    branches from a 64-wide next-token table, successors on every hit) from
+    a GPU step, verified and appended (tokens, hidden-state rows, query)."""
+    rng = np.random.default_rng(1024)
+    V = 4000
+    w = synth.make_workload(2, B=3, L=2000, ld=2600, d=64, V=V, nohit=0.5, seed=91)
+    tk = synth.make_next_topk(w.tokens, w.lengths, V, 64, seed=91)
+    p = native.make_params(8, 32, 64, 255, 11, float("-inf"), oracle.SUCC_ON_STRICT)
+    eng = native.Engine(w.B, w.ld, w.d, p)
+    eng.run(cuda_i32(w.tokens), cuda_i32(w.lengths), cuda_bf16(w.reps), cuda_bf16(w.query),
+            next_topk=cuda_i32(tk))
+    torch.cuda.synchronize()
+    g = eng.out.to_host()
+    assert g["draft_tokens"].shape[1] == 1024 and int(g["n_nodes"].max()) > 300
+    lg = planted_logits(g["draft_tokens"], g["parents"], g["n_nodes"], V, rng, p_accept=0.9)
+    node_reps = synth.f32_to_bf16_bits(
+        rng.standard_normal(g["draft_tokens"].shape + (w.d,)).astype(np.float32))
+    mem = (w.tokens, w.lengths, w.reps, w.query)
+    gpu, o, o_mem = run_both(lg, g["draft_tokens"], g["parents"], g["n_nodes"], mem,
+                             node_reps, ws=eng.ws)
+    assert_same(gpu, o, o_mem)
+    assert o.n_accept.max() >= 8
+
+
 @pytest.mark.parametrize("N,depth", [(300, 200), (600, 450)])
 def test_deep_chains(N, depth):
     """Chains of N nodes (N x S <= 1024 caps the row splits: at N = 600 one
