@@ -41,6 +41,7 @@ namespace {
 constexpr int kProducerWarp = kConsumers2 / 32;  // warp 8
 constexpr int kBarQ = 15;                        // named barrier for |q|^2
 constexpr int kBarMerge = 14;                    // named barrier for the final merge
+constexpr int kPlanCache = kConsumers2 + 32;     // plan entries kept in shared memory
 
 struct SemArgs {
     SemLaunch p;
@@ -164,6 +165,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     uint64_t *empty = full + kMaxStages2;                      // [NS] stage consumed
     uint64_t *redbar = empty + kMaxStages2;                    // [NS] partial sums written
     volatile int *abort_flag = (volatile int *)(redbar + kMaxStages2);
+    int64_t *s_plan = (int64_t *)(abort_flag + 4);            // [kPlanCache]
 
     pdl_wait_then_release();  // the plan and the lexical outcomes come from the previous kernel
     const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
@@ -171,7 +173,15 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     const int B = a.nvseq ? *a.nvseq : a.B, d = a.d, k = a.k;
     const int ostride = a.out_stride ? a.out_stride : k;
     if (B <= 0) return;
-    const int64_t *plan = args.plan;
+    // A plan of up to kPlanCache entries is read once, one entry per thread
+    // (one memory round trip), and searched in shared memory; a longer one is
+    // searched in global memory.
+    const bool cached = B < kPlanCache;
+    if (cached) {
+        if (t <= B) s_plan[t] = args.plan[t];
+        __syncthreads();
+    }
+    const int64_t *plan = cached ? s_plan : args.plan;
     const int64_t G = plan[B];
     if (G < 0 || G > (int64_t)B * a.ld) {  // never expected: the plan is corrupt
         if (t == 0 && c == 0) atomicOr(ws.dev_status, ADAPLD_DEV_INTERNAL);
@@ -477,7 +487,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
 // partials, the barriers, the abort flag and the merge decision.
 inline size_t semantic_smem(int ns, int stage) {
     return (size_t)ns * stage + (size_t)(ns > 3 ? ns : 3) * 32 * 8 * 4 + 16 * 4 +
-           3 * kMaxStages2 * 8 + 16;
+           3 * kMaxStages2 * 8 + 16 + (size_t)kPlanCache * 8;
 }
 
 template <int MAXC, int SR, bool GATHER>
