@@ -564,6 +564,7 @@ def run_native(args):
         "warmup": max(3, args.warmup), "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": conf,
+        "sequence_steps_per_s": value * w.B,
         "roofline": {"bound": "hbm", "kernel": dom_kernel,
                      "achieved": achieved, "peak": peak, "peak_kind": peak_kind,
                      "unit": "GB/s", "frac": achieved / peak,
