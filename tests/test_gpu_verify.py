@@ -385,3 +385,32 @@ def test_random_trees(case):
                 rng.standard_normal((B, N, d)).astype(np.float32))
     gpu, o, o_mem = run_both(lg, draft, par, nn, mem, node_reps)
     assert_same(gpu, o, o_mem)
+
+
+@pytest.mark.parametrize("case,N,V", [(0, 1024, 16384), (1, 1024, 16392), (2, 300, 128256),
+                                      (3, 700, 40000)])
+def test_random_large_trees(case, N, V):
+    """Large random trees (up to the 1024-node maximum, parents within 8 of
+    their child, so paths run deep) over vocabularies at, just past and far
+    past one 16384-entry row split, tie-heavy logits with planted choices."""
+    rng = np.random.default_rng(9100 + case)
+    B = 2
+    draft = np.full((B, N), -1, np.int32)
+    par = np.full((B, N), -1, np.int32)
+    nn = np.array([N, int(rng.integers(1, N))], np.int32)
+    for b in range(B):
+        for i in range(1, int(nn[b])):
+            par[b, i] = int(rng.integers(max(0, i - 8), i))
+        draft[b, : nn[b]] = rng.integers(0, V, size=int(nn[b]))
+    lg = rng.integers(-3, 3, size=(B, N, V)).astype(np.float32)
+    for b in range(B):
+        kids = {}
+        for c in range(1, int(nn[b])):
+            kids.setdefault(int(par[b, c]), []).append(c)
+        for i, ks in kids.items():
+            if rng.random() < 0.9:  # plant a child with children of its own when there is one
+                inner = [c for c in ks if c in kids] or ks
+                lg[b, i, draft[b, inner[int(rng.integers(len(inner)))]]] = 7.0
+    gpu, o, o_mem = run_both(synth.f32_to_bf16_bits(lg), draft, par, nn)
+    assert_same(gpu, o, o_mem)
+    assert o.n_accept.max() >= 4
