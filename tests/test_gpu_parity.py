@@ -333,7 +333,7 @@ def test_repeated_calls_reuse_workspace():
 
 
 # ------------------------------------------------ randomised configurations
-@pytest.mark.parametrize("case", range(24))
+@pytest.mark.parametrize("case", range(64))
 def test_random_configurations(case):
     """Random parameter combinations (n_max, k, W, D, succ_len, tau, ablation
     flags, ragged lengths, d, the next-token table, the embedding table)

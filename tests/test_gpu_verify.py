@@ -352,7 +352,7 @@ def test_full_size_config5():
     assert o.n_accept.max() >= 1
 
 
-@pytest.mark.parametrize("case", range(16))
+@pytest.mark.parametrize("case", range(48))
 def test_random_trees(case):
     """Random trees (every parent before its child, random fan-out), tie-heavy
     logits with planted choices, random lengths and capacities, the append
