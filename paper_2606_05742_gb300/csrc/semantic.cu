@@ -153,6 +153,7 @@ constexpr int semantic_min_blocks() {
 template <int MAXC, int SR, bool GATHER>
 __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, SR>()))
     semantic_kernel(SemArgs args) {
+    static_assert(32 % SR == 0, "a stage never straddles a 32-row id window");
     const SemLaunch &a = args.p;
     const Workspace &ws = args.ws;
     extern __shared__ __align__(128) uint8_t smem[];
@@ -227,8 +228,15 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             const int jend = (int)(seg_end - plan[p]);
             const uint8_t *base = (const uint8_t *)(a.reps + (int64_t)b * a.ld * d);
             const int32_t *Mb = GATHER ? a.tokens + (int64_t)b * a.ld : nullptr;
-            int win = -1, wtok = 0;
-            for (int j = (int)(g - plan[p]); j < jend; j += SR) {
+            // row ids in windows of 32 (SR divides 32, so a window starts on
+            // a stage); the next window is loaded one window ahead
+            const int jstart = (int)(g - plan[p]);
+            int win = jstart, wtok = 0, wnext = 0;
+            if (GATHER) {
+                wtok = jstart + lane < jend ? Mb[jstart + lane] : 0;
+                wnext = jstart + 32 + lane < jend ? Mb[jstart + 32 + lane] : 0;
+            }
+            for (int j = jstart; j < jend; j += SR) {
                 const int nrows = min(SR, jend - j);
                 const int s = it % NS, r = it / NS;
                 int ok = 1;
@@ -245,9 +253,10 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
                 const uint32_t bytes = (uint32_t)(nrows * row_bytes);
                 uint8_t *dst = ring + (size_t)s * stage_bytes;
                 if (GATHER) {
-                    if (win < 0 || j + nrows > win + 32) {
-                        win = j;
-                        wtok = j + lane < jend ? Mb[j + lane] : 0;
+                    if (j >= win + 32) {
+                        win += 32;
+                        wtok = wnext;
+                        wnext = win + 32 + lane < jend ? Mb[win + 32 + lane] : 0;
                     }
                     int rowtok[SR];
 #pragma unroll
