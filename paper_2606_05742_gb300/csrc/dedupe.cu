@@ -349,26 +349,38 @@ __device__ void expand_one(const ExpandLaunch &a, const Workspace &ws, ExpandSha
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int b = a.vseq_b ? a.vseq_b[p] : p;
     const int64_t row = a.vseq_out ? a.vseq_out[p] : p;
-    if (!a.vseq_b) {
-        if (a.hit_kind && a.hit_kind[b] != ADAPLD_HIT_SEM) return;
-        if (!a.hit_kind && a.active && !a.active[b]) return;
-    }
-    const int len = a.lengths[b];
-    if (len < 2 || (int64_t)len > a.ld) return;
-    const int n = min(a.n_cand[row], a.k);
-    if (n <= 0) return;
     const int k = a.k;
     int32_t *crow = a.cand + row * a.stride;
     float *srow = a.score + row * a.stride;
-    if (t < n) {
-        const int r = crow[t];
-        const int rl = ws.rep_len[b];
-        sh.key[t] = r >= 0 && r < rl - 1 ? ws.rep_tok[(int64_t)b * a.ld + r] : -1;
-        sh.sc[t] = srow[t];
-    }
-    const int p0 = sl * kSlice4, p1 = min(p0 + kSlice4, len - 1);
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
-    for (int i = t; i < p1 - p0; i += kExpandThreads) sh.tok[i] = canon(M[p0 + i], a.vocab);
+    // every load that does not depend on another at once (one memory round
+    // trip): this slice's tokens, positions [p0, p0 + kSlice4) clipped at ld,
+    // copied to shared memory, and the sequence's outcome, length, list
+    // length and candidates
+    const int p0 = sl * kSlice4;
+    const int nld = (int)min((int64_t)kSlice4, a.ld - p0);
+    for (int i = t; i < nld; i += kExpandThreads) cp_async4(sh.tok + i, M + p0 + i);
+    bool skip = false;
+    if (!a.vseq_b) {
+        if (a.hit_kind) skip = a.hit_kind[b] != ADAPLD_HIT_SEM;
+        else if (a.active) skip = !a.active[b];
+    }
+    const int len = a.lengths[b];
+    const int ncr = a.n_cand[row];
+    const int rl = ws.rep_len[b];
+    const int r = t < k ? crow[t] : -1;
+    const float sct = t < k ? srow[t] : 0.f;
+    cp_async_wait_all();  // (also before an exit: the copies target this CTA's memory)
+    if (skip || len < 2 || (int64_t)len > a.ld) return;
+    const int n = min(ncr, k);
+    if (n <= 0) return;
+    if (t < n) {
+        sh.key[t] = r >= 0 && r < rl - 1 ? ws.rep_tok[(int64_t)b * a.ld + r] : -1;
+        sh.sc[t] = sct;
+    }
+    const int p1 = min(p0 + kSlice4, len - 1);
+    __syncthreads();  // the copies of every thread have landed
+    for (int i = t; i < p1 - p0; i += kExpandThreads) sh.tok[i] = canon(sh.tok[i], a.vocab);
     __syncthreads();
 
     // the k most recent positions of each listed token in this slice

@@ -82,17 +82,6 @@ struct TokSrc {
     const TreeSmem *wsm;
 };
 
-// Asynchronous global -> shared copies (no registers held while in flight).
-__device__ __forceinline__ void cp_async16(void *smem, const void *gmem) {
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(smem)), "l"(gmem));
-}
-__device__ __forceinline__ void cp_async4(void *smem, const void *gmem) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_u32(smem)), "l"(gmem));
-}
-__device__ __forceinline__ void cp_async_wait_all() {
-    asm volatile("cp.async.wait_all;" ::: "memory");
-}
-
 // One warp's dot product of a bf16 row in global memory with a bf16 vector
 // in shared memory (both widened exactly to fp32), in batches of U 16-byte
 // chunks per lane: chunk
