@@ -376,8 +376,15 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
  *     call's contents (each call clears what must start at zero), so calls
  *     that overlap on the GPU -- on different streams, or from different host
  *     threads -- race and must not be issued.  Serialise them.
- *   - The device status word of this variant is internal (not readable with
- *     adapld_read_device_status()).
+ *   - The array's device address is cached per device ordinal for the
+ *     process.  A context other than the device's primary context, or a
+ *     primary context re-created after cudaDeviceReset(), is not supported:
+ *     the cached address would belong to the old context.
+ *   - A bounded wait that expires inside the kernel sets ADAPLD_DEV_TIMEOUT in
+ *     the array's status word and leaves that call's outputs invalid (they
+ *     may look like "no candidates").  Read the word with
+ *     adapld_semantic_topk_static_status(); adapld_read_device_status() does
+ *     not apply to this variant.
  */
 #define ADAPLD_STATIC_SCRATCH_BYTES (1u << 20)
 #define ADAPLD_STATIC_MAX_B 1024
@@ -386,6 +393,13 @@ int adapld_semantic_topk_static(const uint16_t *reps, int64_t ld, int32_t d,
                                 const uint8_t *active, int32_t B, int32_t k, float tau,
                                 int32_t *cand, float *score, int32_t *n_cand,
                                 adapld_stream_t stream);
+
+/* Synchronises `stream` and returns in *status (host memory) the ADAPLD_DEV_*
+ * bits raised by the most recent adapld_semantic_topk_static() call on the
+ * current device (0 = none; each call clears the word when it starts).  Pass
+ * the stream of that call.  Allocates nothing.  The paper has no counterpart.
+ * Errors: ADAPLD_ERR_NULL, ADAPLD_ERR_CUDA. */
+int adapld_semantic_topk_static_status(int32_t *status, adapld_stream_t stream);
 
 /*
  * Greedy verification of the draft trees and the append to the memory

@@ -5,51 +5,11 @@
 #include <cstdint>
 #include <cstring>
 
-#include "common.cuh"
+#include "checks.h"
 
 using namespace adapld;
 
 namespace {
-
-bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
-
-int check_params(const adapld_params *p) {
-    if (!p) return ADAPLD_ERR_NULL;
-    if (p->n_max < 1 || p->n_max > 8) return ADAPLD_ERR_NMAX;
-    if (p->k < 1 || p->k > kMaxK) return ADAPLD_ERR_K;
-    if (p->branch_width < 0 || p->branch_width > kMaxW) return ADAPLD_ERR_WIDTH;
-    if (p->draft_len < 1 || p->draft_len > 256) return ADAPLD_ERR_DRAFT_LEN;
-    if (p->succ_len < 1 || p->succ_len > 16) return ADAPLD_ERR_SUCC_LEN;
-    if (std::isnan(p->tau)) return ADAPLD_ERR_TAU;
-    if (adapld_tree_nodes(p) > kMaxNodes) return ADAPLD_ERR_TOO_LARGE;
-    return ADAPLD_OK;
-}
-
-int check_shape(int32_t B, int64_t ld) {
-    if (B < 1 || B > 65535) return ADAPLD_ERR_BATCH;
-    if (ld < 1) return ADAPLD_ERR_LD;
-    if ((int64_t)B * ld >= ((int64_t)1 << 31)) return ADAPLD_ERR_TOO_LARGE;
-    return ADAPLD_OK;
-}
-
-int check_dim(int32_t d) {
-    if (d < 8 || d > 16384 || (d % 8) != 0) return ADAPLD_ERR_DIM;
-    return ADAPLD_OK;
-}
-
-int check_ws(void *ws, size_t ws_bytes, int32_t B, int64_t ld, int32_t W) {
-    if (!ws) return ADAPLD_ERR_WORKSPACE;
-    if (!aligned16(ws)) return ADAPLD_ERR_ALIGN;
-    if (ws_bytes < layout_workspace(nullptr, B, ld, W).total_bytes) return ADAPLD_ERR_WORKSPACE;
-    return ADAPLD_OK;
-}
-
-int check_emb(const adapld_embeddings *e) {
-    if (!e) return ADAPLD_OK;
-    if (!e->table || !aligned16(e->table) || e->vocab < 1) return ADAPLD_ERR_EMBEDDINGS;
-    if (e->dim < 8 || e->dim > 16384 || (e->dim % 8) != 0) return ADAPLD_ERR_EMBEDDINGS;
-    return ADAPLD_OK;
-}
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA; }
 
@@ -58,11 +18,27 @@ int record(void *ev, cudaStream_t s) {
     return cuda_status(cudaEventRecord((cudaEvent_t)ev, s));
 }
 
-#define ADAPLD_TRY(x)                   \
-    do {                                \
-        int rc_ = (x);                  \
-        if (rc_ != ADAPLD_OK) return rc_; \
-    } while (0)
+// Every argument check of a step, on device pointers and sizes only: a step
+// fails here, before anything is enqueued, or not at all on the host side.
+int check_step_args(const int32_t *tokens, int64_t ld, const int32_t *lengths,
+                    const uint16_t *reps, int32_t d, const uint16_t *query,
+                    const int32_t *next_topk, int32_t Kn, int32_t B, const adapld_params *p,
+                    const adapld_step_out *out, void *ws, size_t ws_bytes,
+                    const adapld_embeddings *emb) {
+    if (!tokens || !lengths || !reps || !query || !out) return ADAPLD_ERR_NULL;
+    if (!out->hit_kind || !out->match_n || !out->cand || !out->score || !out->n_cand)
+        return ADAPLD_ERR_NULL;
+    const adapld_tree_out &to = out->tree;
+    if (!to.anchor || !to.draft_tokens || !to.parents || !to.positions || !to.mask || !to.n_nodes)
+        return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_params(p));
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_dim(d));
+    if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
+    if (next_topk && (Kn < 1 || Kn > kMaxW)) return ADAPLD_ERR_TOPK_TABLE;
+    ADAPLD_TRY(check_emb(emb));
+    return check_ws(ws, ws_bytes, B, ld, p->branch_width);
+}
 
 }  // namespace
 
@@ -111,7 +87,7 @@ int adapld_lexical_match(const int32_t *tokens, int64_t ld, const int32_t *lengt
     if (!tokens || !lengths || !hit_kind || !match_n || !cand || !n_cand) return ADAPLD_ERR_NULL;
     ADAPLD_TRY(check_shape(B, ld));
     if (n_max < 1 || n_max > 8) return ADAPLD_ERR_NMAX;
-    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
+    ADAPLD_TRY(check_k(k));
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, 1);
@@ -129,8 +105,8 @@ int adapld_semantic_topk(const uint16_t *reps, int64_t ld, int32_t d, const uint
     ADAPLD_TRY(check_shape(B, ld));
     ADAPLD_TRY(check_dim(d));
     if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
-    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
-    if (std::isnan(tau)) return ADAPLD_ERR_TAU;
+    ADAPLD_TRY(check_k(k));
+    ADAPLD_TRY(check_tau(tau));
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, 1);
@@ -147,8 +123,8 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
     if (!tokens || !lengths || !emb || !cand || !score || !n_cand) return ADAPLD_ERR_NULL;
     ADAPLD_TRY(check_shape(B, ld));
     ADAPLD_TRY(check_emb(emb));
-    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
-    if (std::isnan(tau)) return ADAPLD_ERR_TAU;
+    ADAPLD_TRY(check_k(k));
+    ADAPLD_TRY(check_tau(tau));
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, 1);
@@ -205,19 +181,9 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
                    const adapld_step_out *out, void *ws, size_t ws_bytes,
                    const adapld_embeddings *emb, const adapld_step_events *ev,
                    adapld_stream_t stream) {
-    if (!tokens || !lengths || !reps || !query || !out) return ADAPLD_ERR_NULL;
-    if (!out->hit_kind || !out->match_n || !out->cand || !out->score || !out->n_cand)
-        return ADAPLD_ERR_NULL;
+    ADAPLD_TRY(check_step_args(tokens, ld, lengths, reps, d, query, next_topk, Kn, B, p, out, ws,
+                               ws_bytes, emb));
     const adapld_tree_out &to = out->tree;
-    if (!to.anchor || !to.draft_tokens || !to.parents || !to.positions || !to.mask || !to.n_nodes)
-        return ADAPLD_ERR_NULL;
-    ADAPLD_TRY(check_params(p));
-    ADAPLD_TRY(check_shape(B, ld));
-    ADAPLD_TRY(check_dim(d));
-    if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
-    if (next_topk && (Kn < 1 || Kn > kMaxW)) return ADAPLD_ERR_TOPK_TABLE;
-    ADAPLD_TRY(check_emb(emb));
-    ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, p->branch_width));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     const bool semantic = !(p->flags & ADAPLD_NO_SEMANTIC);
@@ -285,12 +251,11 @@ int adapld_step_from_host(const int32_t *tokens_h, int64_t ld, const int32_t *le
                           uint16_t *reps_d, uint16_t *query_d, const adapld_step_out *out_d,
                           const adapld_step_out *out_h, void *ws, size_t ws_bytes,
                           adapld_stream_t stream) {
-    if (!tokens_h || !lengths_h || !reps_h || !query_h || !tokens_d || !lengths_d || !reps_d ||
-        !query_d || !out_d || !out_h)
-        return ADAPLD_ERR_NULL;
-    ADAPLD_TRY(check_params(p));
-    ADAPLD_TRY(check_shape(B, ld));
-    ADAPLD_TRY(check_dim(d));
+    if (!tokens_h || !lengths_h || !reps_h || !query_h || !out_h) return ADAPLD_ERR_NULL;
+    // the step's own checks on the device buffers, before the first copy is
+    // enqueued
+    ADAPLD_TRY(check_step_args(tokens_d, ld, lengths_d, reps_d, d, query_d, nullptr, 0, B, p,
+                               out_d, ws, ws_bytes, nullptr));
     cudaStream_t s = (cudaStream_t)stream;
     auto h2d = [&](void *dst, const void *src, size_t bytes) {
         return cuda_status(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, s));

@@ -11,7 +11,7 @@
 // or allocating library routine.
 #include <mutex>
 
-#include "common.cuh"
+#include "checks.h"
 
 using namespace adapld;
 
@@ -68,14 +68,13 @@ extern "C" int adapld_semantic_topk_static(const uint16_t *reps, int64_t ld, int
                                            int32_t *cand, float *score, int32_t *n_cand,
                                            adapld_stream_t stream) {
     if (!reps || !query || !lengths || !cand || !score || !n_cand) return ADAPLD_ERR_NULL;
-    if (B < 1) return ADAPLD_ERR_BATCH;
     if (B > ADAPLD_STATIC_MAX_B) return ADAPLD_ERR_STATIC_LIMIT;
-    if (ld < 1) return ADAPLD_ERR_LD;
-    if ((int64_t)B * ld >= ((int64_t)1 << 31)) return ADAPLD_ERR_TOO_LARGE;
-    if (d < 8 || d > 16384 || (d % 8) != 0) return ADAPLD_ERR_DIM;
-    if ((((uintptr_t)reps) & 15u) || (((uintptr_t)query) & 15u)) return ADAPLD_ERR_ALIGN;
-    if (k < 1 || k > kMaxK) return ADAPLD_ERR_K;
-    if (tau != tau) return ADAPLD_ERR_TAU;
+    // the same checks, in the same order, as adapld_semantic_topk()
+    ADAPLD_TRY(check_shape(B, ld));
+    ADAPLD_TRY(check_dim(d));
+    if (!aligned16(reps) || !aligned16(query)) return ADAPLD_ERR_ALIGN;
+    ADAPLD_TRY(check_k(k));
+    ADAPLD_TRY(check_tau(tau));
     void *base = nullptr;
     const int rc = scratch_address(&base);
     if (rc != ADAPLD_OK) return rc;
@@ -87,4 +86,16 @@ extern "C" int adapld_semantic_topk_static(const uint16_t *reps, int64_t ld, int
     SemLaunch a{reps, ld, d, query, lengths, active, B, k, tau, cand, score, n_cand,
                 nullptr, false};
     return launch_semantic(a, w, s) == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA;
+}
+
+extern "C" int adapld_semantic_topk_static_status(int32_t *status, adapld_stream_t stream) {
+    if (!status) return ADAPLD_ERR_NULL;
+    void *base = nullptr;
+    const int rc = scratch_address(&base);
+    if (rc != ADAPLD_OK) return rc;
+    // the status word is the first int32 of the array (static_layout)
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaMemcpyAsync(status, base, sizeof(int32_t), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return ADAPLD_ERR_CUDA;
+    return cudaStreamSynchronize(s) == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA;
 }

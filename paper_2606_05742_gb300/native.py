@@ -36,9 +36,12 @@ EXPORTED = [
     "adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
     "adapld_step", "adapld_step_ex", "adapld_read_device_status",
     "adapld_semantic_topk_static", "adapld_embedding_topk", "adapld_accept_greedy",
-    "adapld_step_from_host",
+    "adapld_step_from_host", "adapld_semantic_topk_static_status",
 ]
 STATIC_MAX_B = 1024
+ERR_NULL = -1
+ERR_ALIGN = -8
+ERR_WORKSPACE = -9
 ERR_STATIC_LIMIT = -15
 
 
@@ -122,6 +125,7 @@ def load() -> ctypes.CDLL:
         lib.adapld_read_device_status.argtypes = [P, P, P]
         lib.adapld_semantic_topk_static.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P,
                                                     P, P]
+        lib.adapld_semantic_topk_static_status.argtypes = [P, P]
         lib.adapld_accept_greedy.argtypes = [P, i32, P, P, P, i32, i32, P, P, P, P, i64, P, P,
                                              P, i32, P, P, P, sz, P]
         lib.adapld_step_from_host.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, P, P, P,
@@ -129,7 +133,8 @@ def load() -> ctypes.CDLL:
         for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
                   "adapld_step", "adapld_step_ex", "adapld_read_device_status",
                   "adapld_semantic_topk_static", "adapld_embedding_topk",
-                  "adapld_accept_greedy", "adapld_step_from_host"):
+                  "adapld_accept_greedy", "adapld_step_from_host",
+                  "adapld_semantic_topk_static_status"):
             getattr(lib, f).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -191,6 +196,15 @@ def semantic_topk_static(reps, query, lengths, k: int, tau: float, cand, score, 
                                             _ptr(active), B, k, tau, _ptr(cand), _ptr(score),
                                             _ptr(n_cand), _stream(stream))
     _check(rc, "adapld_semantic_topk_static")
+
+
+def semantic_topk_static_status(stream=None) -> int:
+    """ADAPLD_DEV_* bits of the last adapld_semantic_topk_static call on the
+    current device (synchronises the stream)."""
+    st = ctypes.c_int32(-1)
+    _check(load().adapld_semantic_topk_static_status(ctypes.byref(st), _stream(stream)),
+           "adapld_semantic_topk_static_status")
+    return st.value
 
 
 def _tree_out(anchor, draft_tokens, parents, positions, mask, n_nodes, stats=None) -> TreeOut:

@@ -58,6 +58,15 @@ class Report:
         return (f"exact={self.exact} tie_resolved={self.tie_resolved} "
                 f"max_score_err={self.max_score_err:.3g}")
 
+    @staticmethod
+    def merge(reports) -> "Report":
+        out = Report()
+        for r in reports:
+            out.exact += r.exact
+            out.tie_resolved += r.tie_resolved
+            out.max_score_err = max(out.max_score_err, r.max_score_err)
+        return out
+
 
 def check_semantic_list(gc, gs, gn, s_all, eps, k, tau, rep: Report, where=""):
     """Validates a GPU semantic top-k list against every fp64 score."""

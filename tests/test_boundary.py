@@ -207,6 +207,33 @@ def test_step_from_host_argument_errors(lib):
     bad = list(args)
     bad[4] = 12
     assert lib.adapld_step_from_host(*bad) == -7
+    # the step's own checks on the device buffers also run before the first
+    # copy: without a GPU an enqueued copy would fail with ADAPLD_ERR_CUDA
+    # (-20), so each of these codes shows that nothing was enqueued
+    bad = list(args)
+    bad[14] = None                                   # no workspace
+    assert lib.adapld_step_from_host(*bad) == -9
+    bad = list(args)
+    bad[15] = 64                                     # workspace too small
+    assert lib.adapld_step_from_host(*bad) == -9
+    bad = list(args)
+    bad[14] = FAKE + 4                               # misaligned workspace
+    assert lib.adapld_step_from_host(*bad) == -8
+    bad = list(args)
+    bad[10] = FAKE + 2                               # misaligned device reps
+    assert lib.adapld_step_from_host(*bad) == -8
+    bad = list(args)
+    bad[11] = FAKE + 8                               # misaligned device query
+    assert lib.adapld_step_from_host(*bad) == -8
+    so_missing = native.StepOut(FAKE, FAKE, None, FAKE, FAKE, None,
+                                native.TreeOut(FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None))
+    bad = list(args)
+    bad[12] = ctypes.byref(so_missing)               # a required device output
+    assert lib.adapld_step_from_host(*bad) == -1
+    bad = list(args)
+    p_bad = native.make_params(3, 40, 2, 8)          # k out of range
+    bad[7] = ctypes.byref(p_bad)
+    assert lib.adapld_step_from_host(*bad) == -4
 
 
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
