@@ -93,7 +93,7 @@ int adapld_lexical_match(const int32_t *tokens, int64_t ld, const int32_t *lengt
     Workspace w = layout_workspace(ws, B, ld, 1);
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
     LexLaunch a{tokens, ld, lengths, B, n_max, k, hit_kind, match_n, cand, n_cand,
-                nullptr, nullptr, nullptr, false};
+                nullptr, nullptr, nullptr};
     return cuda_status(launch_lexical(a, w, s));
 }
 
@@ -187,21 +187,28 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     const bool semantic = !(p->flags & ADAPLD_NO_SEMANTIC);
-    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
+    // (the workspace counters are zeroed by the lexical kernel)
     if (emb) ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
 
     ADAPLD_TRY(record(ev ? ev->lexical_begin : nullptr, s));
-    // with a token-embedding table the plan is built over the distinct-token
-    // lists instead
     LexLaunch la{tokens, ld, lengths, B, p->n_max, p->k, out->hit_kind, out->match_n, out->cand,
-                 out->n_cand, out->score, out->status, to.stats, semantic && !emb};
+                 out->n_cand, out->score, out->status, to.stats};
+    la.zero = w.dev_status;
+    la.zero_words = w.counters_bytes / sizeof(int32_t);
     ADAPLD_TRY(cuda_status(launch_lexical(la, w, s)));
+    // the semantic plan: derived by the semantic kernel itself for small
+    // batches, else by one CTA from the outcomes (with a token-embedding
+    // table it is built over the distinct-token lists instead)
+    const bool small_plan = B < kPlanInKernelB;
+    if (semantic && !emb && !small_plan)
+        ADAPLD_TRY(cuda_status(launch_outcome_plan(lengths, ld, B, out->hit_kind, w, s)));
     ADAPLD_TRY(record(ev ? ev->lexical_end : nullptr, s));
 
     if (semantic) {
         ADAPLD_TRY(record(ev ? ev->semantic_begin : nullptr, s));
         SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
                      out->n_cand, out->hit_kind, true};
+        sa.plan_from_outcome = !emb && small_plan;
         if (emb) {  // Eq. 4 over token embeddings, scored once per distinct token
             // lists for the fallback sequences, and for lexical hits too when
             // those draft successors (their backoff needs them)

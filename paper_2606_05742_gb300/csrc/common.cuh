@@ -12,15 +12,19 @@ namespace adapld {
 constexpr int kMaxK = 32;          // candidates per list (one per warp lane)
 constexpr int kMaxW = 64;          // branch width
 constexpr int kMaxNodes = 1024;    // draft-tree node slots
-constexpr int kChunk1 = 4096;      // lexical scan: positions per CTA
+constexpr int kChunk1 = 4096;      // distinct-token lists: positions per CTA
 constexpr int kThreads1 = 256;
+constexpr int kChunkL = 8192;      // lexical scan: positions per chunk
+constexpr int kThreadsL = 512;
+constexpr int kMaxClusterL = 8;    // lexical scan: CTAs per sequence (one portable cluster)
+constexpr int kWideClusterL = 16;  // ... when the whole grid fits one CTA per SM
+constexpr int kPlanInKernelB = 288;  // below this B the semantic kernel derives its plan
 constexpr int kSlice4 = 8192;      // successor scan: positions per CTA
 constexpr int kThreads4 = 512;
 constexpr int kMaxGrid2 = 1024;    // semantic kernel: CTAs at most
 constexpr int kConsumers2 = 256;   // semantic kernel: consumer threads (8 warps)
 constexpr int kMaxStages2 = 8;
 constexpr int kSlotInts = 68;      // partial top-k slot: count, 32 ids, 32 scores (+pad)
-constexpr int kPart1Ints = 2 + kMaxK;
 constexpr int kPart4Ints = 1 + kMaxK;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded waits: 2 s
 
@@ -29,8 +33,6 @@ constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded waits: 2 
 // fully rewrites before reading.
 struct Workspace {
     int32_t *dev_status;     // [1]  ADAPLD_DEV_* bits
-    int32_t *global_ticket;  // [1]  lexical kernel: CTAs done with their sequence
-    int32_t *ticket1;        // [B]  lexical kernel: chunks done per sequence
     int32_t *done2;          // [B]  semantic kernel: CTAs done per sequence
     int32_t *ticket4;        // [B]  successor scan: slices done per sequence
     int32_t *ticket5;        // [B]  tree kernel: CTAs done per sequence
@@ -40,7 +42,6 @@ struct Workspace {
     int32_t *rticket;        // [B]  distinct-token lists: chunks counted per sequence
     int32_t *xticket;        // [B]  expansion of the fallback lists: slices done
     int32_t *xticket2;       // [B*W] expansion of the backoff lists: slices done
-    int32_t *part1;          // [B][C1][kPart1Ints]  per-chunk lexical results
     int64_t *plan;           // [B+1] prefix sums of semantic rows per sequence
     int32_t *slots2;         // [B + kMaxGrid2][kSlotInts] partial top-k lists
     int32_t *part4;          // [B][S4][W][kPart4Ints] per-slice successor lists
@@ -103,14 +104,12 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         return r;
     };
     const size_t BW = (size_t)B * w.W;
-    w.counters_bytes = sizeof(int32_t) * (4 + 6 * (size_t)B + 2 * BW);
+    w.counters_bytes = sizeof(int32_t) * (4 + 5 * (size_t)B + 2 * BW);
     w.dev_status = (int32_t *)take(w.counters_bytes);
     if (p) {
-        w.global_ticket = w.dev_status + 1;
-        w.npairs = w.dev_status + 2;
-        w.gticket_rep = w.dev_status + 3;
-        w.ticket1 = w.dev_status + 4;
-        w.done2 = w.ticket1 + B;
+        w.npairs = w.dev_status + 1;
+        w.gticket_rep = w.dev_status + 2;
+        w.done2 = w.dev_status + 4;
         w.ticket4 = w.done2 + B;
         w.ticket5 = w.ticket4 + B;
         w.done3 = w.ticket5 + B;
@@ -118,7 +117,6 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
         w.xticket = w.rticket + B;
         w.xticket2 = w.xticket + B;
     }
-    w.part1 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1 * kPart1Ints);
     w.plan = (int64_t *)take(sizeof(int64_t) * ((size_t)B + 1));
     w.slots2 = (int32_t *)take(sizeof(int32_t) * ((size_t)B + kMaxGrid2) * kSlotInts);
     w.part4 = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.S4 * w.W * kPart4Ints);
@@ -260,6 +258,34 @@ __device__ __forceinline__ void cp_async4(void *smem, const void *gmem) {
 }
 __device__ __forceinline__ void cp_async_wait_all() {
     asm volatile("cp.async.wait_all;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+    asm volatile("cp.async.commit_group;" ::: "memory");
+}
+template <int N>
+__device__ __forceinline__ void cp_async_wait_group() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
+// Thread-block clusters: a barrier over every thread of the cluster (release
+// of this thread's earlier writes, acquire of the others'), and a 32-bit load
+// from the shared memory of CTA `rank` of the cluster at the offset of
+// `local` in this CTA's shared memory.
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// The same barrier for a thread with no shared-memory writes to publish.
+__device__ __forceinline__ void cluster_sync_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ int ld_cluster_i32(const int *local, uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+    int v;
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(remote) : "memory");
+    return v;
 }
 
 __device__ __forceinline__ uint4 ldg_nc_v4(const void *p) {
@@ -452,6 +478,9 @@ cudaError_t launch_dependent(void (*kern)(KArgs...), dim3 grid, dim3 block, size
     return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
 
+// Streaming multiprocessors of the current device (0 on error).
+int device_sms();
+
 struct LexLaunch {
     const int32_t *tokens;
     int64_t ld;
@@ -461,9 +490,21 @@ struct LexLaunch {
     float *score;            // optional: zeroed for every sequence
     int32_t *status;         // optional
     int32_t *stats;          // optional: zeroed
-    bool build_plan;         // also build the semantic plan (step path)
+    // optional: words the kernel zeroes (the workspace counters of the later
+    // kernels of a step, which then needs no memset); the lexical kernel
+    // itself uses no counters
+    int32_t *zero = nullptr;
+    size_t zero_words = 0;
 };
+// Launched as a programmatic dependent of the previous kernel in the stream
+// (it waits for it before touching memory).
 cudaError_t launch_lexical(const LexLaunch &a, const Workspace &ws, cudaStream_t s);
+
+// Semantic plan from the lexical outcomes, for batches too large for the
+// semantic kernel to derive it (B >= kPlanInKernelB): one CTA, launched as a
+// programmatic dependent of the lexical kernel.
+cudaError_t launch_outcome_plan(const int32_t *lengths, int64_t ld, int32_t B,
+                                const int32_t *hit_kind, const Workspace &ws, cudaStream_t s);
 
 // Semantic work plan for the standalone semantic entry point (one CTA):
 // ws.plan[b] = rows of earlier selected sequences (selection: active == NULL
@@ -500,6 +541,9 @@ struct SemLaunch {
     const int32_t *nvseq = nullptr;
     int32_t out_stride = 0;  // 0: k
     int32_t *status = nullptr;  // per real sequence ADAPLD_SEQ_* bits (nullable)
+    // step path, B < kPlanInKernelB: the kernel derives the plan from
+    // hit_kind and lengths (the lexical kernel wrote no plan)
+    bool plan_from_outcome = false;
 };
 cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_t s);
 

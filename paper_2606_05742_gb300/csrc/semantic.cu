@@ -42,6 +42,7 @@ constexpr int kProducerWarp = kConsumers2 / 32;  // warp 8
 constexpr int kBarQ = 15;                        // named barrier for |q|^2
 constexpr int kBarMerge = 14;                    // named barrier for the final merge
 constexpr int kPlanCache = kConsumers2 + 32;     // plan entries kept in shared memory
+static_assert(kPlanCache == kPlanInKernelB, "the lexical kernel leaves small plans to this one");
 
 struct SemArgs {
     SemLaunch p;
@@ -176,9 +177,25 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
     if (B <= 0) return;
     // A plan of up to kPlanCache entries is read once, one entry per thread
     // (one memory round trip), and searched in shared memory; a longer one is
-    // searched in global memory.
+    // searched in global memory.  On the step path with B < kPlanCache the
+    // CTA derives the plan itself from the lexical outcomes and the lengths
+    // (one round trip and a block scan): a sequence without a lexical hit
+    // and with a valid length contributes its len-1 rows.  hit_kind may
+    // already read SEM or NONE for a sequence another CTA has finished; both
+    // mean "no lexical hit", so every CTA derives the same plan.
     const bool cached = B < kPlanCache;
-    if (cached) {
+    if (a.plan_from_outcome) {
+        int64_t rows = 0;
+        if (t < B) {
+            const int len = a.lengths[t];
+            if (a.hit_kind[t] != ADAPLD_HIT_LEX && len >= 1 && (int64_t)len <= a.ld) rows = len - 1;
+        }
+        int64_t total;
+        const int64_t ex = block_exclusive_scan(rows, &total, (int64_t *)red);
+        if (t < B) s_plan[t] = ex;
+        if (t == 0) s_plan[B] = total;
+        __syncthreads();
+    } else if (cached) {
         if (t <= B) s_plan[t] = args.plan[t];
         __syncthreads();
     }
@@ -563,7 +580,7 @@ SemTuning semantic_tuning() {
 
 }  // namespace
 
-int semantic_sms() {
+int device_sms() {
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
@@ -576,7 +593,7 @@ cudaError_t launch_semantic(const SemLaunch &a, const Workspace &ws, cudaStream_
                                     a.n_cand, ws, s);
         if (e != cudaSuccess) return e;
     }
-    const int sms = semantic_sms();
+    const int sms = device_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
     const SemTuning tun = semantic_tuning();
     SemArgs args{a, ws, 0, 0, kWaitLimitNs, 0, ws.plan, ws.done2, ws.slots2};

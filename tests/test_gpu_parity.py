@@ -448,6 +448,20 @@ def test_long_history_many_chunks():
         check_all(w, run_step(w, P), P)
 
 
+@pytest.mark.parametrize("xmax", ["1", "2", "3", "8", "16"])
+def test_lexical_cluster_shapes(xmax, monkeypatch):
+    """Every cluster width of the lexical kernel (CTAs per sequence, hence
+    chunks per CTA from 1 to 9) gives the oracle's outcome: histories of
+    several 8192-position chunks, rows that start off a 16-byte boundary
+    (odd ld), ragged lengths, a small vocabulary (many hits) and n_max = 8."""
+    monkeypatch.setenv("ADAPLD_LEXICAL_CLUSTER", xmax)
+    w = synth.make_workload(5, B=5, L=70001, d=8, V=64, nohit=0.2, seed=43,
+                            lengths=[70001, 8193, 16385, 2, 40000])
+    for n_max in (1, 8):
+        P = P_of(w, tau=NEG_INF, n_max=n_max)
+        check_all(w, run_step(w, P), P)
+
+
 def test_semantic_wait_timeout_is_reported_and_recoverable(monkeypatch):
     """Failure path without a fault: with the test switch the semantic
     kernel's producer issues no copy, so every bounded wait expires; the call
@@ -652,7 +666,7 @@ def test_step_from_host_rejects_before_copying():
         assert (r == 7).all()
     assert call() == 0                               # the same buffers, valid call
     torch.cuda.synchronize()
-    assert (dev[0].cpu() == tok_h).all()
+    assert (dev[0].cpu() == tok_h.flatten()).all()
 
 
 def test_end_to_end_from_host_matches_device_path():
