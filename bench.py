@@ -168,113 +168,134 @@ class ClockSampler:
 
 
 # --------------------------------------------------------- oracle timing
-class OracleSample:
-    """A bounded sample of the workload for timing the CPU oracle: one forced
-    lexical miss and one lexical-hit sequence, truncated to ``rows`` positions
-    and generated on the host.  The oracle's cost is linear in the positions,
-    so a full step is extrapolated as n_miss * t_miss * (L-1)/(rows-1) +
-    n_hit * t_hit * L/rows, with n_miss the lexical misses (the sequences
-    that run the semantic fallback) of the timed workload's own histories
-    (generated from the same seed; the oracle's lexical step counts them)."""
+class OracleRun:
+    """The CPU oracle timed on the benchmark's own workload: every sequence of
+    the batch at full length, the same bytes the GPU step reads (host copies
+    of the device inputs), one sequence per task on a pool of host threads
+    (the C oracle runs outside the GIL).  One step = the oracle's whole
+    draft-construction step over the batch."""
 
-    def __init__(self, cfg_id: int, seed: int, rows: int, batch=None):
-        import oracle
-        from paper_2606_05742_gb300 import synth
-        c = synth.CONFIGS[cfg_id]
-        self.L = c["L"]
-        B = c["B"] if batch is None else batch
-        self.rows = min(rows, self.L)
-        self.w = synth.make_workload(cfg_id, B=2, L=self.rows, nohit=0.5, seed=seed + 1000)
-        self.miss = int(self.w.forced[0])
-        self.hit = 1 - self.miss
-        tokens, lengths, _ = synth.make_tokens(cfg_id, B=B, seed=seed)
-        self.n_miss = sum(
-            1 for b in range(B)
-            if oracle.lexical(tokens[b, : lengths[b]], c["n_max"], c["k"])[0] == 0)
-        self.n_hit = B - self.n_miss
-        self.desc = (f"oracle (1 thread) on 1 forced-miss + 1 lexical-hit sequence of config "
-                     f"{cfg_id} truncated to {self.rows} positions (d={c['d']}), extrapolated "
-                     f"linearly to {self.n_miss} misses + {self.n_hit} hits of length {self.L}")
+    def __init__(self, tokens, lengths, reps, query, n_max, k, W, D, succ_len, tau, flags=0):
+        self.args = (tokens, lengths, reps, query)
+        self.params = (n_max, k, W, D, succ_len, tau, flags)
+        self.B = tokens.shape[0]
+        self.hit = None
 
-    def rate(self) -> float:
-        import oracle
-        w = self.w
-        t = {}
-        for b in (self.miss, self.hit):
-            s = time.perf_counter()
-            oracle.step(w.tokens[b:b + 1], w.lengths[b:b + 1], w.reps[b:b + 1],
-                        w.query[b:b + 1], w.n_max, w.k, w.W, w.D, w.succ_len, w.tau)
-            t[b] = time.perf_counter() - s
-        est = (self.n_miss * t[self.miss] * (self.L - 1) / (self.rows - 1)
-               + self.n_hit * t[self.hit] * self.L / self.rows)
-        return 1.0 / est
-
-    def rate_parallel(self, threads: int) -> float:
-        """The same oracle over a whole batch of truncated sequences (n_miss
-        copies of the miss, n_hit of the hit), one sequence per task on a
-        pool of ``threads`` host threads (the C oracle runs outside the GIL),
-        wall time extrapolated linearly to full length."""
+    def step(self, threads: int) -> float:
+        """Runs one step on `threads` host threads; returns its wall time (s)."""
         import concurrent.futures as cf
 
         import oracle
-        w = self.w
-        seqs = [self.miss] * self.n_miss + [self.hit] * self.n_hit
+        tokens, lengths, reps, query = self.args
+        n_max, k, W, D, succ_len, tau, flags = self.params
+        hit = np.zeros(self.B, np.int32)
 
         def one(b):
-            oracle.step(w.tokens[b:b + 1], w.lengths[b:b + 1], w.reps[b:b + 1],
-                        w.query[b:b + 1], w.n_max, w.k, w.W, w.D, w.succ_len, w.tau)
+            r = oracle.step(tokens[b:b + 1], lengths[b:b + 1], reps[b:b + 1], query[b:b + 1],
+                            n_max, k, W, D, succ_len, tau, flags)
+            hit[b] = r.hit[0]
 
-        with cf.ThreadPoolExecutor(max_workers=threads) as ex:
-            s = time.perf_counter()
-            list(ex.map(one, seqs))
-            wall = time.perf_counter() - s
-        return 1.0 / (wall * (self.L - 1) / (self.rows - 1))
+        s = time.perf_counter()
+        if threads == 1:
+            for b in range(self.B):
+                one(b)
+        else:
+            with cf.ThreadPoolExecutor(max_workers=threads) as ex:
+                list(ex.map(one, range(self.B)))
+        wall = time.perf_counter() - s
+        self.hit = hit
+        return wall
 
-    def parallel_desc(self, threads: int) -> str:
+    def outcomes(self) -> dict:
+        h = self.hit
+        return {"lexical": int((h == 1).sum()), "semantic": int((h == 2).sum()),
+                "none": int((h == 0).sum())}
+
+    def desc(self, threads: int, cfg_id: int) -> str:
         plural = "s" if threads > 1 else ""
-        return self.desc.replace("oracle (1 thread)", f"oracle ({threads} thread{plural}, one "
-                                 "sequence per task)") + " (wall time of the batch)"
+        return (f"oracle (plain C, fp64) on {threads} host thread{plural}, one sequence per "
+                f"task: whole steps over the full config-{cfg_id} batch ({self.B} sequences, "
+                "full length, the GPU step's own inputs copied to the host)")
 
 
 def host_threads(batch: int) -> int:
     return max(1, min(batch, os.cpu_count() or 1))
 
 
+def host_copy(w):
+    """numpy copies of a device workload's inputs (bf16 as uint16 bits)."""
+    import torch
+    tok = w.tokens.cpu().numpy()
+    ln = w.lengths.cpu().numpy()
+    reps = w.reps.view(torch.int16).cpu().numpy().view(np.uint16)
+    q = w.query.view(torch.int16).cpu().numpy().view(np.uint16)
+    return tok, ln, reps, q
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    sample = OracleSample(args.config, args.seed, rows=4096, batch=args.batch)
-    threads = host_threads(sample.n_miss + sample.n_hit)
+    from paper_2606_05742_gb300 import synth
+    import torch
+    flags = parse_flags(args.flags)
+    if args.embeddings:
+        print(json.dumps({"impl": "reference", "unavailable": "the reference arm times the "
+                          "single-cache step only"}), flush=True)
+        return
+    if torch.cuda.is_available():  # the native arm's bytes, drawn on the GPU, copied here
+        w = synth.make_workload(args.config, device="cuda", seed=args.seed, B=args.batch)
+        tok, ln, reps, q = host_copy(w)
+        del w
+        torch.cuda.empty_cache()
+    else:
+        w = synth.make_workload(args.config, seed=args.seed, B=args.batch)
+        tok, ln, reps, q = w.tokens, w.lengths, w.reps, w.query
+    c = synth.CONFIGS[args.config]
+    run = OracleRun(tok, ln, reps, q, c["n_max"], c["k"], c["W"], c["D"], 1, synth.TAU, flags)
+    threads = host_threads(run.B)
     for _ in range(args.warmup):
-        sample.rate_parallel(threads)
-    vals = []
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        vals.append(sample.rate_parallel(threads))
-        if time.perf_counter() - t0 > 150:
+        run.step(threads)
+    walls = []
+    for _ in range(args.steps):  # whole steps, bounded by wall time
+        walls.append(run.step(threads))
+        if sum(walls) > 120:
             break
-    desc = sample.parallel_desc(threads)
-    value = statistics.median(vals)
+    total = sum(walls)
+    value = len(walls) / total
+    conf = workload_config(args.config, args.batch, flags, None)
+    conf["outcomes"] = run.outcomes()
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
-        "n_gpus": args.gpus, "steps": len(vals), "warmup": args.warmup,
-        "ms_per_step": 1000.0 / value, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": workload_config(args.config),
+        "n_gpus": args.gpus, "steps": len(walls), "warmup": args.warmup,
+        "ms_per_step": 1000.0 * total / len(walls), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": conf, "parallelism": "host threads (rank 0 only)", "accumulate": "fp64",
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
-                         "sample": desc},
+                         "sample": run.desc(threads, args.config)},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
 
 
-def workload_config(cfg_id):
+def workload_config(cfg_id, batch=None, flags=0, emb_shape=None):
+    """The workload as both arms describe it (the same object for the same
+    arguments)."""
     from paper_2606_05742_gb300 import synth
     c = synth.CONFIGS[cfg_id]
-    return {"workload": f"config{cfg_id}: {synth.describe(cfg_id)} tau={synth.TAU}",
-            "B": c["B"], "L": c["L"], "d": c["d"], "global_batch": c["B"],
+    B = c["B"] if batch is None else batch
+    conf = {"workload": f"config{cfg_id}: {synth.describe(cfg_id)} tau={synth.TAU}",
+            "B": B, "L": c["L"], "d": c["d"], "global_batch": B,
             "l2": "inputs larger than L2 (no flush needed)"}
+    if emb_shape is not None:
+        conf["workload"] += (f" + token-embedding fallback ({emb_shape[0]} x {emb_shape[1]} "
+                             "table; two-representation mode)")
+    if flags:
+        conf["workload"] += f" ablation flags {flags}"
+        conf["flags"] = flags
+    if batch is not None:
+        conf["workload"] += f" (resized: B={B})"
+    return conf
 
 
 # ---------------------------------------------------------- native arm
@@ -291,18 +312,26 @@ def parse_flags(text):
     return flags
 
 
-def step_launches(flags, W, emb):
+def step_launches(flags, W, emb, k=32, B=8, ld=131072):
     """Kernels one step launches (mirrors the launch sequence of adapld_step)."""
     succ = W > 0 and not (flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"]))
     semantic = not flags & FLAG_NAMES["no_semantic"]
-    n = 2                                   # lexical, tree
+    lists = 1 if ld - 1 <= 4096 else 3      # distinct-token list kernels (one chunk: one)
+    n = 1                                   # lexical
     if semantic:
-        n += 1 + (4 if emb else 0)          # semantic (+ three list kernels, expansion)
-    if succ:
-        n += 1                              # successor scan
         if emb:
-            n += 3 if semantic else 6       # backoff plan, gathered pass, expansion
-                                            # (+ the lists, built by the tree stage)
+            n += lists + 2                  # lists, gathered pass, expansion
+        else:
+            n += 1 + (1 if B >= 288 else 0)  # semantic (+ the plan for large batches)
+    if succ and not emb and W * k <= 16:
+        n += 1                              # successor scan fused with the tree
+    elif succ:
+        if emb and not semantic:
+            n += lists                      # the lists, built by the tree stage
+        n += 2 + (3 if emb else 0)          # scan, tree (+ backoff plan, gathered pass,
+                                            # expansion)
+    else:
+        n += 1                              # tree
     return n
 
 
@@ -494,6 +523,7 @@ def run_native(args):
 
     # end-to-end through the public API from pinned host buffers
     e2e = None
+    host_in = None  # numpy views of the pinned host inputs (also the oracle's inputs)
     if not args.no_e2e and emb is None:
         tok_h = w.tokens.cpu().pin_memory()
         len_h = w.lengths.cpu().pin_memory()
@@ -502,6 +532,9 @@ def run_native(args):
         # the host link at a fraction of the rate in probes)
         reps_h = w.reps.cpu().pin_memory()
         q_h = w.query.cpu().pin_memory()
+        host_in = (tok_h.numpy(), len_h.numpy(),
+                   reps_h.view(torch.int16).numpy().view(np.uint16),
+                   q_h.view(torch.int16).numpy().view(np.uint16))
         dev_in = (torch.empty_like(w.tokens), torch.empty_like(w.lengths),
                   torch.empty_like(w.reps), torch.empty_like(w.query))
         host_out = native.Outputs.allocate(w.B, p, device="cpu", pin_memory=True)
@@ -524,7 +557,7 @@ def run_native(args):
         te = max_over_ranks(e0.elapsed_time(e1), dev)
         e2e = {"value": job_throughput(world, KE, te), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
-        del reps_h, dev_in
+        del dev_in
 
     if rank != 0:
         if world > 1:
@@ -536,34 +569,35 @@ def run_native(args):
     achieved = nbytes[dom_name] / (sem_avg_ms / 1000.0) / 1e9
     step_gbs = nbytes["step"] / (ms_per_step / 1000.0) / 1e9
     cpu = None
-    if not args.no_cpu_baseline:
-        sample = OracleSample(cfg, args.seed, rows=65536, batch=args.batch)
-        threads = host_threads(sample.n_miss + sample.n_hit)
-        v1 = statistics.median([sample.rate() for _ in range(3)])
-        vp = statistics.median([sample.rate_parallel(threads) for _ in range(3)])
-        cpu = {"value": vp, "unit": UNIT, "cores": threads, "kind": "oracle",
-               "sample": sample.parallel_desc(threads), "value_1_thread": v1,
-               "sample_1_thread": sample.desc}
+    if not args.no_cpu_baseline and emb is None:
+        # whole oracle steps over the same batch: one step on every host
+        # thread it can use, then one on a single thread (about 10-30 s of
+        # host CPU work at configs 3 and 5)
+        if host_in is None:
+            host_in = host_copy(w)
+        run = OracleRun(*host_in, w.n_max, w.k, w.W, w.D, w.succ_len, w.tau, flags)
+        threads = host_threads(w.B)
+        walls = [run.step(threads) for _ in range(2)]
+        wall1 = run.step(1)
+        cpu = {"value": len(walls) / sum(walls), "unit": UNIT, "cores": threads,
+               "kind": "oracle", "sample": run.desc(threads, cfg) + f"; {len(walls)} steps",
+               "value_1_thread": 1.0 / wall1, "sample_1_thread": run.desc(1, cfg) + "; 1 step",
+               "outcomes_match": run.outcomes() == {
+                   "lexical": int((g["hit_kind"] == 1).sum()),
+                   "semantic": int((g["hit_kind"] == 2).sum()),
+                   "none": int((g["hit_kind"] == 0).sum())}}
+    host_in = None
     hk = g["hit_kind"]
-    conf = workload_config(cfg)
-    if emb is not None:
-        conf["workload"] += (f" + token-embedding fallback ({emb.shape[0]} x {emb.shape[1]} "
-                             "table; two-representation mode)")
-    if flags:
-        conf["workload"] += f" ablation: {args.flags}"
-        conf["flags"] = flags
-    if args.batch is not None:
-        conf["workload"] += f" (resized: B={w.B})"
-        conf["B"] = conf["global_batch"] = w.B
-    conf.update({"parallelism": f"replicas x{world} (batch per GPU)",
-                 "outcomes": {"lexical": int((hk == 1).sum()), "semantic": int((hk == 2).sum()),
-                              "none": int((hk == 0).sum())},
-                 "accumulate": "fp32"})
+    conf = workload_config(cfg, args.batch, flags,
+                           None if emb is None else (int(emb.shape[0]), int(emb.shape[1])))
+    conf["outcomes"] = {"lexical": int((hk == 1).sum()), "semantic": int((hk == 2).sum()),
+                        "none": int((hk == 0).sum())}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K,
         "warmup": max(3, args.warmup), "ms_per_step": ms_per_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": conf,
+        "parallelism": f"replicas x{world} (batch per GPU)", "accumulate": "fp32",
         "sequence_steps_per_s": value * w.B,
         "roofline": {"bound": "hbm", "kernel": dom_kernel,
                      "achieved": achieved, "peak": peak, "peak_kind": peak_kind,
@@ -578,7 +612,7 @@ def run_native(args):
         "cpu_baseline": cpu,
         "e2e": e2e,
         "verify": verify,
-        "gpu_launches": step_launches(flags, w.W, emb is not None) * K,
+        "gpu_launches": step_launches(flags, w.W, emb is not None, w.k, w.B, w.ld) * K,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

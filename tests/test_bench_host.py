@@ -28,6 +28,9 @@ def test_step_launches():
     assert bench.step_launches(native.NO_SEMANTIC, 4, True) == 9
     assert bench.step_launches(native.NO_BRANCH | native.NO_SEMANTIC, 4, False) == 2
     assert bench.step_launches(0, 0, False) == 3
+    assert bench.step_launches(0, 2, False, k=8, B=256, ld=4096) == 3   # fused tree stage
+    assert bench.step_launches(0, 3, False, k=8, B=300, ld=40) == 5     # + outcome plan
+    assert bench.step_launches(0, 2, True, k=8, B=256, ld=4096) == 9    # one list kernel
 
 
 class _W:
@@ -61,19 +64,25 @@ def test_algorithmic_bytes_by_variant():
 
 
 def test_reference_arm_prints_one_line(capsys):
-    """`bench.py --impl reference` times the oracle on host threads and prints
-    the contract's JSON line (small workload: config 1)."""
+    """`bench.py --impl reference` times whole oracle steps over the full
+    workload on host threads and prints the contract's JSON line, with the
+    same config object the native arm prints (small workload: config 1)."""
     import json
     import argparse
-    args = argparse.Namespace(config=1, seed=0, steps=2, warmup=1, gpus=1, batch=None)
+    args = argparse.Namespace(config=1, seed=0, steps=2, warmup=1, gpus=1, batch=None,
+                              flags="", embeddings=False)
     bench.run_reference(args)
     out = [ln for ln in capsys.readouterr().out.splitlines() if ln.startswith("{")]
     assert len(out) == 1
     line = json.loads(out[0])
-    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["impl"] == "reference" and line["value"] > 0 and line["steps"] == 2
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
     assert line["e2e"] == {"value": line["value"], "unit": line["unit"],
                            "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    conf = bench.workload_config(1)
+    conf["outcomes"] = line["config"]["outcomes"]
+    assert line["config"] == conf
+    assert sum(conf["outcomes"].values()) == conf["B"]
 
 
 def test_algorithmic_bytes_embedding_mode():
@@ -97,13 +106,28 @@ def test_algorithmic_bytes_embedding_mode():
     assert x["tree"] - base["tree"] == extra
 
 
-def test_oracle_sample_counts_the_workloads_misses():
-    """The CPU baseline extrapolates to the timed workload's own lexical
-    misses: every forced miss, plus histories that miss naturally."""
+def test_oracle_run_times_whole_steps_of_the_batch():
+    """The CPU baseline runs the oracle's whole step over every sequence of
+    the batch (one per task): the outcomes it reports are the oracle's own,
+    whatever the thread count."""
+    import oracle
     from paper_2606_05742_gb300 import synth
-    sample = bench.OracleSample(2, 0, rows=256)
-    tokens, lengths, forced = synth.make_tokens(2, seed=0)
-    assert sample.n_miss + sample.n_hit == synth.CONFIGS[2]["B"]
-    assert sample.n_miss >= len(forced)
-    small = bench.OracleSample(2, 0, rows=256, batch=4)
-    assert small.n_miss + small.n_hit == 4
+    w = synth.make_workload(2, B=5, L=600, d=16, nohit=0.4, seed=3)
+    run = bench.OracleRun(w.tokens, w.lengths, w.reps, w.query, w.n_max, w.k, w.W, w.D,
+                          w.succ_len, w.tau)
+    assert run.step(3) > 0
+    ref = oracle.step(w.tokens, w.lengths, w.reps, w.query, w.n_max, w.k, w.W, w.D,
+                      w.succ_len, w.tau)
+    assert (run.hit == ref.hit).all()
+    o = run.outcomes()
+    assert o["none"] + o["lexical"] + o["semantic"] == 5 and o["lexical"] >= 1
+    run.step(1)
+    assert (run.hit == ref.hit).all()
+
+
+def test_workload_config_is_shared_by_both_arms():
+    a = bench.workload_config(5)
+    assert a == bench.workload_config(5, None, 0, None)
+    assert a["B"] == 8 and a["L"] == 131072 and a["d"] == 8192
+    r = bench.workload_config(2, batch=4, flags=native.NO_SUCC)
+    assert r["B"] == r["global_batch"] == 4 and r["flags"] == native.NO_SUCC
