@@ -280,12 +280,26 @@ __device__ __forceinline__ void cluster_sync_relaxed() {
     asm volatile("barrier.cluster.arrive.relaxed.aligned;\n\t"
                  "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
-__device__ __forceinline__ int ld_cluster_i32(const int *local, uint32_t rank) {
+__device__ __forceinline__ uint32_t cluster_addr(const void *local, uint32_t rank) {
     uint32_t remote;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+    return remote;
+}
+__device__ __forceinline__ int ld_cluster_i32(const int *local, uint32_t rank) {
     int v;
-    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(remote) : "memory");
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(cluster_addr(local, rank)) : "memory");
     return v;
+}
+__device__ __forceinline__ float ld_cluster_f32(const float *local, uint32_t rank) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(cluster_addr(local, rank)) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_cluster_i32(int *local, uint32_t rank, int v) {
+    asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(cluster_addr(local, rank)), "r"(v) : "memory");
+}
+__device__ __forceinline__ void st_cluster_f32(float *local, uint32_t rank, float v) {
+    asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(cluster_addr(local, rank)), "f"(v) : "memory");
 }
 
 __device__ __forceinline__ uint4 ldg_nc_v4(const void *p) {

@@ -62,7 +62,6 @@ __device__ __forceinline__ int stage_chunk(int *buf, const int32_t *M, int j0, i
 
 __global__ void __launch_bounds__(kThreadsL, 2) lexical_kernel(LexArgs args) {
     const LexLaunch &a = args.p;
-    const Workspace &ws = args.ws;
     extern __shared__ __align__(16) int dyn[];  // [1 or 2][kBufL] staged chunks
     __shared__ int suf[8];
     __shared__ int wval[kWarpsL];

@@ -1,5 +1,13 @@
 // Rerank and draft-tree construction (Sec. 3.4-3.6, Eq. 6-15, Algorithm 1).
 //
+// In single-cache mode with histories of at most 16 slices of 8192 positions
+// (every workload shape here) the stage is one kernel of thread-block
+// clusters, tree_cluster_kernel (see its comment below): the CTAs of a
+// sequence scan slices, score rows and hand their results to CTA rank 0
+// through distributed shared memory.  The kernels below serve the other
+// cases (token-embedding mode, whose successor backoff runs between the scan
+// and the scoring, and longer histories).
+//
 // With at most 16 successor rows per sequence (W*k <= 16) the stage is one
 // kernel: succ_scan_kernel<U, true>, where the CTA that completes a
 // sequence's scan (or CTA 0 of a sequence without successors) goes on to
@@ -35,6 +43,8 @@
 // vector, the candidates' continuation tokens and the token after each scored
 // row.  With one slice the fused kernel reads every history token it needs
 // from the staged slice.
+#include <cstdlib>
+
 #include "common.cuh"
 
 namespace adapld {
@@ -77,6 +87,8 @@ struct TreeSmem {
 // Where a CTA reads history tokens: the staged history (s_tok: positions
 // [0, ld) of the sequence), or global memory; wsm, when set, holds the
 // continuation windows of the candidates (M[s_cand[q]+1] = win[slot[q]][0]).
+__device__ __forceinline__ float *s_red_of(TreeSmem &sm) { return sm.red; }
+
 struct TokSrc {
     const int *s_tok;
     const TreeSmem *wsm;
@@ -290,26 +302,34 @@ __device__ __forceinline__ int branch_set(const TreeLaunch &a, int b, const SeqV
     }
     if (t == kThreads4 - 1) s_misc[0] = v.lex ? next_of(0) : -1;
     __syncthreads();
-    if (t == 0) {
-        int nb = 0;
-        if (a.next_topk) {
-            for (int r = 0; r < a.Kn && nb < W; ++r)
-                if (s_next[r] >= 0) s_br[nb++] = s_next[r];
-        } else {
-            for (int r = 0; r < v.nc && nb < W; ++r) {
-                const int tkn = s_next[r];
-                bool dup = false;
-                for (int e = 0; e < nb; ++e) dup |= s_br[e] == tkn;
-                if (!dup) s_br[nb++] = tkn;
+    if (t < 32) {  // warp 0: the first W distinct continuations (or the first W ids of
+                   // the table row), then Eq. 11's removal of main[0], order kept
+        const int lane = t;
+        const int n = a.next_topk ? a.Kn : v.nc;
+        const int main0 = s_misc[0];
+        int nb = 0, taken = 0;
+        for (int base = 0; base < n && taken < W; base += 32) {  // (nc <= 32: one pass)
+            const int r = base + lane;
+            const bool in = r < n;
+            const int tkn = in ? s_next[r] : 0;
+            bool keep;
+            if (a.next_topk) {
+                keep = in && tkn >= 0;
+            } else {  // the first occurrence of each token in rank order
+                const unsigned peers = __match_any_sync(0xffffffffu, tkn) &
+                                       __ballot_sync(0xffffffffu, in);
+                keep = in && __ffs(peers) - 1 == lane;
             }
+            const unsigned below = (1u << lane) - 1u;
+            const unsigned km = __ballot_sync(0xffffffffu, keep);
+            const bool sel = keep && taken + __popc(km & below) < W;
+            const bool fin = sel && !(v.lex && tkn == main0);
+            const unsigned fm = __ballot_sync(0xffffffffu, fin);
+            if (fin) s_br[nb + __popc(fm & below)] = tkn;
+            nb += __popc(fm);
+            taken += __popc(km);
         }
-        if (v.lex) {  // Eq. 11
-            int m = 0;
-            for (int e = 0; e < nb; ++e)
-                if (s_br[e] != s_misc[0]) s_br[m++] = s_br[e];
-            nb = m;
-        }
-        s_misc[1] = nb;
+        if (lane == 0) s_misc[1] = nb;
     }
     __syncthreads();
     return s_misc[1];
@@ -338,6 +358,62 @@ __device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int 
     __syncwarp();
 }
 
+// The k most recent positions p in [lo, hi) with M[p] == br[w], for every
+// branch w < nb, most recent first: store(w, rank, p) for rank < k, then
+// count(w, c) once per branch (by thread w) with c = their number (<= k);
+// s_tok[p - p0] holds M[p].  Block-wide (every thread).  The range is split
+// into one contiguous part per warp (higher warps more recent), so all 16
+// warps scan at once: a first pass counts each warp's matches per branch (wc:
+// 16 * nb ints of scratch), a second stores each warp's matches at ranks
+// after those of the warps above it, until k.
+template <class Store, class Count>
+__device__ __forceinline__ void scan_branches(const int *s_tok, int64_t p0, int64_t lo,
+                                              int64_t hi, const int *br, int nb, int k, int *wc,
+                                              Store store, Count count) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    constexpr int NW = kThreads4 / 32, U4 = 4;
+    const int64_t n = hi > lo ? hi - lo : 0;
+    const int64_t per = (n + NW * 32 * U4 - 1) / (NW * 32 * U4) * (32 * U4);  // per warp
+    const int64_t wlo = lo + warp * per;
+    const int64_t whi = min(wlo + per, hi);
+    const int groups = whi > wlo ? (int)((whi - wlo + 31) / 32) : 0;  // a multiple of U4
+                                                                       // unless clipped
+    for (int w = 0; w < nb; ++w) {
+        const int bt = br[w];
+        int c = 0;
+        for (int g = 0; g < groups; g += U4) {  // U4 independent loads per step
+            int tk[U4];
+#pragma unroll
+            for (int u = 0; u < U4; ++u) {
+                const int64_t p = wlo + 32 * (g + u) + lane;
+                tk[u] = p < whi ? s_tok[p - p0] : ~bt;
+            }
+#pragma unroll
+            for (int u = 0; u < U4; ++u) c += __popc(__ballot_sync(0xffffffffu, tk[u] == bt));
+        }
+        if (lane == 0) wc[warp * nb + w] = c;
+    }
+    __syncthreads();
+    for (int w = 0; w < nb; ++w) {
+        int off = 0;
+        for (int u = warp + 1; u < NW; ++u) off += wc[u * nb + w];
+        if (off >= k || wc[warp * nb + w] == 0) continue;
+        const int bt = br[w];
+        for (int g = groups - 1; g >= 0 && off < k; --g) {
+            const int64_t p = wlo + 32 * g + lane;
+            const unsigned m = __ballot_sync(0xffffffffu, p < whi && s_tok[p - p0] == bt);
+            const int rank = off + __popc((m >> lane) >> 1);  // higher lanes are more recent
+            if (((m >> lane) & 1u) && rank < k) store(w, rank, (int)p);
+            off += __popc(m);
+        }
+    }
+    if ((int)threadIdx.x < nb) {
+        int total = 0;
+        for (int u = 0; u < NW; ++u) total += wc[u * nb + threadIdx.x];
+        count((int)threadIdx.x, min(total, k));
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Publishes the successor-candidate count of branch w of sequence b.  A
 // branch token that never occurs earlier backs off (Sec. 3.5) to the
@@ -351,6 +427,134 @@ __device__ __forceinline__ void register_successors(const TreeLaunch &a, const W
         ws.pair_b[idx] = b;
         ws.pair_tok[idx] = token;
         ws.pair_out[idx] = b * ws.W + w;
+    }
+}
+
+// Lays out and writes the draft tree of sequence b (the root, the main chain
+// of a lexical hit, then each branch with its successor chain) and the
+// per-sequence outputs: tokens, parents, position ids, the ancestor mask,
+// the ranked candidates (lexical / reranked), anchor, node count, statistics
+// and status.  sm holds the ranked candidates (cand, score, slot), the
+// branch set (br, nb branches), the successor picked per branch (succ, stok)
+// when the sequence drafts successors, and the continuation windows (win)
+// when use_win.  Block-wide (every thread).
+__device__ __forceinline__ void emit_tree(const TreeLaunch &a, int b, const SeqView &v, TreeSmem &sm,
+                          const TokSrc &src, bool use_win, int nb, int status0) {
+    int *s_cand = sm.cand;
+    float *s_score = sm.score;
+    int *s_br = sm.br;
+    int *s_succ = sm.succ;
+    int *s_misc = sm.misc;
+    int *node_par = sm.node_par;
+    short *node_depth = sm.node_depth;
+    short *node_path = sm.node_path;
+    int *node_src = sm.node_src;
+    const int t = threadIdx.x;
+    const int k = a.p.k, W = a.p.branch_width, D = a.p.draft_len;
+    const int succ_len = a.p.succ_len;
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const int js = (v.lex || v.sem) ? s_cand[0] : -1;
+    const int N = 1 + D + W * (1 + succ_len);
+    // node layout, in parallel: the root, the main chain (l nodes), then per
+    // branch w its node and its successor chain of added_w nodes, starting at
+    // 1 + l + the sizes of the branches before it (a warp scan)
+    const int l = (v.valid && v.lex) ? min(D, v.len - 1 - js) : 0;
+    int *s_start = sm.next;  // (free once the branch set is built)
+    const int nbv = v.valid ? nb : 0;
+    if (t < 32) {
+        const int lane = t;
+        int carry = 1 + l, ext = 0;
+        for (int base = 0; base < nbv; base += 32) {
+            const int w = base + lane;
+            int size = 0, added = 0;
+            if (w < nbv) {
+                if (v.need_succ && s_succ[w] >= 0) added = min(succ_len, v.len - 1 - s_succ[w]);
+                size = 1 + added;
+            }
+            int incl = size;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += u;
+            }
+            if (w < nbv) s_start[w] = carry + incl - size;
+            carry += __shfl_sync(0xffffffffu, incl, 31);
+            ext += __popc(__ballot_sync(0xffffffffu, added > 0));
+        }
+        if (lane == 0) {
+            s_misc[0] = v.valid ? carry : 0;
+            s_misc[3] = ext;
+        }
+    }
+    if (v.valid && t <= l) {  // the root and the main chain
+        node_par[t] = t - 1;
+        node_depth[t] = (short)t;
+        node_path[t] = t == 0 ? 0 : 1;
+        node_src[t] = t == 0 ? v.len - 1 : js + t;
+    }
+    __syncthreads();
+    {
+        const int lane = t & 31, warp = t >> 5;
+        for (int w = warp; w < nbv; w += kThreads4 / 32) {  // branch w: its node, then
+                                                             // its successors
+            const int st = s_start[w];
+            const int size = (w + 1 < nbv ? s_start[w + 1] : s_misc[0]) - st;
+            if (lane < size) {
+                const int nd = st + lane;
+                node_par[nd] = lane == 0 ? 0 : nd - 1;
+                node_depth[nd] = (short)(1 + lane);
+                node_path[nd] = (short)(2 + w);
+                node_src[nd] = lane == 0 ? -2 - w : s_succ[w] + lane;  // -2-w: the branch token
+            }
+        }
+    }
+    __syncthreads();
+    const int n = s_misc[0];
+    const int64_t ob = (int64_t)b * N;
+    for (int i = t; i < N; i += kThreads4) {
+        int tok = -1, par = -1, pos = -1;
+        if (i < n) {
+            const int s = node_src[i], path = node_path[i], depth = node_depth[i];
+            if (s < 0)
+                tok = s_br[-2 - s];
+            else if (src.s_tok)
+                tok = src.s_tok[s];
+            else if (path == 1 && use_win && depth <= kWin)  // main chain: s = j* + depth
+                tok = sm.win[sm.slot[0]][depth - 1];
+            else if (path >= 2 && depth == 2)  // a branch's first successor token
+                tok = sm.stok[path - 2];
+            else
+                tok = __ldg(M + s);
+            par = node_par[i];
+            pos = v.len - 1 + depth;
+        }
+        a.out.draft_tokens[ob + i] = tok;
+        a.out.parents[ob + i] = par;
+        a.out.positions[ob + i] = pos;
+    }
+    uint8_t *mk = a.out.mask + (int64_t)b * N * N;
+    for (int idx = t; idx < N * N; idx += kThreads4) {
+        const int i = idx / N, j = idx % N;
+        const bool anc = i < n && j < n &&
+                         (j == i || j == 0 ||
+                          (node_path[i] == node_path[j] && j <= i && node_path[i] != 0));
+        mk[idx] = anc ? 1 : 0;
+    }
+    if ((v.lex || v.rr) && t < k) {
+        a.cand[(int64_t)b * k + t] = t < v.nc ? s_cand[t] : -1;
+        a.score[(int64_t)b * k + t] = t < v.nc ? s_score[t] : 0.f;
+    }
+    if (t == 0) {
+        a.out.anchor[b] = js;
+        a.out.n_nodes[b] = n;
+        if (a.out.stats) {
+            atomicAdd(a.out.stats + (v.lex ? 0 : (v.sem ? 1 : 2)), 1);
+            if (s_misc[3]) atomicAdd(a.out.stats + 3, s_misc[3]);
+        }
+        if (a.status)  // the embedding fallback may have flagged a token id
+            a.status[b] = (status0 & ADAPLD_SEQ_BAD_TOKEN) |
+                          (v.valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) |
+                          (v.cand_ok ? 0 : ADAPLD_SEQ_BAD_CANDIDATE);
     }
 }
 
@@ -560,16 +764,11 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
     int *s_br = sm.br;
     int *s_succ = sm.succ;
     int *s_misc = sm.misc;
-    int *node_par = sm.node_par;
-    short *node_depth = sm.node_depth;
-    short *node_path = sm.node_path;
-    int *node_src = sm.node_src;
     float *s_red = sm.red;
 
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int nwarps = kThreads4 / 32;
-    const int k = a.p.k, d = a.d, W = a.p.branch_width, D = a.p.draft_len;
-    const int succ_len = a.p.succ_len;
+    const int k = a.p.k, d = a.d;
     const uint32_t flags = a.p.flags;
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
@@ -697,7 +896,6 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
         if (t < v.nc) s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
         __syncthreads();
     }
-    const int js = (v.lex || v.sem) ? s_cand[0] : -1;
     if (v.branch_on && !v.need_succ)
         nb = branch_set(a, b, v, s_cand, s_next, s_br, s_misc,
                         TokSrc{src.s_tok, use_win ? &sm : nullptr});
@@ -739,94 +937,7 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
         __syncthreads();
     }
 
-    const int N = 1 + D + W * (1 + succ_len);
-    if (t == 0) {
-        int n = 0, ext = 0;
-        if (v.valid) {
-            node_par[0] = -1;
-            node_depth[0] = 0;
-            node_path[0] = 0;
-            node_src[0] = v.len - 1;
-            n = 1;
-            if (v.lex) {
-                const int l = min(D, v.len - 1 - js);
-                for (int i = 0; i < l; ++i, ++n) {
-                    node_par[n] = i == 0 ? 0 : n - 1;
-                    node_depth[n] = (short)(i + 1);
-                    node_path[n] = 1;
-                    node_src[n] = js + 1 + i;
-                }
-            }
-            for (int w = 0; w < nb; ++w) {
-                node_par[n] = 0;
-                node_depth[n] = 1;
-                node_path[n] = (short)(2 + w);
-                node_src[n] = -2 - w;  // the branch token itself
-                ++n;
-                if (v.need_succ && s_succ[w] >= 0) {
-                    const int tb = s_succ[w];
-                    int added = 0;
-                    for (int i = 1; i <= succ_len && tb + i <= v.len - 1; ++i, ++n, ++added) {
-                        node_par[n] = n - 1;
-                        node_depth[n] = (short)(1 + i);
-                        node_path[n] = (short)(2 + w);
-                        node_src[n] = tb + i;
-                    }
-                    if (added > 0) ++ext;
-                }
-            }
-        }
-        s_misc[0] = n;
-        s_misc[3] = ext;
-    }
-    __syncthreads();
-    const int n = s_misc[0];
-    const int64_t ob = (int64_t)b * N;
-    for (int i = t; i < N; i += kThreads4) {
-        int tok = -1, par = -1, pos = -1;
-        if (i < n) {
-            const int s = node_src[i], path = node_path[i], depth = node_depth[i];
-            if (s < 0)
-                tok = s_br[-2 - s];
-            else if (src.s_tok)
-                tok = src.s_tok[s];
-            else if (path == 1 && use_win && depth <= kWin)  // main chain: s = j* + depth
-                tok = sm.win[sm.slot[0]][depth - 1];
-            else if (path >= 2 && depth == 2)  // a branch's first successor token
-                tok = sm.stok[path - 2];
-            else
-                tok = __ldg(M + s);
-            par = node_par[i];
-            pos = v.len - 1 + depth;
-        }
-        a.out.draft_tokens[ob + i] = tok;
-        a.out.parents[ob + i] = par;
-        a.out.positions[ob + i] = pos;
-    }
-    uint8_t *mk = a.out.mask + (int64_t)b * N * N;
-    for (int idx = t; idx < N * N; idx += kThreads4) {
-        const int i = idx / N, j = idx % N;
-        const bool anc = i < n && j < n &&
-                         (j == i || j == 0 ||
-                          (node_path[i] == node_path[j] && j <= i && node_path[i] != 0));
-        mk[idx] = anc ? 1 : 0;
-    }
-    if ((v.lex || v.rr) && t < k) {
-        a.cand[(int64_t)b * k + t] = t < v.nc ? s_cand[t] : -1;
-        a.score[(int64_t)b * k + t] = t < v.nc ? s_score[t] : 0.f;
-    }
-    if (t == 0) {
-        a.out.anchor[b] = js;
-        a.out.n_nodes[b] = n;
-        if (a.out.stats) {
-            atomicAdd(a.out.stats + (v.lex ? 0 : (v.sem ? 1 : 2)), 1);
-            if (s_misc[3]) atomicAdd(a.out.stats + 3, s_misc[3]);
-        }
-        if (a.status)  // the embedding fallback may have flagged a token id
-            a.status[b] = (status0 & ADAPLD_SEQ_BAD_TOKEN) |
-                          (v.valid ? 0 : ADAPLD_SEQ_BAD_LENGTH) |
-                          (v.cand_ok ? 0 : ADAPLD_SEQ_BAD_CANDIDATE);
-    }
+    emit_tree(a, b, v, sm, src, use_win, nb, status0);
 }
 
 // U: row loads in flight per lane.  U = 16 (one CTA per SM by registers)
@@ -843,6 +954,284 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
                  TokSrc{nullptr, nullptr}, &pf, -1, false);
 }
 
+// ---------------------------------------------------------------------------
+// The whole tree stage as one kernel of thread-block clusters (single-cache
+// mode; histories of at most 16 slices of 8192 positions).  Grid (X, B),
+// 512 threads; the X CTAs of a sequence are one cluster and share its work
+// through distributed shared memory instead of global tickets:
+//   P0  every CTA stages its slice of the history (span positions and the one
+//       after), reads the outcome, and starts the copy of the reference
+//       vector (the query for a rerank, R[j*+1] for successor rows) and the
+//       candidates' continuation windows;
+//   P1  (lexical hits that draft successors) the candidates are reranked
+//       (Eq. 6-7) over the cluster's warps; rank 0 collects the scores and
+//       every CTA sorts them alike;
+//   P2  every CTA derives the branch set (Eq. 10-11);
+//   P3  each CTA scans its slice for the branch tokens, a warp per branch,
+//       keeping the k most recent occurrences;
+//   P4  after a cluster barrier every CTA merges the slices' lists (ranks
+//       hold contiguous slices, higher ranks more recent) from the other
+//       CTAs' shared memory;
+//   P5  the scored rows (successor candidates against R[j*+1], Eq. 13, or
+//       the lexical candidates against the query, Eq. 6) are spread over the
+//       cluster's warps, one row per warp; each score and the token after
+//       its row go to rank 0's shared memory;
+//   P6  after a second barrier rank 0 ranks (Eq. 7), picks each branch's
+//       successor (Eq. 14) and writes the tree.
+// Every CTA passes every cluster barrier (no early exit before them); the
+// barriers' conditions depend only on the sequence, hence agree in a cluster.
+// A scored row is split into parts of 4096 elements (512 16-byte chunks,
+// one batch of loads at U = 16), each part one warp's work item, so a warp
+// waits for at most one batch of row loads per item.
+constexpr int kPartCh = 512;
+__host__ __device__ inline int row_parts(int d) { return ((d >> 3) + kPartCh - 1) / kPartCh; }
+
+struct ClusterLayout {
+    uint32_t tok, cnt, lst, mcnt, mlst, wc, sc, tk, pd, ps, total;
+};
+
+__host__ __device__ inline ClusterLayout cluster_layout(int d, int span, int W, int k, int T) {
+    ClusterLayout L;
+    size_t o = align_up((size_t)d * 2, 16);  // the reference vector (bf16)
+    L.tok = (uint32_t)o;
+    o = align_up(o + 4 * ((size_t)span + 1), 16);
+    L.cnt = (uint32_t)o;  // this CTA's occurrences per branch
+    o += 4 * (size_t)W;
+    L.lst = (uint32_t)o;  // [W][k], most recent first
+    o += 4 * (size_t)W * k;
+    L.mcnt = (uint32_t)o;  // merged over the cluster
+    o += 4 * (size_t)W;
+    L.mlst = (uint32_t)o;
+    o += 4 * (size_t)W * k;
+    L.wc = (uint32_t)o;  // scan scratch: matches per (warp, branch)
+    o += 4 * (size_t)(kThreads4 / 32) * W;
+    L.sc = (uint32_t)o;  // rank 0: every task's score
+    o += 4 * (size_t)T;
+    L.tk = (uint32_t)o;  // rank 0: the token after every task's row
+    o += 4 * (size_t)T;
+    const int P = row_parts(d);
+    L.pd = (uint32_t)o;  // rank 0: partial <row, ref> per (task, part)
+    o += 4 * (size_t)T * P;
+    L.ps = (uint32_t)o;  // rank 0: partial |row|^2 per (task, part)
+    o += 4 * (size_t)T * P;
+    L.total = (uint32_t)o;
+    return L;
+}
+
+struct ClusterArgs {
+    TreeLaunch p;
+    int span;  // history positions per CTA (<= kSlice4)
+    int T;     // scored rows per sequence at most
+};
+
+template <int U>
+__global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel(ClusterArgs args) {
+    const TreeLaunch &a = args.p;
+    __shared__ TreeSmem sm;
+    extern __shared__ __align__(16) uint8_t dyn[];
+    const int k = a.p.k, d = a.d, W = a.p.branch_width;
+    const ClusterLayout L = cluster_layout(d, args.span, W, k, args.T);
+    uint16_t *s_ref = (uint16_t *)dyn;
+    int *s_tok = (int *)(dyn + L.tok);
+    int *s_cnt = (int *)(dyn + L.cnt);
+    int *s_lst = (int *)(dyn + L.lst);
+    int *s_mcnt = (int *)(dyn + L.mcnt);
+    int *s_mlst = (int *)(dyn + L.mlst);
+    int *s_wc = (int *)(dyn + L.wc);
+    float *s_sc = (float *)(dyn + L.sc);
+    int *s_tk = (int *)(dyn + L.tk);
+    float *s_pd = (float *)(dyn + L.pd);
+    float *s_ps = (float *)(dyn + L.ps);
+    int *s_cand = sm.cand;
+    float *s_score = sm.score;
+
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int nwarps = kThreads4 / 32;
+    const int b = blockIdx.y, x = blockIdx.x, X = gridDim.x;
+    const int gwarp = x * nwarps + warp, gwarps = X * nwarps;  // the cluster's warps
+    const uint32_t flags = a.p.flags;
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
+    pdl_wait_then_release();
+
+    // ---- P0: the slice [p0, p0 + span] (clipped at ld) while the outcome is read
+    const int64_t p0 = (int64_t)x * args.span;
+    const int nld = p0 < a.ld ? (int)min((int64_t)args.span + 1, a.ld - p0) : 0;
+    for (int i = t; i < nld; i += kThreads4) cp_async4(s_tok + i, M + p0 + i);
+    const SeqView v = view_of(a, b);
+    const int status0 = (a.status && t == 0 && x == 0) ? a.status[b] : 0;
+    if (t < kMaxK) sm.slot[t] = t;
+    if (t < v.nc) {
+        s_cand[t] = v.cand_t;
+        s_score[t] = v.score_t;
+    }
+    __syncthreads();
+    const bool whole = X == 1;                      // the slice is the whole history
+    const bool rank_first = v.rr && v.need_succ;    // reranked before the branch set
+    const bool rerank_only = v.rr && !v.need_succ;  // reranked in P5
+    const bool use_win = !whole && v.nc > 0 && (v.lex || v.branch_on);
+    if (rank_first || rerank_only)
+        vec_issue(a.query + (int64_t)b * d, d, s_ref);
+    else if (v.need_succ)
+        vec_issue(R + (int64_t)(s_cand[0] + 1) * d, d, s_ref);
+    if (use_win && t < v.nc * kWin) {  // M[c+1 .. c+kWin] of each candidate c
+        const int r = t / kWin, o = t - r * kWin;
+        const int p = s_cand[r] + 1 + o;
+        sm.win[r][o] = p <= v.len - 1 ? __ldg(M + p) : -1;
+    }
+    auto tok_of = [&](int p) {  // M[p], from the slice where it is staged
+        const int64_t q = p - p0;
+        return (q >= 0 && q < nld) ? s_tok[q] : __ldg(M + p);
+    };
+
+    // ---- P1: the rerank the branch set depends on
+    if (rank_first) {
+        const float qss = vec_finish(s_ref, d, s_red_of(sm));
+        for (int q = gwarp; q < v.nc; q += gwarps) {
+            float dot, ss;
+            warp_row_dot<U>(R + (int64_t)s_cand[q] * d, s_ref, d, dot, ss);
+            if (lane == 0) st_cluster_f32(&s_sc[q], 0, cosine_from(dot, ss, qss));
+        }
+        cluster_sync_all();
+        if (t < v.nc) s_score[t] = ld_cluster_f32(&s_sc[t], 0);
+        __syncthreads();
+        if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc, sm.slot);
+        __syncthreads();
+        vec_issue(R + (int64_t)(s_cand[0] + 1) * d, d, s_ref);  // the successor reference
+    } else {
+        cp_async_wait_all();
+        __syncthreads();  // the slice and the windows are visible
+    }
+
+    // ---- P2: the branch set; P3: this slice's occurrences of each branch token
+    int nb = 0;
+    if (v.need_succ) {
+        nb = branch_set(a, b, v, s_cand, sm.next, sm.br, sm.misc,
+                        TokSrc{whole ? s_tok : nullptr, use_win ? &sm : nullptr});
+        const int64_t p1 = min(p0 + args.span, (int64_t)v.len - 1);  // positions <= len-2
+        scan_branches(
+            s_tok, p0, p0, p1, sm.br, nb, k, s_wc,
+            [&](int w, int rank, int p) { s_lst[w * k + rank] = p; },
+            [&](int w, int c) { s_cnt[w] = c; });
+    }
+    cluster_sync_all();  // every slice's lists are complete
+
+    // ---- P4: the successor candidates of each branch, most recent first
+    if (v.need_succ) {
+        for (int w = warp; w < nb; w += nwarps) {
+            const int total = warp_merge_desc(
+                X, k, [&](int r) { return ld_cluster_i32(&s_cnt[w], r); },
+                [&](int r, int i) { return ld_cluster_i32(&s_lst[w * k + i], r); },
+                s_mlst + w * k);
+            if (lane == 0) s_mcnt[w] = total;
+        }
+        __syncthreads();
+    }
+
+    // ---- P5: the scored rows over the cluster's warps, in parts; the partial
+    // sums (and the token after each row) go to rank 0
+    const int ntasks = v.need_succ ? nb * k : (rerank_only ? v.nc : 0);
+    const int nch = d >> 3, P = row_parts(d);
+    float rss = 0.f;
+    if (ntasks > 0) {
+        auto row_of = [&](int task) {
+            if (!v.need_succ) return s_cand[task];
+            const int w = task / k, i = task - w * k;
+            return i < s_mcnt[w] ? s_mlst[task] : -1;
+        };
+        // item = (task, part); a warp's items are gwarp, gwarp + gwarps, ...
+        auto part_dot = [&](int row, int part, uint4 (&w)[U], bool loaded, float &dot,
+                            float &ss) {
+            const uint16_t *rp = R + (int64_t)row * d;
+            const int base = part * kPartCh, end = min(base + kPartCh, nch);
+            dot = 0.f;
+            ss = 0.f;
+            for (int c0 = base; c0 < end; c0 += 32 * U) {
+                if (!(loaded && c0 == base)) row_batch_load<U>(rp, end, c0, w);
+                row_batch_acc<U>(w, s_ref, end, c0, dot, ss);
+            }
+            dot = warp_sum(dot);
+            ss = warp_sum(ss);
+        };
+        const int items = ntasks * P;
+        const int task0 = gwarp / P, part0 = gwarp - task0 * P;
+        const int row0 = gwarp < items ? row_of(task0) : -1;
+        uint4 w0[U];
+        if (row0 >= 0)
+            row_batch_load<U>(R + (int64_t)row0 * d, min(part0 * kPartCh + kPartCh, nch),
+                              part0 * kPartCh, w0);
+        const int tk0 = (v.need_succ && row0 >= 0 && part0 == 0 && lane == 0)
+                            ? tok_of(row0 + 1) : -1;
+        rss = vec_finish(s_ref, d, s_red_of(sm));
+        for (int it = gwarp; it < items; it += gwarps) {
+            const int task = it / P, part = it - task * P;
+            const int row = it == gwarp ? row0 : row_of(task);
+            float dot = 0.f, ss = 0.f;
+            if (row >= 0) part_dot(row, part, w0, it == gwarp, dot, ss);
+            if (lane == 0) {
+                st_cluster_f32(&s_pd[it], 0, dot);
+                st_cluster_f32(&s_ps[it], 0, ss);
+                if (v.need_succ && part == 0)
+                    st_cluster_i32(&s_tk[task], 0,
+                                   it == gwarp ? tk0 : (row >= 0 ? tok_of(row + 1) : -1));
+            }
+        }
+    }
+    cp_async_wait_all();  // (a reference row staged for no row: done before any exit)
+    cluster_sync_all();  // rank 0 holds every score; no CTA reads another's memory after this
+    if (x != 0) return;
+
+    // ---- P6 (rank 0): the cosines from the partial sums (parts in order), rank,
+    // branch, pick successors, emit
+    for (int task = t; task < ntasks; task += kThreads4) {
+        float dot = 0.f, ss = 0.f;
+        for (int part = 0; part < P; ++part) {
+            dot += s_pd[task * P + part];
+            ss += s_ps[task * P + part];
+        }
+        const bool real = v.need_succ ? (task - (task / k) * k) < s_mcnt[task / k] : true;
+        s_sc[task] = real ? cosine_from(dot, ss, rss) : -INFINITY;
+    }
+    __syncthreads();
+    if (rerank_only) {
+        if (t < v.nc) s_score[t] = s_sc[t];
+        __syncthreads();
+        if (warp == 0) warp_sort_desc(s_cand, s_score, v.nc, sm.slot);
+        __syncthreads();
+    } else if (v.lex && (flags & ADAPLD_NO_LEX_RERANK)) {
+        if (t < v.nc) s_score[t] = __int_as_float(0x7fc00000);  // NaN: not computed
+        __syncthreads();
+    }
+    if (v.branch_on && !v.need_succ)
+        nb = branch_set(a, b, v, s_cand, sm.next, sm.br, sm.misc,
+                        TokSrc{whole ? s_tok : nullptr, use_win ? &sm : nullptr});
+    if (v.need_succ) {
+        for (int w = warp; w < nb; w += nwarps) {  // Eq. 14: argmax per branch
+            const bool in = lane < s_mcnt[w];
+            float bs = in ? s_sc[w * k + lane] : -INFINITY;
+            int bj = in ? s_mlst[w * k + lane] : -1;
+            int btk = in ? s_tk[w * k + lane] : -1;
+#pragma unroll
+            for (int o = 16; o; o >>= 1) {
+                const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+                const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+                const int ot = __shfl_xor_sync(0xffffffffu, btk, o);
+                if (better(os, oj, bs, bj)) {
+                    bs = os;
+                    bj = oj;
+                    btk = ot;
+                }
+            }
+            if (lane == 0) {
+                sm.succ[w] = bj >= 0 ? bj : -1;
+                sm.stok[w] = btk;
+            }
+        }
+        __syncthreads();
+    }
+    emit_tree(a, b, v, sm, TokSrc{whole ? s_tok : nullptr, nullptr}, use_win, nb, status0);
+}
+
 }  // namespace
 
 // Successor rows per sequence up to which the fused kernel scores them in the
@@ -852,6 +1241,38 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
 // rows (configs 2 and 3) the second kernel's parallel rows win by 4-14 us.
 constexpr int kMaxFusedTasks = kRowsPerCta5;
 static_assert(kMaxFusedTasks <= kMaxK, "fused lists live in TreeSmem::lpos");
+
+// The cluster kernel's shape for this launch: CTAs per sequence (enough for
+// every slice of 8192 positions and, up to 8 -- or 16 when the grid then
+// still fits one CTA per SM -- one warp per scored row) and positions per CTA.
+// Returns false where it does not apply (token-embedding mode, whose
+// successor backoff runs between the scan and the scoring; histories of more
+// than 16 slices; shared memory beyond one SM).
+bool cluster_shape(const TreeLaunch &a, int sms, int tasks, int *X, int *span, size_t *smem) {
+    if (a.emb.table) return false;
+    if (const char *e = std::getenv("ADAPLD_TREE_CLUSTER"))  // A/B switch for measurements
+        if (e[0] == '0') return false;
+    const int S = chunks_of(a.ld - 1, kSlice4);
+    if (S > kWideClusterL) return false;
+    const int R = (tasks + kRowsPerCta5 - 1) / kRowsPerCta5;
+    const int cap = (int64_t)a.B * kWideClusterL <= sms ? kWideClusterL : kMaxClusterL;
+    int x = R < cap ? R : cap;
+    if (x < S) x = S;
+    // one CTA per sequence: the older single kernel (succ_scan_kernel<U, true>)
+    // measured faster (config 4: 21.2 against 25.2 us; config 1: 12.9 against
+    // 15.0)
+    if (x < 2) return false;
+    const int64_t n = a.ld - 1;
+    int sp = (int)((n + x - 1) / x);
+    if (sp < 1) sp = 1;
+    const size_t dyn =
+        cluster_layout(a.d, sp, a.p.branch_width, a.p.k, tasks).total;
+    if (dyn + sizeof(TreeSmem) > 227 * 1024) return false;
+    *X = x;
+    *span = sp;
+    *smem = dyn;
+    return true;
+}
 
 cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s) {
     const int W = a.p.branch_width, k = a.p.k;
@@ -863,6 +1284,38 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
         return cudaErrorInvalidDevice;
+    int X = 0, span = 0;
+    size_t csmem = 0;
+    if (cluster_shape(a, sms, tasks, &X, &span, &csmem)) {  // the stage as one kernel
+        ClusterArgs ca{a, span, tasks};
+        // 16 row loads in flight per lane (one CTA per SM) while the grid fits
+        // one wave; not with clusters of 16, of which only 7 are resident at
+        // one CTA per SM on GB300 (config 5's 8 sequences took two waves)
+        auto kern = ((int64_t)X * a.B <= sms && X <= kMaxClusterL) ? tree_cluster_kernel<16>
+                                                                   : tree_cluster_kernel<8>;
+        cudaError_t e =
+            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)csmem);
+        if (e != cudaSuccess) return e;
+        if (X > kMaxClusterL) {
+            e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+            if (e != cudaSuccess) return e;
+        }
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(X, a.B);
+        cfg.blockDim = dim3(kThreads4);
+        cfg.dynamicSmemBytes = csmem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[2];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = X;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = X > 1 ? 2 : 1;  // a plain launch is a cluster of one CTA
+        return cudaLaunchKernelEx(&cfg, kern, ca);
+    }
     const size_t vsmem = (size_t)a.d * sizeof(uint16_t);  // the staged query / reference row
     const size_t ssmem = vsmem + (size_t)(kSlice4 + 1) * sizeof(int);  // + a slice's tokens
     if (succ_possible) {

@@ -462,6 +462,22 @@ def test_lexical_cluster_shapes(xmax, monkeypatch):
         check_all(w, run_step(w, P), P)
 
 
+@pytest.mark.parametrize("B,L,W,k", [(3, 900, 2, 8), (4, 9000, 3, 8), (3, 20000, 4, 32),
+                                     (5, 40000, 8, 32), (20, 70000, 1, 4), (3, 100000, 2, 16),
+                                     (2, 131073, 64, 32)])
+def test_tree_cluster_shapes(B, L, W, k):
+    """The single-kernel tree stage over clusters of 1 to 16 CTAs per
+    sequence (history slices from 1 to 16, scored rows from a few to 2048,
+    several rows per warp), against the oracle, with and without the
+    text-rule successors of lexical hits (their rerank runs across the
+    cluster before the branch set)."""
+    w = synth.make_workload(5, B=B, L=L, d=64, V=300, nohit=0.5, seed=L + W,
+                            lengths=[L] + [max(2, L - 977 * i) for i in range(1, B)])
+    for flags in (0, oracle.SUCC_ON_STRICT):
+        P = P_of(w, tau=NEG_INF, W=W, k=k, flags=flags)
+        check_all(w, run_step(w, P), P)
+
+
 def test_semantic_wait_timeout_is_reported_and_recoverable(monkeypatch):
     """Failure path without a fault: with the test switch the semantic
     kernel's producer issues no copy, so every bounded wait expires; the call
