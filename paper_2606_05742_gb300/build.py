@@ -2,7 +2,11 @@
 
 Each ``csrc/*.cu`` translation unit compiles in parallel to an object file
 under ``_build/``, then nvcc links them into the shared library next to this
-file.  Rebuilds only what changed.
+file.  Rebuilds only what changed.  ``build(checked=True)`` builds the
+checked debug library ``libadapld_checked.so`` (``-DADAPLD_CHECKED``: every
+computed index in the kernels is tested before use and a failure raises
+ADAPLD_DEV_INTERNAL instead of touching memory) from objects of its own
+under ``_build/checked/``.
 """
 from __future__ import annotations
 
@@ -18,6 +22,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(HERE, "libadapld.so")
+LIB_CHECKED = os.path.join(HERE, "libadapld_checked.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
@@ -37,15 +42,17 @@ def _deps_mtime() -> float:
     return max(os.path.getmtime(f) for f in files)
 
 
-def build(verbose: bool = False, extra_flags=None) -> str:
-    os.makedirs(BUILD, exist_ok=True)
+def build(verbose: bool = False, extra_flags=None, checked: bool = False) -> str:
+    bdir = os.path.join(BUILD, "checked") if checked else BUILD
+    lib = LIB_CHECKED if checked else LIB
+    os.makedirs(bdir, exist_ok=True)
     srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
     dep_t = _deps_mtime()
-    flags = NVCC_FLAGS + list(extra_flags or [])
+    flags = NVCC_FLAGS + (["-DADAPLD_CHECKED"] if checked else []) + list(extra_flags or [])
     jobs = []
     objs = []
     for src in srcs:
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(bdir, os.path.basename(src)[:-3] + ".o")
         objs.append(obj)
         if (not os.path.exists(obj) or os.path.getmtime(obj) < max(os.path.getmtime(src), dep_t)):
             jobs.append([nvcc(), *ARCH, *flags, "-c", src, "-o", obj])
@@ -59,11 +66,11 @@ def build(verbose: bool = False, extra_flags=None) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=max(1, min(len(jobs), os.cpu_count() or 4))) as ex:
         list(ex.map(run, jobs))
-    if jobs or not os.path.exists(LIB) or os.path.getmtime(LIB) < max(map(os.path.getmtime, objs)):
-        tmp = LIB + f".tmp{os.getpid()}"
+    if jobs or not os.path.exists(lib) or os.path.getmtime(lib) < max(map(os.path.getmtime, objs)):
+        tmp = lib + f".tmp{os.getpid()}"
         run([nvcc(), *ARCH, "-shared", "-o", tmp, *objs])
-        os.replace(tmp, LIB)
-    return LIB
+        os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":

@@ -149,6 +149,28 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
 // ---- device helpers ------------------------------------------------------------
 #ifdef __CUDACC__
 
+// The checked build (-DADAPLD_CHECKED: a debug library, build.build(checked=
+// True)) tests every computed index below before the access it guards: a
+// failed test raises ADAPLD_DEV_INTERNAL in the status word (nullable) and
+// the access is skipped -- never a trap.  In the normal build the tests
+// compile to nothing.
+#ifdef ADAPLD_CHECKED
+constexpr bool kChecked = true;
+#else
+constexpr bool kChecked = false;
+#endif
+
+// lo <= i < hi (always true in the normal build).
+__device__ __forceinline__ bool idx_ok(int64_t i, int64_t lo, int64_t hi, int32_t *status) {
+    if constexpr (!kChecked) {
+        return true;
+    } else {
+        const bool ok = i >= lo && i < hi;
+        if (!ok && status) atomicOr(status, ADAPLD_DEV_INTERNAL);
+        return ok;
+    }
+}
+
 // Programmatic dependent launch: wait until the previous kernel in the stream
 // has completed and its writes are visible (a no-op when this kernel was not
 // launched as a dependent), then allow the next kernel to begin launching.

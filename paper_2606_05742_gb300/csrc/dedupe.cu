@@ -188,7 +188,8 @@ __device__ int mark_chunk(const DedupeLaunch &a, const Workspace &ws, int b, int
 // position order to out (s_word: the chunk's 128 words in shared memory).
 // One scan over the word counts gives every offset.
 __device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32_t *s_word,
-                              int *s_off, int64_t *s_scan, int32_t *out) {
+                              int *s_off, int64_t *s_scan, int32_t *out, int64_t room,
+                              int32_t *dst) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t w = t < kWordsPerChunk ? s_word[t] : 0u;
     int64_t all;
@@ -201,9 +202,10 @@ __device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32
     for (int e = 0; e < kPerThread; ++e) {
         const int i = e * (kThreads1 / 32) + warp;
         const uint32_t wi = s_word[i];
-        if ((wi >> lane) & 1u) {
+        const int o = s_off[i] + __popc(wi & ((1u << lane) - 1u));
+        if (((wi >> lane) & 1u) && idx_ok(o, 0, room, dst)) {
             const int j = j0 + e * kThreads1 + t;
-            out[s_off[i] + __popc(wi & ((1u << lane) - 1u))] = canon(M[j], a.vocab);
+            out[o] = canon(M[j], a.vocab);
         }
     }
 }
@@ -265,7 +267,8 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
         int64_t total;  // the block's sum
         (void)block_exclusive_scan(mine, &total, s_scan);
         if (SINGLE) {  // one chunk: offset 0, no ticket
-            scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld);
+            scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld, a.ld,
+                          ws.dev_status);
             if (t == 0) {
                 ws.rep_len[b] = (int)total + 1;
                 ws.rep_tok[(int64_t)b * a.ld + total] = M[len - 1];  // the anchor (as stored)
@@ -326,8 +329,10 @@ __global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args)
     const uint32_t *bits = ws.rep_bits + ((int64_t)b * ws.C1 + c) * kWordsPerChunk;
     if (t < kWordsPerChunk) s_word[t] = __ldcg(bits + t);
     __syncthreads();
-    scatter_chunk(a, b, j0, s_word, s_off, s_scan,
-                  ws.rep_tok + (int64_t)b * a.ld + __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c));
+    const int off = __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c);
+    if (!idx_ok(off, 0, a.ld, ws.dev_status)) return;
+    scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld + off,
+                  a.ld - off, ws.dev_status);
 }
 
 // ---------------------------------------------------------------- expansion
@@ -402,7 +407,7 @@ __device__ void expand_one(const ExpandLaunch &a, const Workspace &ws, ExpandSha
             for (int u = 0; u < U; ++u) {
                 const int q = top - 32 * u - lane;
                 const int rank = cnt + __popc(m[u] & ((1u << lane) - 1u));
-                if (((m[u] >> lane) & 1u) && rank < k) {
+                if (((m[u] >> lane) & 1u) && rank < k && idx_ok(q, p0, p1, ws.dev_status)) {
                     if (single)
                         sh.lst[i][rank] = q;
                     else
@@ -441,7 +446,7 @@ __device__ void expand_one(const ExpandLaunch &a, const Workspace &ws, ExpandSha
         WarpTopK tk;
         tk.reset();
         for (int i = 0; i < n; ++i) {
-            const int c = sh.cnt[i];
+            const int c = idx_ok(sh.cnt[i], 0, k + 1, ws.dev_status) ? sh.cnt[i] : 0;
             tk.insert(lane < c, sh.sc[i], lane < c ? sh.lst[i][lane] : -1, k);
         }
         if (lane < k) {

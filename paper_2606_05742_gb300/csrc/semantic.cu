@@ -243,6 +243,9 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
             }
             const int b = real_seq(a, p);
             const int jend = (int)(seg_end - plan[p]);
+            // (checked build: the segment lies inside the sequence's rows)
+            if (!idx_ok(jend, 1, a.ld + 1, ws.dev_status) || !idx_ok(b, 0, a.B, ws.dev_status))
+                break;
             const uint8_t *base = (const uint8_t *)(a.reps + (int64_t)b * a.ld * d);
             const int32_t *Mb = GATHER ? a.tokens + (int64_t)b * a.ld : nullptr;
             // row ids in windows of 32 (SR divides 32, so a window starts on
@@ -437,7 +440,7 @@ __global__ void __launch_bounds__(kConsumers2 + 32, (semantic_min_blocks<MAXC, S
         volatile int *s_flag = (volatile int *)abort_flag + 1;  // the merge decision
         if (warp == 0) {
             int last = 0;
-            if (!aborted && !*abort_flag) {
+            if (!aborted && !*abort_flag && idx_ok(p + c, 0, B + grid, ws.dev_status)) {
                 int32_t *sp = args.slots + (int64_t)(p + c) * kSlotInts;
                 if (lane == 0) sp[0] = tk.n;
                 if (lane < tk.n) {

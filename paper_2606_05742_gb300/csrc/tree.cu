@@ -439,7 +439,8 @@ __device__ __forceinline__ void register_successors(const TreeLaunch &a, const W
 // when the sequence drafts successors, and the continuation windows (win)
 // when use_win.  Block-wide (every thread).
 __device__ __forceinline__ void emit_tree(const TreeLaunch &a, int b, const SeqView &v, TreeSmem &sm,
-                          const TokSrc &src, bool use_win, int nb, int status0) {
+                          const TokSrc &src, bool use_win, int nb, int status0,
+                          int32_t *dst = nullptr) {
     int *s_cand = sm.cand;
     float *s_score = sm.score;
     int *s_br = sm.br;
@@ -499,7 +500,7 @@ __device__ __forceinline__ void emit_tree(const TreeLaunch &a, int b, const SeqV
                                                              // its successors
             const int st = s_start[w];
             const int size = (w + 1 < nbv ? s_start[w + 1] : s_misc[0]) - st;
-            if (lane < size) {
+            if (lane < size && idx_ok(st + lane, 1, N, dst)) {
                 const int nd = st + lane;
                 node_par[nd] = lane == 0 ? 0 : nd - 1;
                 node_depth[nd] = (short)(1 + lane);
@@ -517,6 +518,8 @@ __device__ __forceinline__ void emit_tree(const TreeLaunch &a, int b, const SeqV
             const int s = node_src[i], path = node_path[i], depth = node_depth[i];
             if (s < 0)
                 tok = s_br[-2 - s];
+            else if (!idx_ok(s, 0, v.len, dst))
+                tok = -1;
             else if (src.s_tok)
                 tok = src.s_tok[s];
             else if (path == 1 && use_win && depth <= kWin)  // main chain: s = j* + depth
@@ -667,7 +670,8 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
             for (int u = 0; u < G; ++u) {
                 const int p = top - 32 * u - lane;
                 const int rank = cnt + __popc(m[u] & ((1u << lane) - 1u));
-                if (((m[u] >> lane) & 1u) && rank < k) lst[rank] = p;
+                if (((m[u] >> lane) & 1u) && rank < k && idx_ok(p, p0, p1, ws.dev_status))
+                    lst[rank] = p;
                 cnt += __popc(m[u]);
             }
         }
@@ -827,7 +831,8 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
         return i < n ? pos : -1;
     };
     const int first_task = task0 + warp;
-    const int row0 = first_task < task1 ? row_of(first_task, true) : -1;
+    int row0 = first_task < task1 ? row_of(first_task, true) : -1;
+    if (!idx_ok(row0, -1, v.len - 1, ws.dev_status)) row0 = -1;
     uint4 w0[U];
     if (row0 >= 0) row_batch_load<U>(R + (int64_t)row0 * d, d >> 3, 0, w0);
     if (ntasks > 0)
@@ -860,7 +865,8 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
             if (lane == 0) record(first_task, row0, sc, tk0);
         }
         for (int task = first_task + nwarps; task < task1; task += nwarps) {
-            const int row = row_of(task, false);
+            int row = row_of(task, false);
+            if (!idx_ok(row, -1, v.len - 1, ws.dev_status)) row = -1;
             float sc = 0.f;
             if (row >= 0) {
                 float dot, ss;
@@ -937,7 +943,7 @@ __device__ void tree_body(const TreeLaunch &a, const Workspace &ws, int b, const
         __syncthreads();
     }
 
-    emit_tree(a, b, v, sm, src, use_win, nb, status0);
+    emit_tree(a, b, v, sm, src, use_win, nb, status0, ws.dev_status);
 }
 
 // U: row loads in flight per lane.  U = 16 (one CTA per SM by registers)
@@ -1022,6 +1028,7 @@ struct ClusterArgs {
     TreeLaunch p;
     int span;  // history positions per CTA (<= kSlice4)
     int T;     // scored rows per sequence at most
+    int32_t *dev_status;  // the workspace's status word (checked build)
 };
 
 template <int U>
@@ -1079,7 +1086,9 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
         const int p = s_cand[r] + 1 + o;
         sm.win[r][o] = p <= v.len - 1 ? __ldg(M + p) : -1;
     }
+    int32_t *dst = args.dev_status;
     auto tok_of = [&](int p) {  // M[p], from the slice where it is staged
+        if (!idx_ok(p, 0, v.len, dst)) return -1;
         const int64_t q = p - p0;
         return (q >= 0 && q < nld) ? s_tok[q] : __ldg(M + p);
     };
@@ -1088,8 +1097,9 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
     if (rank_first) {
         const float qss = vec_finish(s_ref, d, s_red_of(sm));
         for (int q = gwarp; q < v.nc; q += gwarps) {
-            float dot, ss;
-            warp_row_dot<U>(R + (int64_t)s_cand[q] * d, s_ref, d, dot, ss);
+            float dot = 0.f, ss = 0.f;
+            if (idx_ok(s_cand[q], 0, v.len - 1, dst))
+                warp_row_dot<U>(R + (int64_t)s_cand[q] * d, s_ref, d, dot, ss);
             if (lane == 0) st_cluster_f32(&s_sc[q], 0, cosine_from(dot, ss, qss));
         }
         cluster_sync_all();
@@ -1111,7 +1121,10 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
         const int64_t p1 = min(p0 + args.span, (int64_t)v.len - 1);  // positions <= len-2
         scan_branches(
             s_tok, p0, p0, p1, sm.br, nb, k, s_wc,
-            [&](int w, int rank, int p) { s_lst[w * k + rank] = p; },
+            [&](int w, int rank, int p) {
+                if (idx_ok(rank, 0, k, dst) && idx_ok(w, 0, nb, dst) && idx_ok(p, p0, p1, dst))
+                    s_lst[w * k + rank] = p;
+            },
             [&](int w, int c) { s_cnt[w] = c; });
     }
     cluster_sync_all();  // every slice's lists are complete
@@ -1135,9 +1148,9 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
     float rss = 0.f;
     if (ntasks > 0) {
         auto row_of = [&](int task) {
-            if (!v.need_succ) return s_cand[task];
             const int w = task / k, i = task - w * k;
-            return i < s_mcnt[w] ? s_mlst[task] : -1;
+            const int row = !v.need_succ ? s_cand[task] : (i < s_mcnt[w] ? s_mlst[task] : -1);
+            return idx_ok(row, -1, v.len - 1, dst) ? row : -1;
         };
         // item = (task, part); a warp's items are gwarp, gwarp + gwarps, ...
         auto part_dot = [&](int row, int part, uint4 (&w)[U], bool loaded, float &dot,
@@ -1168,7 +1181,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
             const int row = it == gwarp ? row0 : row_of(task);
             float dot = 0.f, ss = 0.f;
             if (row >= 0) part_dot(row, part, w0, it == gwarp, dot, ss);
-            if (lane == 0) {
+            if (lane == 0 && idx_ok(it, 0, (int64_t)args.T * P, dst)) {
                 st_cluster_f32(&s_pd[it], 0, dot);
                 st_cluster_f32(&s_ps[it], 0, ss);
                 if (v.need_succ && part == 0)
@@ -1229,7 +1242,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
         }
         __syncthreads();
     }
-    emit_tree(a, b, v, sm, TokSrc{whole ? s_tok : nullptr, nullptr}, use_win, nb, status0);
+    emit_tree(a, b, v, sm, TokSrc{whole ? s_tok : nullptr, nullptr}, use_win, nb, status0, dst);
 }
 
 }  // namespace
@@ -1287,7 +1300,7 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
     int X = 0, span = 0;
     size_t csmem = 0;
     if (cluster_shape(a, sms, tasks, &X, &span, &csmem)) {  // the stage as one kernel
-        ClusterArgs ca{a, span, tasks};
+        ClusterArgs ca{a, span, tasks, ws.dev_status};
         // 16 row loads in flight per lane (one CTA per SM) while the grid fits
         // one wave; not with clusters of 16, of which only 7 are resident at
         // one CTA per SM on GB300 (config 5's 8 sequences took two waves)

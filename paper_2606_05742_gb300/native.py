@@ -96,6 +96,38 @@ class StepEvents(ctypes.Structure):
 _lib = None
 
 
+def _configure(lib: ctypes.CDLL) -> ctypes.CDLL:
+    P, i32, i64, sz, f32 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t,
+                            ctypes.c_float)
+    lib.adapld_tree_nodes.argtypes = [P]
+    lib.adapld_tree_nodes.restype = i32
+    lib.adapld_workspace_bytes.argtypes = [i32, i64, i32, P]
+    lib.adapld_workspace_bytes.restype = sz
+    lib.adapld_status_string.argtypes = [ctypes.c_int]
+    lib.adapld_status_string.restype = ctypes.c_char_p
+    lib.adapld_lexical_match.argtypes = [P, i64, P, i32, i32, i32, P, P, P, P, P, sz, P]
+    lib.adapld_semantic_topk.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P, P, P, sz, P]
+    lib.adapld_build_draft_tree.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, i32, P,
+                                            P, P, P, P, sz, P]
+    lib.adapld_step.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P]
+    lib.adapld_step_ex.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P, P, P]
+    lib.adapld_embedding_topk.argtypes = [P, i64, P, P, P, i32, i32, f32, P, P, P, P, P, sz, P]
+    lib.adapld_read_device_status.argtypes = [P, P, P]
+    lib.adapld_semantic_topk_static.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P, P, P]
+    lib.adapld_semantic_topk_static_status.argtypes = [P, P]
+    lib.adapld_accept_greedy.argtypes = [P, i32, P, P, P, i32, i32, P, P, P, P, i64, P, P, P,
+                                         i32, P, P, P, sz, P]
+    lib.adapld_step_from_host.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, P, P, P, sz,
+                                          P]
+    for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
+              "adapld_step", "adapld_step_ex", "adapld_read_device_status",
+              "adapld_semantic_topk_static", "adapld_embedding_topk",
+              "adapld_accept_greedy", "adapld_step_from_host",
+              "adapld_semantic_topk_static_status"):
+        getattr(lib, f).restype = ctypes.c_int
+    return lib
+
+
 def load() -> ctypes.CDLL:
     """Loads the CUDA library; raises if it has not been built."""
     global _lib
@@ -104,40 +136,16 @@ def load() -> ctypes.CDLL:
             raise RuntimeError(
                 f"{LIB_PATH} is missing: build it first (python -c 'import __graft_entry__ as g; "
                 "g.build()'); there is no CPU fallback")
-        lib = ctypes.CDLL(LIB_PATH)
-        P, i32, i64, sz, f32 = (ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t,
-                                ctypes.c_float)
-        lib.adapld_tree_nodes.argtypes = [P]
-        lib.adapld_tree_nodes.restype = i32
-        lib.adapld_workspace_bytes.argtypes = [i32, i64, i32, P]
-        lib.adapld_workspace_bytes.restype = sz
-        lib.adapld_status_string.argtypes = [ctypes.c_int]
-        lib.adapld_status_string.restype = ctypes.c_char_p
-        lib.adapld_lexical_match.argtypes = [P, i64, P, i32, i32, i32, P, P, P, P, P, sz, P]
-        lib.adapld_semantic_topk.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P, P, P, sz,
-                                             P]
-        lib.adapld_build_draft_tree.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, i32, P,
-                                                P, P, P, P, sz, P]
-        lib.adapld_step.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P]
-        lib.adapld_step_ex.argtypes = [P, i64, P, P, i32, P, P, i32, i32, P, P, P, sz, P, P, P]
-        lib.adapld_embedding_topk.argtypes = [P, i64, P, P, P, i32, i32, f32, P, P, P, P, P, sz,
-                                              P]
-        lib.adapld_read_device_status.argtypes = [P, P, P]
-        lib.adapld_semantic_topk_static.argtypes = [P, i64, i32, P, P, P, i32, i32, f32, P, P,
-                                                    P, P]
-        lib.adapld_semantic_topk_static_status.argtypes = [P, P]
-        lib.adapld_accept_greedy.argtypes = [P, i32, P, P, P, i32, i32, P, P, P, P, i64, P, P,
-                                             P, i32, P, P, P, sz, P]
-        lib.adapld_step_from_host.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, P, P, P,
-                                              sz, P]
-        for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
-                  "adapld_step", "adapld_step_ex", "adapld_read_device_status",
-                  "adapld_semantic_topk_static", "adapld_embedding_topk",
-                  "adapld_accept_greedy", "adapld_step_from_host",
-                  "adapld_semantic_topk_static_status"):
-            getattr(lib, f).restype = ctypes.c_int
-        _lib = lib
+        _lib = _configure(ctypes.CDLL(LIB_PATH))
     return _lib
+
+
+def load_library(path: str) -> ctypes.CDLL:
+    """Another build of the library (e.g. the checked debug build), configured
+    like the default one; not cached."""
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing; there is no CPU fallback")
+    return _configure(ctypes.CDLL(path))
 
 
 def status_string(code: int) -> str:

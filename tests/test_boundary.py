@@ -39,6 +39,14 @@ def test_library_exports_every_declared_symbol(lib):
         assert hasattr(lib, name), name
 
 
+def test_checked_build_exports_every_declared_symbol():
+    """The checked debug build (every kernel index tested) has the same ABI."""
+    chk = native.load_library(build.build(checked=True))
+    for name in declared_functions():
+        assert hasattr(chk, name), name
+    assert chk.adapld_status_string(-9) == native.load().adapld_status_string(-9)
+
+
 def test_status_strings(lib):
     for code in (0, -1, -2, -3, -4, -5, -6, -7, -8, -9, -10, -11, -12, -13, -14, -15, -16, -17,
                  -20):
