@@ -2,20 +2,26 @@
 // n-gram).
 //
 // Grid (X, B), 512 threads; the X CTAs of a sequence form one thread-block
-// cluster (X <= 8, or 16 for a few long sequences).  CTA x scans a contiguous range of
-// 8192-position chunks, most recent chunk first.  A chunk and its n_max-1
-// token halo are staged in shared memory with 16-byte cp.async copies (4-byte
-// copies for the unaligned head and tail), the next chunk's copies in flight
-// while the current one is scanned.  For each position j the backward match
-// length m(j) = #{i : M[j-i'] == M[len-1-i'] for all i' <= i}, capped at
-// min(n_max, len-1), is computed: one comparison with the anchor token for
-// every position, extended only where it matches.  The chunk maximum and the
-// positions reaching it, most recent first, are ranked with warp ballots and
-// one scan over (block, warp) cells.  The CTA keeps the best length over its
-// chunks and its k most recent positions.  The cluster then merges its CTAs'
-// results through distributed shared memory (CTA rank 0 reads them; ranks hold
-// contiguous ranges, higher ranks more recent): n* = max m, candidates = the
-// k most recent positions with m(j) = n*.  No global ticket, no counters.
+// cluster (X <= 8, or 16 for a few long sequences).  CTA x scans a contiguous
+// range of 8192-position chunks, most recent chunk first; thread t of a chunk
+// owns the 16 consecutive positions j0 + 16 t .. j0 + 16 t + 15.  Each thread
+// loads its window -- its 16 tokens and the 8 before them -- from global
+// memory into registers (16-byte loads where the row is aligned); the window
+// of the CTA's most recent chunk is requested before the sequence length
+// arrives (it is at the same place whatever the length), so the two round
+// trips overlap.  For each position j the backward match length
+// m(j) = #{i : M[j-i'] == M[len-1-i'] for all i' <= i}, capped at
+// min(n_max, len-1), is built as bit masks over the thread's 16 positions:
+// the positions matching the anchor token, then those of them whose next
+// older token matches too, and so on while any is left.  A warp reduces its
+// maximum and the count of its positions reaching it, scanned from the top
+// lane; after one CTA barrier every thread knows the chunk maximum and where
+// its own hits rank, most recent first, and writes them straight into the
+// CTA's running result (a longer match replaces it, an equal one appends).
+// With several CTAs each one then pushes its result into the shared memory
+// of CTA rank 0 (distributed shared memory), and after one cluster barrier
+// rank 0 merges them locally: n* = max m, candidates = the k most recent
+// positions with m(j) = n* (higher ranks hold more recent chunks).
 //
 // On the step path the kernel also zeroes the workspace counters of the
 // step's later kernels, so a step needs no memset, and it is launched as a
@@ -31,8 +37,11 @@ namespace adapld {
 namespace {
 
 constexpr int kWarpsL = kThreadsL / 32;
-constexpr int kPerThreadL = kChunkL / kThreadsL;  // positions per thread and chunk (16)
-constexpr int kBufL = kChunkL + 16;               // chunk + halo (<= 7) + alignment (<= 3)
+constexpr int kPerThreadL = kChunkL / kThreadsL;  // consecutive positions per thread (16)
+constexpr int kHaloL = 8;                         // tokens before them (n_max - 1 <= 7 used)
+constexpr int kWinL = kHaloL + kPerThreadL;       // window of a thread (24 tokens)
+constexpr int kResL = 2 + kMaxK;                  // a CTA's result: m, count, positions
+static_assert(kPerThreadL == 16 && kWinL % 4 == 0, "16 positions, whole 16-byte groups");
 
 struct LexArgs {
     LexLaunch p;
@@ -40,47 +49,58 @@ struct LexArgs {
     int q;  // chunks per CTA
 };
 
-// Stages tokens M[j0-h .. j1) (indices below 0 are never read and are not
-// copied) into buf, global index i at buf[i - (j0-h) + off], where `off`
-// makes 16-byte aligned global addresses land on 16-byte aligned slots.
-__device__ __forceinline__ int stage_chunk(int *buf, const int32_t *M, int j0, int j1, int h) {
-    const int t = threadIdx.x;
-    const int b0 = j0 - h;
-    const int off = (int)((((uintptr_t)M >> 2) & 3) + b0) & 3;
-    const int gs = max(b0, 0);
-    int f = gs + ((4 - ((gs - b0 + off) & 3)) & 3);  // first 16-byte boundary >= gs
-    int l = j1 - ((j1 - b0 + off) & 3);             // last 16-byte boundary <= j1
-    if (f > j1) f = j1;
-    if (l < f) l = f;
-    const int shift = off - b0;  // buf index of global index i: i + shift
-    for (int v = t; v < (l - f) >> 2; v += kThreadsL)
-        cp_async16(buf + (f + 4 * v + shift), M + f + 4 * v);
-    if (t < f - gs) cp_async4(buf + (gs + t + shift), M + gs + t);
-    if (t >= 32 && t - 32 < j1 - l) cp_async4(buf + (l + (t - 32) + shift), M + l + (t - 32));
-    return off;
+// W[w] = M[base - kHaloL + w] for w < kWinL; entries outside the row [0, lim)
+// read as -1 (positions are bounded separately, so they are never compared).
+__device__ __forceinline__ void load_window(int (&W)[kWinL], const int32_t *M, int base, int lim,
+                                            bool vec) {
+#pragma unroll
+    for (int g = 0; g < kWinL / 4; ++g) {
+        const int i0 = base - kHaloL + 4 * g;
+        if (vec && i0 >= 0 && i0 + 4 <= lim) {
+            const int4 v = __ldg(reinterpret_cast<const int4 *>(M + i0));
+            W[4 * g] = v.x;
+            W[4 * g + 1] = v.y;
+            W[4 * g + 2] = v.z;
+            W[4 * g + 3] = v.w;
+        } else {
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                W[4 * g + u] = (i0 + u >= 0 && i0 + u < lim) ? __ldg(M + i0 + u) : -1;
+        }
+    }
 }
 
 __global__ void __launch_bounds__(kThreadsL, 2) lexical_kernel(LexArgs args) {
     const LexLaunch &a = args.p;
-    extern __shared__ __align__(16) int dyn[];  // [1 or 2][kBufL] staged chunks
-    __shared__ int suf[8];
-    __shared__ int wval[kWarpsL];
-    __shared__ int wcnt[kPerThreadL * kWarpsL];  // hits per (block, warp)
-    __shared__ int wbase[kPerThreadL * kWarpsL]; // hits ranked before each (block, warp)
-    __shared__ int clist[kMaxK];                 // this chunk's ranked positions
-    __shared__ int res[2 + kMaxK];               // this CTA's result: m, count, positions
+    __shared__ int wmax_s[kWarpsL];            // per warp: its longest match in the chunk
+    __shared__ int wtot_s[kWarpsL];            // ... and its positions reaching it
+    __shared__ int res[kResL];                 // this CTA's result
+    __shared__ int mres[kWideClusterL][kResL]; // rank 0: every CTA's result
 
     pdl_wait_then_release();
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const int b = blockIdx.y, x = blockIdx.x, X = gridDim.x;
+    // every CTA of the cluster has started before results are pushed (the
+    // matching wait comes after the scan)
+    if (X > 1) cluster_arrive_relaxed();
+    const int32_t *M = a.tokens + (int64_t)b * a.ld;
+    const bool vec = ((uintptr_t)M & 15) == 0;
+    const int lim = (int)a.ld;
+    // the most recent chunk of this CTA were the sequence full: its window
+    // is requested together with the length
+    const int c_spec = min(x * args.q + args.q, chunks_of(a.ld - 1, kChunkL)) - 1;
+    int W[kWinL];
+    int loaded = -1;
+    if (c_spec >= x * args.q) {
+        load_window(W, M, c_spec * kChunkL + kPerThreadL * t, lim, vec);
+        loaded = c_spec;
+    }
     const int len = a.lengths[b];
     const bool valid = len >= 1 && (int64_t)len <= a.ld;
     const int nj = valid ? len - 1 : 0;  // candidates j in [0, len-2]
     const int top = valid ? min(a.n_max, len - 1) : 0;
-    const int h = top > 0 ? top - 1 : 0;  // halo before a chunk
     const int nchunks = (nj + kChunkL - 1) / kChunkL;
     const int c_lo = x * args.q, c_hi = min(c_lo + args.q, nchunks);
-    const int32_t *M = a.tokens + (int64_t)b * a.ld;
 
     if (a.zero) {  // the later kernels' counters (grid-stride over every thread)
         const size_t nthreads = (size_t)gridDim.x * gridDim.y * kThreadsL;
@@ -88,179 +108,114 @@ __global__ void __launch_bounds__(kThreadsL, 2) lexical_kernel(LexArgs args) {
             a.zero[i] = 0;
     }
     if (a.stats && b == 0 && x == 0 && t < 4) a.stats[t] = 0;
-    if (t == 0) {
-        res[0] = 0;
-        res[1] = 0;
-    }
-    if (t < top) suf[t] = M[len - 1 - t];
-
-    int off = 0;
-    if (c_hi > c_lo && top > 0) {
-        const int jc = (c_hi - 1) * kChunkL;
-        off = stage_chunk(dyn, M, jc, min(jc + kChunkL, nj), h);
-        cp_async_commit();
-    }
-    for (int c = c_hi - 1, i = 0; c >= c_lo && top > 0; --c, ++i) {
-        const int j0 = c * kChunkL, j1 = min(j0 + kChunkL, nj);
-        const int *tok = dyn + (i & 1) * kBufL;
-        const int shift = off - (j0 - h);  // tok[p + shift] = M[p]
-        int next_off = 0;
-        if (c - 1 >= c_lo) {  // the next (older) chunk's copies fly during this scan
-            const int jn = (c - 1) * kChunkL;
-            next_off = stage_chunk(dyn + ((i + 1) & 1) * kBufL, M, jn, jn + kChunkL, h);
-            cp_async_commit();
-            cp_async_wait_group<1>();
-        } else {
-            cp_async_wait_group<0>();
-        }
-        __syncthreads();  // the staged chunk and the suffix are visible
-
-        // match lengths (<= 8) of this thread's 16 positions, 4 bits each: one
-        // comparison with the anchor token per position, extended backwards
-        // only where it matches
-        const int s0 = suf[0];
-        uint32_t first = 0;
+    int suf[8];  // the suffix, most recent token first (broadcast loads)
 #pragma unroll
-        for (int e = 0; e < kPerThreadL; ++e) {
-            const int p = j0 + e * kThreadsL + t;
-            if (p < j1 && tok[p + shift] == s0) first |= 1u << e;
+    for (int i = 0; i < 8; ++i) suf[i] = i < top ? __ldg(M + len - 1 - i) : 0;
+
+    int rm = 0, rn = 0;  // the CTA's best length so far and its positions (same in every thread)
+    for (int c = c_hi - 1; c >= c_lo && top > 0; --c) {
+        const int base = c * kChunkL + kPerThreadL * t;
+        if (c != loaded) {
+            load_window(W, M, base, lim, vec);
+            loaded = c;
         }
-        uint64_t mpack = 0;
-        int mymax = 0;
-        for (uint32_t f = first; f; f &= f - 1) {
-            const int e = __ffs(f) - 1;
-            const int p = j0 + e * kThreadsL + t;
-            int mm = 1;
-            while (mm < top && p - mm >= 0 && tok[p - mm + shift] == suf[mm]) ++mm;
-            mpack |= (uint64_t)mm << (4 * e);
-            mymax = max(mymax, mm);
+        // al: positions whose last i + 1 tokens match the suffix; hits: the
+        // longest such set met, of length mymax
+        uint32_t al = 0;
+#pragma unroll
+        for (int e = 0; e < kPerThreadL; ++e)
+            al |= (uint32_t)(base + e < nj && W[kHaloL + e] == suf[0]) << e;
+        uint32_t hits = al;
+        int mymax = al ? 1 : 0;
+#pragma unroll
+        for (int i = 1; i < 8; ++i) {
+            if (i >= top || al == 0) break;
+            uint32_t eq = 0;
+#pragma unroll
+            for (int e = 0; e < kPerThreadL; ++e)
+                eq |= (uint32_t)(W[kHaloL + e - i] == suf[i]) << e;
+            if (base == 0) eq &= ~((1u << i) - 1u);  // positions j < i have no token j - i
+            al &= eq;
+            if (al) {
+                hits = al;
+                mymax = i + 1;
+            }
         }
-        mymax = warp_max_i(mymax);
-        if (lane == 0) wval[warp] = mymax;
+        // rank most recent first: higher warps, then higher lanes, then
+        // higher positions of a thread
+        const int wmax = warp_max_i(mymax);
+        const int mine = (wmax > 0 && mymax == wmax) ? __popc(hits) : 0;
+        int incl = mine;  // over this lane and the higher ones
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_down_sync(0xffffffffu, incl, o);
+            if (lane + o < 32) incl += u;
+        }
+        if (lane == 0) {
+            wmax_s[warp] = wmax;
+            wtot_s[warp] = incl;
+        }
         __syncthreads();
         int cmax = 0;
 #pragma unroll
-        for (int w = 0; w < kWarpsL; ++w) cmax = max(cmax, wval[w]);
-        int ccnt = 0;
-        if (cmax > 0) {
-            uint32_t hits = 0;
-            for (uint32_t f = first; f; f &= f - 1) {
-                const int e = __ffs(f) - 1;
-                if ((int)((mpack >> (4 * e)) & 15u) == cmax) hits |= 1u << e;
-            }
-            auto hit = [&](int e) { return ((hits >> e) & 1u) != 0; };
-            // most recent first: position blocks e from the top, within a
-            // block higher warps and then higher lanes first.  The hits per
-            // (block, warp) are counted, scanned once in that order, and each
-            // hit's rank is its (block, warp) offset plus the hits of the
-            // higher lanes of its warp.
+        for (int w = 0; w < kWarpsL; ++w) cmax = max(cmax, wmax_s[w]);
+        int before = 0, total = 0;  // the chunk's hits in higher warps / in all
 #pragma unroll
-            for (int e = 0; e < kPerThreadL; ++e) {
-                const unsigned bal = __ballot_sync(0xffffffffu, hit(e));
-                if (lane == 0) wcnt[e * kWarpsL + warp] = __popc(bal);
-            }
-            __syncthreads();
-            constexpr int kCells = kPerThreadL * kWarpsL;  // 256 (block, warp) cells
-            static_assert(kCells <= kThreadsL && kCells % 32 == 0, "one cell per thread");
-            int v = 0, cell = 0;
-            if (t < kCells) {
-                const int e = kPerThreadL - 1 - t / kWarpsL, w = kWarpsL - 1 - t % kWarpsL;
-                cell = e * kWarpsL + w;
-                v = wcnt[cell];
-            }
-            int incl = v;
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int u = __shfl_up_sync(0xffffffffu, incl, o);
-                if (lane >= o) incl += u;
-            }
-            if (t < kCells && lane == 31) wval[warp] = incl;  // (cmax is already read)
-            __syncthreads();
-            int before = 0, total = 0;
-#pragma unroll
-            for (int w = 0; w < kCells / 32; ++w) {
-                const int x = wval[w];
-                before += w < warp ? x : 0;
-                total += x;
-            }
-            if (t < kCells) wbase[cell] = before + incl - v;
-            __syncthreads();
-#pragma unroll
-            for (int e = 0; e < kPerThreadL; ++e) {
-                const bool mine = hit(e);
-                const unsigned bal = __ballot_sync(0xffffffffu, mine);
-                const unsigned higher = lane == 31 ? 0u : (bal & (0xffffffffu << (lane + 1)));
-                const int rank = wbase[e * kWarpsL + warp] + __popc(higher);
-                if (mine && rank < a.k) clist[rank] = j0 + e * kThreadsL + t;
-            }
-            ccnt = min(total, a.k);
+        for (int w = 0; w < kWarpsL; ++w) {
+            const int n = wmax_s[w] == cmax ? wtot_s[w] : 0;
+            total += n;
+            before += w > warp ? n : 0;
         }
-        __syncthreads();  // clist complete
-        // fold the chunk into the CTA's result (chunks arrive most recent first)
-        if (warp == 0 && cmax > 0) {
-            const int rm = res[0], rn = res[1];
-            __syncwarp();
-            if (cmax > rm) {
-                if (lane < ccnt) res[2 + lane] = clist[lane];
-                if (lane == 0) {
-                    res[0] = cmax;
-                    res[1] = ccnt;
+        if (cmax > 0 && cmax >= rm) {  // a longer match replaces the result, an equal one appends
+            const int off = cmax > rm ? 0 : rn;
+            const int room = a.k - off;
+            if (wmax == cmax && mine > 0) {
+                int r = before + incl - mine;
+                for (uint32_t h = hits; h && r < room; ++r) {
+                    const int e = 31 - __clz(h);
+                    h &= ~(1u << e);
+                    res[2 + off + r] = base + e;
                 }
-            } else if (cmax == rm) {
-                const int add = min(ccnt, a.k - rn);
-                if (lane < add) res[2 + rn + lane] = clist[lane];
-                if (lane == 0) res[1] = rn + add;
             }
+            rn = off + min(total, room);
+            rm = cmax;
         }
-        __syncthreads();  // before the buffers, wval, wcnt and clist are reused
-        off = next_off;
+        __syncthreads();  // res is complete; wmax_s and wtot_s may be rewritten
     }
 
-    // ---- the sequence's result: CTA rank 0 merges the cluster's CTAs ---------
+    // ---- the sequence's result ------------------------------------------------
     int32_t *cb = a.cand + (int64_t)b * a.k;
-    if (X == 1) {
-        __syncthreads();
+    int best = rm, total = rm > 0 ? rn : 0;
+    if (X > 1) {
+        cluster_wait();  // every CTA has started
         if (warp == 0) {
-            const int best = res[0];
-            const int total = best > 0 ? res[1] : 0;
-            if (lane < a.k) cb[lane] = lane < total ? res[2 + lane] : -1;
-            if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
-            if (lane == 0) {
-                a.match_n[b] = best;
-                a.n_cand[b] = total;
-                a.hit_kind[b] = best > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
-                if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
-            }
+            if (lane == 0) st_cluster_i32(&mres[x][0], 0, rm);
+            if (lane == 1) st_cluster_i32(&mres[x][1], 0, rn);
+            if (lane < rn) st_cluster_i32(&mres[x][2 + lane], 0, res[2 + lane]);
         }
-    } else {
-        // every CTA's result is in its shared memory (warp 0 wrote it)
-        if (warp == 0)
-            cluster_sync_all();
-        else
-            cluster_sync_relaxed();
-        if (x == 0 && warp == 0) {
-            int best = lane < X ? ld_cluster_i32(&res[0], lane) : 0;
+        cluster_sync_all();  // the pushes are visible to rank 0
+        if (x != 0) return;
+        if (warp == 0) {
+            best = lane < X ? mres[lane][0] : 0;
             best = warp_max_i(best);
-            int total = 0;
-            if (best > 0) {
+            total = 0;
+            if (best > 0)
                 total = warp_merge_desc(
-                    X, a.k,
-                    [&](int r) {
-                        return ld_cluster_i32(&res[0], r) == best ? ld_cluster_i32(&res[1], r)
-                                                                  : 0;
-                    },
-                    [&](int r, int i) { return ld_cluster_i32(&res[2 + i], r); }, cb);
-            }
-            if (lane >= total && lane < a.k) cb[lane] = -1;
-            if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
-            if (lane == 0) {
-                a.match_n[b] = best;
-                a.n_cand[b] = total;
-                a.hit_kind[b] = best > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
-                if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
-            }
+                    X, a.k, [&](int r) { return mres[r][0] == best ? mres[r][1] : 0; },
+                    [&](int r, int i) { return mres[r][2 + i]; }, cb);
         }
-        cluster_sync_relaxed();  // the CTAs' shared memory stays until rank 0 has read it
+    } else if (warp == 0 && lane < total) {
+        cb[lane] = res[2 + lane];
+    }
+    if (warp == 0) {
+        if (lane >= total && lane < a.k) cb[lane] = -1;
+        if (a.score && lane < a.k) a.score[(int64_t)b * a.k + lane] = 0.f;
+        if (lane == 0) {
+            a.match_n[b] = best;
+            a.n_cand[b] = total;
+            a.hit_kind[b] = best > 0 ? ADAPLD_HIT_LEX : ADAPLD_HIT_NONE;
+            if (a.status) a.status[b] = valid ? 0 : ADAPLD_SEQ_BAD_LENGTH;
+        }
     }
 }
 
@@ -311,10 +266,7 @@ cudaError_t launch_lexical(const LexLaunch &a, const Workspace &ws, cudaStream_t
     const int X = chunks < xmax ? chunks : xmax;
     const int q = (chunks + X - 1) / X;
     LexArgs args{a, ws, q};
-    const size_t smem = sizeof(int) * (size_t)kBufL * (q > 1 ? 2 : 1);
-    cudaError_t e = cudaFuncSetAttribute(lexical_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
     if (X > 8) {
         e = cudaFuncSetAttribute(lexical_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
@@ -322,7 +274,7 @@ cudaError_t launch_lexical(const LexLaunch &a, const Workspace &ws, cudaStream_t
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(X, a.B);
     cfg.blockDim = dim3(kThreadsL);
-    cfg.dynamicSmemBytes = smem;
+    cfg.dynamicSmemBytes = 0;
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
