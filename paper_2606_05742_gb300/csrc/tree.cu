@@ -361,56 +361,82 @@ __device__ __forceinline__ void warp_sort_desc(int *s_cand, float *s_score, int 
 // The k most recent positions p in [lo, hi) with M[p] == br[w], for every
 // branch w < nb, most recent first: store(w, rank, p) for rank < k, then
 // count(w, c) once per branch (by thread w) with c = their number (<= k);
-// s_tok[p - p0] holds M[p].  Block-wide (every thread).  The range is split
-// into one contiguous part per warp (higher warps more recent), so all 16
-// warps scan at once: a first pass counts each warp's matches per branch (wc:
-// 16 * nb ints of scratch), a second stores each warp's matches at ranks
-// after those of the warps above it, until k.
+// s_tok[p - p0] holds M[p] and hi - lo <= 16 * kThreads4.  Block-wide (every
+// thread).  Thread t owns the consecutive positions lo + pt t .. + pt - 1
+// (pt <= 16) and keeps their tokens in registers; per branch it forms the bit
+// mask of its matches, a warp with any match scans the counts from its top
+// lane, and the warps' totals (wc: 16 * nb ints of scratch) give, after one
+// CTA barrier per four branches, every match its rank: higher warps, then
+// higher lanes, then higher positions first.
 template <class Store, class Count>
 __device__ __forceinline__ void scan_branches(const int *s_tok, int64_t p0, int64_t lo,
                                               int64_t hi, const int *br, int nb, int k, int *wc,
                                               Store store, Count count) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    constexpr int NW = kThreads4 / 32, U4 = 4;
-    const int64_t n = hi > lo ? hi - lo : 0;
-    const int64_t per = (n + NW * 32 * U4 - 1) / (NW * 32 * U4) * (32 * U4);  // per warp
-    const int64_t wlo = lo + warp * per;
-    const int64_t whi = min(wlo + per, hi);
-    const int groups = whi > wlo ? (int)((whi - wlo + 31) / 32) : 0;  // a multiple of U4
-                                                                       // unless clipped
-    for (int w = 0; w < nb; ++w) {
-        const int bt = br[w];
-        int c = 0;
-        for (int g = 0; g < groups; g += U4) {  // U4 independent loads per step
-            int tk[U4];
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    constexpr int NW = kThreads4 / 32, PT = 16, NBC = 4;  // branches per pass
+    const int n = hi > lo ? (int)(hi - lo) : 0;
+    const int pt = (n + kThreads4 - 1) / kThreads4;  // <= PT
+    const int q0 = (int)(lo - p0) + pt * t;          // s_tok index of the first position
+    const int cnt = max(0, min(pt, n - pt * t));     // positions of this thread
+    int tk[PT];
+    if (cnt == PT && (q0 & 3) == 0) {
 #pragma unroll
-            for (int u = 0; u < U4; ++u) {
-                const int64_t p = wlo + 32 * (g + u) + lane;
-                tk[u] = p < whi ? s_tok[p - p0] : ~bt;
+        for (int g = 0; g < PT / 4; ++g) {
+            const int4 v = *reinterpret_cast<const int4 *>(s_tok + q0 + 4 * g);
+            tk[4 * g] = v.x;
+            tk[4 * g + 1] = v.y;
+            tk[4 * g + 2] = v.z;
+            tk[4 * g + 3] = v.w;
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < PT; ++e) tk[e] = e < cnt ? s_tok[q0 + e] : 0;
+    }
+    const uint32_t valid = (1u << cnt) - 1u;  // cnt <= 16
+    for (int w0 = 0; w0 < nb; w0 += NBC) {
+        uint32_t m[NBC];
+        int excl[NBC];  // matches of the higher lanes of this warp
+#pragma unroll
+        for (int j = 0; j < NBC; ++j) {
+            m[j] = 0;
+            excl[j] = 0;
+            if (w0 + j >= nb) continue;
+            const int bt = br[w0 + j];
+#pragma unroll
+            for (int e = 0; e < PT; ++e) m[j] |= (uint32_t)(tk[e] == bt) << e;
+            m[j] &= valid;
+            int tot = 0;
+            if (__any_sync(0xffffffffu, m[j] != 0)) {
+                const int c = __popc(m[j]);
+                int incl = c;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int u = __shfl_down_sync(0xffffffffu, incl, o);
+                    if (lane + o < 32) incl += u;
+                }
+                excl[j] = incl - c;
+                tot = __shfl_sync(0xffffffffu, incl, 0);
             }
+            if (lane == 0) wc[warp * nb + w0 + j] = tot;
+        }
+        __syncthreads();
 #pragma unroll
-            for (int u = 0; u < U4; ++u) c += __popc(__ballot_sync(0xffffffffu, tk[u] == bt));
-        }
-        if (lane == 0) wc[warp * nb + w] = c;
-    }
-    __syncthreads();
-    for (int w = 0; w < nb; ++w) {
-        int off = 0;
-        for (int u = warp + 1; u < NW; ++u) off += wc[u * nb + w];
-        if (off >= k || wc[warp * nb + w] == 0) continue;
-        const int bt = br[w];
-        for (int g = groups - 1; g >= 0 && off < k; --g) {
-            const int64_t p = wlo + 32 * g + lane;
-            const unsigned m = __ballot_sync(0xffffffffu, p < whi && s_tok[p - p0] == bt);
-            const int rank = off + __popc((m >> lane) >> 1);  // higher lanes are more recent
-            if (((m >> lane) & 1u) && rank < k) store(w, rank, (int)p);
-            off += __popc(m);
+        for (int j = 0; j < NBC; ++j) {
+            if (m[j] == 0) continue;
+            const int w = w0 + j;
+            int off = excl[j];
+            for (int u = warp + 1; u < NW; ++u) off += wc[u * nb + w];
+            for (uint32_t h = m[j]; h && off < k; ++off) {
+                const int e = 31 - __clz(h);
+                h &= ~(1u << e);
+                store(w, off, (int)(lo + pt * t + e));
+            }
         }
     }
-    if ((int)threadIdx.x < nb) {
+    if (t < nb) {
         int total = 0;
-        for (int u = 0; u < NW; ++u) total += wc[u * nb + threadIdx.x];
-        count((int)threadIdx.x, min(total, k));
+        for (int u = 0; u < NW; ++u) total += wc[u * nb + t];
+        count(t, min(total, k));
     }
 }
 
@@ -973,11 +999,14 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
 //       (Eq. 6-7) over the cluster's warps; rank 0 collects the scores and
 //       every CTA sorts them alike;
 //   P2  every CTA derives the branch set (Eq. 10-11);
-//   P3  each CTA scans its slice for the branch tokens, a warp per branch,
-//       keeping the k most recent occurrences;
+//   P3  each CTA scans its slice for the branch tokens (every thread 16
+//       consecutive positions held in registers, a bit mask per branch),
+//       keeping the k most recent occurrences, and writes its lists into
+//       every CTA's shared memory (or, when X * W * (k + 1) ints exceed
+//       32 KB, leaves them in its own);
 //   P4  after a cluster barrier every CTA merges the slices' lists (ranks
-//       hold contiguous slices, higher ranks more recent) from the other
-//       CTAs' shared memory;
+//       hold contiguous slices, higher ranks more recent) from its own
+//       shared memory (or the other CTAs');
 //   P5  the scored rows (successor candidates against R[j*+1], Eq. 13, or
 //       the lexical candidates against the query, Eq. 6) are spread over the
 //       cluster's warps, one row per warp; each score and the token after
@@ -986,6 +1015,8 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_kernel(TreeArg
 //       successor (Eq. 14) and writes the tree.
 // Every CTA passes every cluster barrier (no early exit before them); the
 // barriers' conditions depend only on the sequence, hence agree in a cluster.
+// A first cluster barrier, arrived at on entry and waited for in P1, makes
+// sure every CTA has started before any writes another's shared memory.
 // A scored row is split into parts of 4096 elements (512 16-byte chunks,
 // one batch of loads at U = 16), each part one warp's work item, so a warp
 // waits for at most one batch of row loads per item.
@@ -993,10 +1024,18 @@ constexpr int kPartCh = 512;
 __host__ __device__ inline int row_parts(int d) { return ((d >> 3) + kPartCh - 1) / kPartCh; }
 
 struct ClusterLayout {
-    uint32_t tok, cnt, lst, mcnt, mlst, wc, sc, tk, pd, ps, total;
+    uint32_t tok, cnt, lst, mcnt, mlst, wc, sc, tk, pd, ps, gath, total;
 };
 
-__host__ __device__ inline ClusterLayout cluster_layout(int d, int span, int W, int k, int T) {
+// Bytes of the lists every CTA pushes into every other (X CTAs x W branches x
+// (count + k positions)); above this they are read remotely instead.
+constexpr size_t kPushBytes = 32 * 1024;
+__host__ __device__ inline size_t push_bytes(int X, int W, int k) {
+    return 4 * (size_t)X * W * (1 + k);
+}
+
+__host__ __device__ inline ClusterLayout cluster_layout(int d, int span, int W, int k, int T,
+                                                       int X) {
     ClusterLayout L;
     size_t o = align_up((size_t)d * 2, 16);  // the reference vector (bf16)
     L.tok = (uint32_t)o;
@@ -1020,6 +1059,8 @@ __host__ __device__ inline ClusterLayout cluster_layout(int d, int span, int W, 
     o += 4 * (size_t)T * P;
     L.ps = (uint32_t)o;  // rank 0: partial |row|^2 per (task, part)
     o += 4 * (size_t)T * P;
+    L.gath = (uint32_t)o;  // every CTA's lists, [X][W][1 + k] (when pushed)
+    if (push_bytes(X, W, k) <= kPushBytes) o += push_bytes(X, W, k);
     L.total = (uint32_t)o;
     return L;
 }
@@ -1037,7 +1078,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
     __shared__ TreeSmem sm;
     extern __shared__ __align__(16) uint8_t dyn[];
     const int k = a.p.k, d = a.d, W = a.p.branch_width;
-    const ClusterLayout L = cluster_layout(d, args.span, W, k, args.T);
+    const ClusterLayout L = cluster_layout(d, args.span, W, k, args.T, gridDim.x);
     uint16_t *s_ref = (uint16_t *)dyn;
     int *s_tok = (int *)(dyn + L.tok);
     int *s_cnt = (int *)(dyn + L.cnt);
@@ -1045,6 +1086,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
     int *s_mcnt = (int *)(dyn + L.mcnt);
     int *s_mlst = (int *)(dyn + L.mlst);
     int *s_wc = (int *)(dyn + L.wc);
+    int *s_gath = (int *)(dyn + L.gath);
     float *s_sc = (float *)(dyn + L.sc);
     int *s_tk = (int *)(dyn + L.tk);
     float *s_pd = (float *)(dyn + L.pd);
@@ -1060,6 +1102,9 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
     const int32_t *M = a.tokens + (int64_t)b * a.ld;
     const uint16_t *R = a.reps + (int64_t)b * a.ld * d;
     pdl_wait_then_release();
+    // every CTA of the cluster has started before another writes its shared
+    // memory (the wait is in P1)
+    cluster_arrive_relaxed();
 
     // ---- P0: the slice [p0, p0 + span] (clipped at ld) while the outcome is read
     const int64_t p0 = (int64_t)x * args.span;
@@ -1095,6 +1140,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
 
     // ---- P1: the rerank the branch set depends on
     if (rank_first) {
+        cluster_wait();
         const float qss = vec_finish(s_ref, d, s_red_of(sm));
         for (int q = gwarp; q < v.nc; q += gwarps) {
             float dot = 0.f, ss = 0.f;
@@ -1109,6 +1155,7 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
         __syncthreads();
         vec_issue(R + (int64_t)(s_cand[0] + 1) * d, d, s_ref);  // the successor reference
     } else {
+        cluster_wait();
         cp_async_wait_all();
         __syncthreads();  // the slice and the windows are visible
     }
@@ -1127,15 +1174,35 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) tree_cluster_kernel
             },
             [&](int w, int c) { s_cnt[w] = c; });
     }
-    cluster_sync_all();  // every slice's lists are complete
+    // with room for them, this slice's lists go into every CTA's shared
+    // memory (slot x of [X][W][1 + k]) before the barrier, so the merge reads
+    // local memory only
+    const bool push = push_bytes(X, W, k) <= kPushBytes;
+    if (push && v.need_succ) {
+        __syncthreads();  // this CTA's lists are complete
+        const int per = nb * (1 + k);
+        for (int i = t; i < X * per; i += kThreads4) {
+            const int r = i / per, j = i - r * per, w = j / (1 + k), e = j - w * (1 + k);
+            const int val = e == 0 ? s_cnt[w] : s_lst[w * k + e - 1];
+            st_cluster_i32(&s_gath[(x * W + w) * (1 + k) + e], r, val);
+        }
+    }
+    cluster_sync_all();  // every slice's lists are complete (and pushed)
 
     // ---- P4: the successor candidates of each branch, most recent first
     if (v.need_succ) {
         for (int w = warp; w < nb; w += nwarps) {
-            const int total = warp_merge_desc(
-                X, k, [&](int r) { return ld_cluster_i32(&s_cnt[w], r); },
-                [&](int r, int i) { return ld_cluster_i32(&s_lst[w * k + i], r); },
-                s_mlst + w * k);
+            int total;
+            if (push)
+                total = warp_merge_desc(
+                    X, k, [&](int r) { return s_gath[(r * W + w) * (1 + k)]; },
+                    [&](int r, int i) { return s_gath[(r * W + w) * (1 + k) + 1 + i]; },
+                    s_mlst + w * k);
+            else
+                total = warp_merge_desc(
+                    X, k, [&](int r) { return ld_cluster_i32(&s_cnt[w], r); },
+                    [&](int r, int i) { return ld_cluster_i32(&s_lst[w * k + i], r); },
+                    s_mlst + w * k);
             if (lane == 0) s_mcnt[w] = total;
         }
         __syncthreads();
@@ -1279,7 +1346,7 @@ bool cluster_shape(const TreeLaunch &a, int sms, int tasks, int *X, int *span, s
     int sp = (int)((n + x - 1) / x);
     if (sp < 1) sp = 1;
     const size_t dyn =
-        cluster_layout(a.d, sp, a.p.branch_width, a.p.k, tasks).total;
+        cluster_layout(a.d, sp, a.p.branch_width, a.p.k, tasks, x).total;
     if (dyn + sizeof(TreeSmem) > 227 * 1024) return false;
     *X = x;
     *span = sp;
