@@ -312,35 +312,14 @@ def parse_flags(text):
     return flags
 
 
-def step_launches(flags, W, emb, k=32, B=8, ld=131072):
-    """Kernels one step launches (mirrors the launch sequence of adapld_step)."""
-    succ = W > 0 and not (flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"]))
-    semantic = not flags & FLAG_NAMES["no_semantic"]
-    lists = 1 if ld - 1 <= 4096 else 3      # distinct-token list kernels (one chunk: one)
-    n = 1                                   # lexical
-    if semantic:
-        if emb:
-            n += lists + 2                  # lists, gathered pass, expansion
-        else:
-            n += 1 + (1 if B >= 288 else 0)  # semantic (+ the plan for large batches)
-    if succ and not emb and W * k <= 16:
-        n += 1                              # successor scan fused with the tree
-    elif succ:
-        if emb and not semantic:
-            n += lists                      # the lists, built by the tree stage
-        n += 2 + (3 if emb else 0)          # scan, tree (+ backoff plan, gathered pass,
-                                            # expansion)
-    else:
-        n += 1                              # tree
-    return n
-
-
 def algorithmic_bytes(w, g, lengths, tokens, flags=0, emb_dim=None):
     """Bytes the step must move at minimum (no re-reads), per kernel.  With a
-    token-embedding table of dimension emb_dim (two-representation mode) a
-    fallback needs one table row per distinct token of the history (the
-    score depends only on the token) plus one pass over the token ids, and a
-    successor backoff the same for its sequence."""
+    token-embedding table of dimension emb_dim (two-representation mode) the
+    fallback needs one table row per distinct token of the fallback
+    histories and anchors taken together (the score depends only on the
+    token, and a row serves every sequence holding it) plus one pass over
+    each history's ids, and a successor backoff one row per distinct token
+    of its sequence."""
     d, k = w.d, w.k
     hk = g["hit_kind"]
     semantic = not flags & FLAG_NAMES["no_semantic"]
@@ -356,10 +335,10 @@ def algorithmic_bytes(w, g, lengths, tokens, flags=0, emb_dim=None):
         n_active = int(active.sum())
         sem_bytes = (sem_rows * d * 2 + n_active * d * 2 + 4 * w.B) if semantic else 0
     else:
-        sem_bytes = 0
-        for b in range(w.B):
-            if active[b] and lengths[b] >= 2:
-                sem_bytes += (distinct(b) + 1) * emb_dim * 2 + 4 * int(lengths[b])
+        fb = [b for b in range(w.B) if active[b] and lengths[b] >= 2]
+        union = (np.unique(np.concatenate([tokens[b, : int(lengths[b])] for b in fb])).size
+                 if fb else 0)
+        sem_bytes = int(union) * emb_dim * 2 + sum(4 * int(lengths[b]) for b in fb)
         sem_bytes += 4 * w.B if semantic else 0
     # tree kernel: rerank rows + query for lexical hits, successor scan + rows
     succ_on = w.W > 0 and not flags & (FLAG_NAMES["no_succ"] | FLAG_NAMES["no_branch"])
@@ -452,10 +431,12 @@ def run_native(args):
         clocks.start()
         time.sleep(0.3)
     call = eng.bind(w.tokens, w.lengths, w.reps, w.query, emb=emb, stream=stream)
+    launches0 = native.kernel_launches()
     start.record(stream)
     for i in range(K):
         call()
     end.record(stream)
+    launches = native.kernel_launches() - launches0  # counted by the library
     torch.cuda.synchronize(dev)
     barrier()
     total_ms = start.elapsed_time(end)
@@ -612,7 +593,7 @@ def run_native(args):
         "cpu_baseline": cpu,
         "e2e": e2e,
         "verify": verify,
-        "gpu_launches": step_launches(flags, w.W, emb is not None, w.k, w.B, w.ld) * K,
+        "gpu_launches": launches,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)

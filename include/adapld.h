@@ -401,6 +401,14 @@ int adapld_semantic_topk_static(const uint16_t *reps, int64_t ld, int32_t d,
  * Errors: ADAPLD_ERR_NULL, ADAPLD_ERR_CUDA. */
 int adapld_semantic_topk_static_status(int32_t *status, adapld_stream_t stream);
 
+/* The number of CUDA kernels the library has enqueued in this process since it
+ * was loaded, over every entry point, stream and device (an atomic counter;
+ * any host thread may read it).  The difference of two readings is the
+ * number of kernels the calls between them launched -- a measurement aid
+ * (e.g. to count the launches of a timed region).  Never fails.  The paper
+ * has no counterpart. */
+unsigned long long adapld_kernel_launches(void);
+
 /*
  * Greedy verification of the draft trees and the append to the memory
  * (Sec. 3.6; Appendix C, Eq. 16: at temperature 0 a draft token is accepted

@@ -1,6 +1,7 @@
 // C ABI of the library (include/adapld.h): argument validation, workspace
 // layout and stream-ordered kernel launches.  No entry point allocates memory
 // or synchronises the host (except adapld_read_device_status).
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -10,6 +11,8 @@
 using namespace adapld;
 
 namespace {
+
+std::atomic<unsigned long long> g_launches{0};  // kernels enqueued by the library
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA; }
 
@@ -132,15 +135,23 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
     // the distinct tokens of the selected histories and the plan over them,
     // the scores of the distinct tokens, then their positions
+    const bool uni = union_applies(B, ld, emb->dim);  // every table row read once
     DedupeLaunch da{tokens, ld,   lengths, B,       emb->vocab, active, nullptr, status,
                     false,  true, nullptr, true,    k,          cand,   score,   n_cand};
+    da.union_insert = uni;
     ADAPLD_TRY(cuda_status(launch_dedupe(da, w, s)));
-    SemLaunch a{emb->table, ld, emb->dim, nullptr, w.rep_len, active, B, k, tau, cand, score, n_cand,
-                nullptr, true};
-    a.tokens = w.rep_tok;
-    a.vocab = emb->vocab;
-    a.status = status;
-    ADAPLD_TRY(cuda_status(launch_semantic(a, w, s)));
+    if (uni) {
+        UnionLaunch ua{emb->table, emb->vocab, emb->dim, ld,  B,     nullptr, active,
+                       k,          tau,        cand,     score, n_cand, status};
+        ADAPLD_TRY(cuda_status(launch_union(ua, w, s)));
+    } else {
+        SemLaunch a{emb->table, ld, emb->dim, nullptr, w.rep_len, active, B, k, tau, cand, score,
+                    n_cand, nullptr, true};
+        a.tokens = w.rep_tok;
+        a.vocab = emb->vocab;
+        a.status = status;
+        ADAPLD_TRY(cuda_status(launch_semantic(a, w, s)));
+    }
     ExpandLaunch ea{tokens, ld,     lengths, emb->vocab, B, nullptr, nullptr, nullptr, cand,
                     score,  n_cand, k,       k,          nullptr, active, w.xticket};
     return cuda_status(launch_expand(ea, w, s));
@@ -209,13 +220,18 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
         SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
                      out->n_cand, out->hit_kind, true};
         sa.plan_from_outcome = !emb && small_plan;
+        // small batches: the fallback reads each table row of the batch's
+        // union once, scored against every fallback query by the tensor
+        // cores (csrc/union.cu), instead of once per sequence
+        const bool uni = emb && union_applies(B, ld, emb->dim);
         if (emb) {  // Eq. 4 over token embeddings, scored once per distinct token
             // lists for the fallback sequences, and for lexical hits too when
             // those draft successors (their backoff needs them)
             const bool lex_lists = (p->flags & ADAPLD_SUCC_ON_STRICT) != 0;
             DedupeLaunch da{tokens, ld, lengths, B, emb->vocab, nullptr,
-                            lex_lists ? nullptr : out->hit_kind, out->status, true, true,
+                            lex_lists ? nullptr : out->hit_kind, out->status, true, !uni,
                             out->hit_kind, false, p->k, nullptr, nullptr, nullptr};
+            da.union_insert = uni;
             ADAPLD_TRY(cuda_status(launch_dedupe(da, w, s)));
             sa.reps = emb->table;
             sa.d = emb->dim;
@@ -225,7 +241,14 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
             sa.vocab = emb->vocab;
             sa.status = out->status;
         }
-        ADAPLD_TRY(cuda_status(launch_semantic(sa, w, s)));
+        if (uni) {
+            UnionLaunch ua{emb->table, emb->vocab, emb->dim, ld,         B,
+                           out->hit_kind, nullptr,  p->k,     p->tau, out->cand,
+                           out->score,    out->n_cand, out->status};
+            ADAPLD_TRY(cuda_status(launch_union(ua, w, s)));
+        } else {
+            ADAPLD_TRY(cuda_status(launch_semantic(sa, w, s)));
+        }
         if (emb) {
             ExpandLaunch ea{tokens, ld, lengths, emb->vocab, B, nullptr, nullptr, nullptr,
                             out->cand, out->score, out->n_cand, p->k, p->k, out->hit_kind,
@@ -326,6 +349,10 @@ int adapld_accept_greedy(const uint16_t *logits, int32_t V, const int32_t *draft
     return cuda_status(launch_verify(a, w, s));
 }
 
+unsigned long long adapld_kernel_launches(void) {
+    return g_launches.load(std::memory_order_relaxed);
+}
+
 int adapld_read_device_status(const void *ws, int32_t *status, adapld_stream_t stream) {
     if (!ws || !status) return ADAPLD_ERR_NULL;
     cudaStream_t s = (cudaStream_t)stream;
@@ -335,3 +362,8 @@ int adapld_read_device_status(const void *ws, int32_t *status, adapld_stream_t s
 }
 
 }  // extern "C"
+
+cudaError_t adapld::counted(cudaError_t e) {
+    if (e == cudaSuccess) g_launches.fetch_add(1, std::memory_order_relaxed);
+    return e;
+}

@@ -69,8 +69,17 @@ struct Workspace {
     int32_t *rep_cnt;        // [B][C1] distinct tokens per chunk, then chunk offsets
     uint32_t *rep_bits;      // [B][C1][128] one bit per position: latest occurrence
     int32_t *xpart;          // [B*W][S4][kMaxK][kPart4Ints] expansion: per-slice lists
+    // the union of the fallback sequences' distinct tokens (two-representation
+    // mode, small batches: every table row is read once per step, not once per
+    // sequence holding it); NULL where union_enabled() is false
+    uint32_t *uhash;         // [UH] token + 1 (0: empty), after htab (one memset clears both)
+    int32_t *ucount;         // [1]  union tokens (a counter)
+    int32_t *ulist;          // [B * ld] the union's tokens, in no particular order
+    int32_t *rep_pos;        // [B][ld] latest position of each listed token
+    float *score_pos;        // [B][ld] Eq. 4 score of the token whose latest position it is
+    int64_t UH;              // union hash slots (a power of two >= 2 B (ld-1))
     int64_t H;               // hash slots per sequence (a power of two >= 2 (ld-1))
-    size_t htab_bytes;
+    size_t htab_bytes;       // htab and uhash
     size_t counters_bytes;
     size_t total_bytes;
     int C1, S4, W;
@@ -88,6 +97,15 @@ __host__ __device__ inline int64_t hash_slots(int64_t ld) {
     int64_t h = 64;
     while (h < 2 * (ld - 1)) h <<= 1;
     return h;
+}
+
+// The union pass of the two-representation fallback applies to batches of at
+// most 16 sequences (its query slices then fit the stages of 4 KB row slices
+// next to the rows; with more queries the per-sequence lists measured faster)
+// whose positions its hash can hold.
+constexpr int kUnionMaxB = 16;
+__host__ __device__ inline bool union_enabled(int32_t B, int64_t ld) {
+    return B <= kUnionMaxB && (int64_t)B * (ld - 1) <= ((int64_t)1 << 24);
 }
 
 // Lays the workspace out at `base` (NULL: sizing only).
@@ -109,6 +127,7 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     if (p) {
         w.npairs = w.dev_status + 1;
         w.gticket_rep = w.dev_status + 2;
+        w.ucount = w.dev_status + 3;
         w.done2 = w.dev_status + 4;
         w.ticket4 = w.done2 + B;
         w.ticket5 = w.ticket4 + B;
@@ -135,8 +154,15 @@ inline Workspace layout_workspace(void *base, int32_t B, int64_t ld, int32_t W) 
     w.succ_es = (float *)take(sizeof(float) * BW * kMaxK);
     w.vpart = (unsigned long long *)take(sizeof(unsigned long long) * (size_t)B * kMaxNodes);
     w.H = hash_slots(ld);
-    w.htab_bytes = sizeof(unsigned long long) * (size_t)B * w.H;
+    const bool uni = union_enabled(B, ld);
+    w.UH = uni ? hash_slots((int64_t)B * (ld - 1) + 1) : 0;
+    const size_t hbytes = sizeof(unsigned long long) * (size_t)B * w.H;
+    w.htab_bytes = hbytes + sizeof(uint32_t) * (size_t)w.UH;
     w.htab = (unsigned long long *)take(w.htab_bytes);
+    w.uhash = (p && uni) ? (uint32_t *)((char *)w.htab + hbytes) : nullptr;
+    w.ulist = uni ? (int32_t *)take(sizeof(int32_t) * (size_t)B * ld) : nullptr;
+    w.rep_pos = uni ? (int32_t *)take(sizeof(int32_t) * (size_t)B * ld) : nullptr;
+    w.score_pos = uni ? (float *)take(sizeof(float) * (size_t)B * ld) : nullptr;
     w.rep_tok = (int32_t *)take(sizeof(int32_t) * (size_t)B * ld);
     w.rep_len = (int32_t *)take(sizeof(int32_t) * (size_t)B);
     w.rep_cnt = (int32_t *)take(sizeof(int32_t) * (size_t)B * w.C1);
@@ -159,6 +185,21 @@ constexpr bool kChecked = true;
 #else
 constexpr bool kChecked = false;
 #endif
+
+// The table row a token id reads: ids outside [0, vocab) read row 0.
+__device__ __forceinline__ int canon(int tok, int vocab) {
+    return tok >= 0 && tok < vocab ? tok : 0;
+}
+
+// lowbias32, an integer hash published by C. Wellons (hash-prospector).
+__device__ __forceinline__ uint32_t hash32(uint32_t x) {
+    x ^= x >> 16;
+    x *= 0x7feb352du;
+    x ^= x >> 15;
+    x *= 0x846ca68bu;
+    x ^= x >> 16;
+    return x;
+}
 
 // lo <= i < hi (always true in the normal build).
 __device__ __forceinline__ bool idx_ok(int64_t i, int64_t lo, int64_t hi, int32_t *status) {
@@ -502,6 +543,10 @@ __device__ __forceinline__ int warp_max_i(int v) {
 #endif  // __CUDACC__
 
 // ---- host-side launchers (one per kernel) ---------------------------------------
+// Counts a kernel launch that was enqueued (e == cudaSuccess) in the
+// process-wide counter adapld_kernel_launches() reports; returns e.
+cudaError_t counted(cudaError_t e);
+
 // Launches `kern` as a programmatic dependent of the previous kernel in the
 // stream (it must call pdl_wait_then_release before reading that kernel's
 // outputs).
@@ -518,7 +563,7 @@ cudaError_t launch_dependent(void (*kern)(KArgs...), dim3 grid, dim3 block, size
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+    return counted(cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...));
 }
 
 // Streaming multiprocessors of the current device (0 on error).
@@ -643,6 +688,10 @@ struct DedupeLaunch {
     int32_t *cand;
     float *score;
     int32_t *n_cand;
+    // also record each listed token's position (rep_pos) and insert the
+    // tokens of the fallback sequences (hit_kind != LEX when hit_kind is
+    // given, else every selected one) into the union hash
+    bool union_insert = false;
 };
 cudaError_t launch_dedupe(const DedupeLaunch &a, const Workspace &ws, cudaStream_t s);
 
@@ -670,6 +719,31 @@ struct ExpandLaunch {
     int32_t *ticket;         // [P] slices done
 };
 cudaError_t launch_expand(const ExpandLaunch &a, const Workspace &ws, cudaStream_t s);
+
+// The union pass of the two-representation fallback (csrc/union.cu), after
+// the distinct-token lists were built with union_insert: every token of the
+// union is read from the table once and scored against the queries (anchor
+// embeddings) of every fallback sequence that holds it; then each sequence's
+// top-k over its list.  Writes cand (list indices, for the expansion),
+// score, n_cand and, with hit_kind, SEM / NONE for the fallback sequences
+// (hit_kind != LEX; with active instead, the selected ones).
+struct UnionLaunch {
+    const uint16_t *table;   // [vocab][d] bf16
+    int32_t vocab, d;
+    int64_t ld;
+    int32_t B;
+    int32_t *hit_kind;       // step path (nullable)
+    const uint8_t *active;   // standalone selection (NULL = every sequence)
+    int32_t k;
+    float tau;
+    int32_t *cand;
+    float *score;
+    int32_t *n_cand;
+    int32_t *status;         // ADAPLD_SEQ_BAD_TOKEN for an anchor outside the table
+};
+cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t s);
+// Whether the union pass serves a batch of this shape.
+bool union_applies(int32_t B, int64_t ld, int32_t d);
 
 struct VerifyLaunch {
     const uint16_t *logits;  // [B][N][V] bf16

@@ -47,26 +47,18 @@ struct ExpandArgs {
     Workspace ws;
 };
 
-// The table row a token id reads: ids outside [0, vocab) read row 0.
-__device__ __forceinline__ int canon(int tok, int vocab) {
-    return tok >= 0 && tok < vocab ? tok : 0;
-}
-
-// lowbias32, an integer hash published by C. Wellons (hash-prospector).
-__device__ __forceinline__ uint32_t hash32(uint32_t x) {
-    x ^= x >> 16;
-    x *= 0x7feb352du;
-    x ^= x >> 15;
-    x *= 0x846ca68bu;
-    x ^= x >> 16;
-    return x;
-}
-
 __device__ __forceinline__ bool seq_selected(const DedupeLaunch &a, int b, int &len) {
     len = a.lengths[b];
     if (len < 1 || (int64_t)len > a.ld) return false;
     if (a.skip_lex_of && __ldcg(a.skip_lex_of + b) == ADAPLD_HIT_LEX) return false;
     return a.active ? a.active[b] != 0 : true;
+}
+
+// Whether sequence b's distinct tokens join the union pass (the fallback
+// sequences: no lexical hit on the step path; the selected ones otherwise).
+__device__ __forceinline__ bool joins_union(const DedupeLaunch &a, const Workspace &ws, int b) {
+    if (!a.union_insert || !ws.uhash) return false;
+    return a.hit_kind ? __ldcg(a.hit_kind + b) != ADAPLD_HIT_LEX : true;
 }
 
 // Latest position stored for token u (-1 if absent or past the probe bound).
@@ -184,12 +176,27 @@ __device__ int mark_chunk(const DedupeLaunch &a, const Workspace &ws, int b, int
     return mine;
 }
 
+// Inserts token u into the union hash (open addressing, token + 1 as the
+// key); a table that runs full raises ADAPLD_DEV_INTERNAL (it is sized for
+// twice the batch's positions, so it never does).
+__device__ __forceinline__ void union_insert(uint32_t *U, int64_t UH, int u, int32_t *dst) {
+    const uint32_t key = (uint32_t)u + 1u;
+    uint64_t h = hash32((uint32_t)u) & (uint64_t)(UH - 1);
+    for (int64_t probe = 0; probe < UH; ++probe) {
+        const uint32_t old = atomicCAS(U + h, 0u, key);
+        if (old == 0u || old == key) return;
+        h = (h + 1) & (uint64_t)(UH - 1);
+    }
+    atomicOr(dst, ADAPLD_DEV_INTERNAL);
+}
+
 // Writes the marked positions' tokens of the chunk starting at j0 in
-// position order to out (s_word: the chunk's 128 words in shared memory).
-// One scan over the word counts gives every offset.
+// position order to out (s_word: the chunk's 128 words in shared memory),
+// and with pos_out their positions, inserting each token into the union hash
+// when uh is given.  One scan over the word counts gives every offset.
 __device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32_t *s_word,
                               int *s_off, int64_t *s_scan, int32_t *out, int64_t room,
-                              int32_t *dst) {
+                              int32_t *dst, int32_t *pos_out, uint32_t *uh, int64_t UH) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t w = t < kWordsPerChunk ? s_word[t] : 0u;
     int64_t all;
@@ -205,7 +212,10 @@ __device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32
         const int o = s_off[i] + __popc(wi & ((1u << lane) - 1u));
         if (((wi >> lane) & 1u) && idx_ok(o, 0, room, dst)) {
             const int j = j0 + e * kThreads1 + t;
-            out[o] = canon(M[j], a.vocab);
+            const int u = canon(M[j], a.vocab);
+            out[o] = u;
+            if (pos_out) pos_out[o] = j;
+            if (uh) union_insert(uh, UH, u, dst);
         }
     }
 }
@@ -267,8 +277,10 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
         int64_t total;  // the block's sum
         (void)block_exclusive_scan(mine, &total, s_scan);
         if (SINGLE) {  // one chunk: offset 0, no ticket
+            const bool uni = joins_union(a, ws, b);
             scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld, a.ld,
-                          ws.dev_status);
+                          ws.dev_status, uni ? ws.rep_pos + (int64_t)b * a.ld : nullptr,
+                          uni ? ws.uhash : nullptr, ws.UH);
             if (t == 0) {
                 ws.rep_len[b] = (int)total + 1;
                 ws.rep_tok[(int64_t)b * a.ld + total] = M[len - 1];  // the anchor (as stored)
@@ -331,8 +343,11 @@ __global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args)
     __syncthreads();
     const int off = __ldcg(ws.rep_cnt + (int64_t)b * ws.C1 + c);
     if (!idx_ok(off, 0, a.ld, ws.dev_status)) return;
+    const bool uni = joins_union(a, ws, b);
     scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld + off,
-                  a.ld - off, ws.dev_status);
+                  a.ld - off, ws.dev_status,
+                  uni ? ws.rep_pos + (int64_t)b * a.ld + off : nullptr, uni ? ws.uhash : nullptr,
+                  ws.UH);
 }
 
 // ---------------------------------------------------------------- expansion
@@ -477,9 +492,10 @@ cudaError_t launch_dedupe(const DedupeLaunch &a, const Workspace &ws, cudaStream
     if (ws.C1 == 1)  // every history is one chunk: one kernel builds the lists
         return a.pdl ? launch_dependent(rep_count_kernel<true>, grid, dim3(kThreads1), 0, s, args)
                      : (rep_count_kernel<true><<<grid, kThreads1, 0, s>>>(args),
-                        cudaGetLastError());
+                        counted(cudaGetLastError()));
     cudaError_t e = a.pdl ? launch_dependent(rep_insert_kernel, grid, dim3(kThreads1), 0, s, args)
-                          : (rep_insert_kernel<<<grid, kThreads1, 0, s>>>(args), cudaGetLastError());
+                          : (rep_insert_kernel<<<grid, kThreads1, 0, s>>>(args),
+                             counted(cudaGetLastError()));
     if (e != cudaSuccess) return e;
     e = launch_dependent(rep_count_kernel<false>, grid, dim3(kThreads1), 0, s, args);
     if (e != cudaSuccess) return e;

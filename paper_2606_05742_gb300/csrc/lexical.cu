@@ -288,7 +288,7 @@ cudaError_t launch_lexical(const LexLaunch &a, const Workspace &ws, cudaStream_t
         attr[1].val.clusterDim.z = 1;
         cfg.numAttrs = 2;
     }
-    return cudaLaunchKernelEx(&cfg, lexical_kernel, args);
+    return counted(cudaLaunchKernelEx(&cfg, lexical_kernel, args));
 }
 
 cudaError_t launch_outcome_plan(const int32_t *lengths, int64_t ld, int32_t B,
@@ -302,7 +302,7 @@ cudaError_t launch_plan(const int32_t *lengths, int64_t ld, int32_t B, const uin
                         const Workspace &ws, cudaStream_t s) {
     PlanArgs a{lengths, ld, B, nullptr, active, k, cand, score, n_cand, ws.plan};
     plan_kernel<<<1, kThreads1, 0, s>>>(a);
-    return cudaGetLastError();
+    return counted(cudaGetLastError());
 }
 
 }  // namespace adapld

@@ -1394,7 +1394,7 @@ cudaError_t launch_tree(const TreeLaunch &a, const Workspace &ws, cudaStream_t s
         attr[1].val.clusterDim.z = 1;
         cfg.attrs = attr;
         cfg.numAttrs = X > 1 ? 2 : 1;  // a plain launch is a cluster of one CTA
-        return cudaLaunchKernelEx(&cfg, kern, ca);
+        return counted(cudaLaunchKernelEx(&cfg, kern, ca));
     }
     const size_t vsmem = (size_t)a.d * sizeof(uint16_t);  // the staged query / reference row
     const size_t ssmem = vsmem + (size_t)(kSlice4 + 1) * sizeof(int);  // + a slice's tokens

@@ -1,0 +1,584 @@
+// Two-representation fallback over the union of the batch's distinct tokens
+// (Sec. 3.3, Eq. 4 as printed: cos(e_{M_j}, e_a) over token embeddings).
+//
+// The per-sequence path (semantic_kernel over each fallback sequence's
+// distinct-token list) reads a table row once per sequence that holds its
+// token; frequent tokens occur in most histories, so a batch reads two to
+// six times the rows its union needs.  Here each row of the union is read
+// from HBM once per step, and its dot products with the queries of all the
+// fallback sequences (the anchors' table rows) form one dense contraction,
+// union rows x queries over d, which runs on the tensor cores:
+//
+//  union_compact_kernel  the union hash (filled by the list scatter) into a
+//      list of tokens: each CTA compacts a slot range and appends it with one
+//      atomic add per 2048 slots (the list's order does not matter: every
+//      score is computed the same way wherever its row lands; a token-ordered
+//      list, tried, was slower).
+//  union_mma_kernel<NT>  persistent, one CTA per SM: 4 producer warps and
+//      8 MMA warps.  A tile is 16 union rows; its K dimension (d) streams
+//      through a ring of stages of 2048-element slices (4 KB; 2 KB when more
+//      than 8 queries leave room for one such stage only), each stage the
+//      tile's row slices and the live queries' slices (8 per query tile
+//      holding one), as many stages as fit 227 KB (2 to 4): the producers'
+//      lanes issue one bulk copy (cp.async.bulk) per slice, completing on the
+//      stage's mbarrier.  Long slices and about 100-200 KB in flight per SM
+//      read fastest (measured: 1 KB slices 2.6 TB/s, 2 KB 3.5, 4 KB 4.5 at
+//      the B = 2 config-5 shape; deeper rings of the same slices read
+//      slower).  Each MMA warp takes a K group of an eighth of the stage:
+//      it multiplies the 16 rows by the queries (mma.sync m16n8k16, bf16 in,
+//      fp32 accumulate; fragments by ldmatrix from slices padded by 16
+//      bytes, so the 8 rows of a fragment hit different banks; query tiles
+//      past the last query are skipped) and by themselves (two more MMAs on
+//      the A fragment, which has a B fragment's lane layout; their diagonals
+//      are |row|^2).  At the end of a tile the K groups' partial sums are
+//      added in a fixed order through shared memory, and the 256 MMA threads
+//      take the tile's (row, query) pairs: the row token's latest position in
+//      the query's sequence (the list kernels' hash; -1: the sequence does not
+//      hold it; the first probes of a thread's pairs were loaded while the
+//      tile streamed) and the cosine written to score_pos[b][latest
+//      position].
+//  seq_topk_kernel  one CTA per fallback sequence: over its list (entry r:
+//      the token whose latest position is rep_pos[r]) the top-k by
+//      (score desc, r desc) at or above tau; r order is latest-position
+//      order, so this is the ranking the expansion expects.
+//
+// Every mbarrier wait is bounded: on expiry the CTA raises ADAPLD_DEV_TIMEOUT,
+// stops issuing copies, drains those in flight and finishes without scores.
+#include <cstdlib>
+
+#include "common.cuh"
+
+namespace adapld {
+
+namespace {
+
+struct UnionArgs {
+    UnionLaunch p;
+    Workspace ws;
+};
+
+struct CompactArgs {
+    Workspace ws;
+    int64_t cap;  // ulist entries (B * ld)
+};
+
+// Whether sequence b is scored by the union pass and listed (the same test
+// in every kernel here): a fallback sequence with a list.
+__device__ __forceinline__ bool union_seq(const UnionLaunch &a, const Workspace &ws, int b,
+                                          int *rows) {
+    const int rl = ws.rep_len[b];
+    *rows = rl - 1;
+    if (rl < 1) return false;
+    if (a.hit_kind) return a.hit_kind[b] != ADAPLD_HIT_LEX;
+    return a.active ? a.active[b] != 0 : true;
+}
+
+__global__ void __launch_bounds__(256) union_compact_kernel(CompactArgs args) {
+    const Workspace &ws = args.ws;
+    __shared__ int64_t s_scan[32];
+    __shared__ int s_base;
+    pdl_wait_then_release();
+    constexpr int kPer = 8;  // slots per thread and step
+    const int64_t per_cta = (ws.UH + gridDim.x - 1) / gridDim.x;
+    const int64_t lo = (int64_t)blockIdx.x * per_cta;
+    const int64_t hi = min(lo + per_cta, ws.UH);
+    for (int64_t base = lo; base < hi; base += 256 * kPer) {
+        uint32_t key[kPer];
+        int mine = 0;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e) {
+            const int64_t i = base + (int64_t)e * 256 + threadIdx.x;
+            key[e] = i < hi ? __ldcg(ws.uhash + i) : 0u;
+            mine += key[e] != 0u;
+        }
+        int64_t total;
+        const int64_t ex = block_exclusive_scan(mine, &total, s_scan);
+        if (threadIdx.x == 0) s_base = total ? atomicAdd(ws.ucount, (int)total) : 0;
+        __syncthreads();
+        int o = s_base + (int)ex;
+#pragma unroll
+        for (int e = 0; e < kPer; ++e)
+            if (key[e] != 0u && idx_ok(o, 0, args.cap, ws.dev_status))
+                ws.ulist[o++] = (int)(key[e] - 1u);
+        __syncthreads();  // before s_base is rewritten
+    }
+}
+
+// Latest position of token u in a sequence's hash T (-1: absent), from the
+// value v already loaded from its first slot h.
+__device__ __forceinline__ int hash_latest(const unsigned long long *T, int64_t H, int u,
+                                           uint64_t h, unsigned long long v) {
+    const unsigned long long key = (unsigned long long)(uint32_t)(u + 1);
+    for (int64_t probe = 0; probe < H; ++probe) {
+        if (v == 0ull) return -1;
+        if ((v >> 32) == key) return (int)(uint32_t)(v & 0xffffffffull);
+        h = (h + 1) & (uint64_t)(H - 1);
+        v = __ldcg(T + h);
+    }
+    return -1;
+}
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+// d += a * b: one m16n8k16 tile, bf16 inputs, fp32 accumulators.
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                          uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+        "{%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Tile shape per query-tile count NT (NQ = 8 NT queries at most): TR union
+// rows per tile, K chunks of KC elements per stage.  The 8 MMA warps split a
+// stage into RG = TR / 16 row groups x KG = 8 / RG K groups.
+template <int NT> struct UCfg;
+template <> struct UCfg<2> { static constexpr int TR = 16, KC = 2048; };
+
+constexpr int kUConsumers = 8;  // MMA warps
+constexpr int kUProducers = 4;  // copy-issuing warps (a bulk copy costs its thread
+                                // about 100 cycles to issue)
+constexpr int kUThreads = (kUConsumers + kUProducers) * 32;
+
+template <int NT>
+struct UGeom {
+    static constexpr int TR = UCfg<NT>::TR, KC = UCfg<NT>::KC, NSMAX = 6;
+    static constexpr int NQ = NT * 8, RG = TR / 16, KG = kUConsumers / RG;
+    static constexpr int REDW = NQ + 1;             // partial dots + |row|^2 per row
+    static constexpr size_t RED = sizeof(float) * (size_t)(KG > 1 ? KG - 1 : 1) * TR * REDW;
+    // the ring takes what the reduction buffer, the mbarriers and the shared
+    // variables leave of 227 KB; its stage count follows the live queries
+    static constexpr size_t RING = 227 * 1024 - RED - 2 * NSMAX * sizeof(uint64_t) - 2048;
+    static constexpr size_t SMEM = RING + RED + 2 * NSMAX * sizeof(uint64_t);
+    // with every query tile live, two stages of KC / 2-element slices fit
+    static_assert(RING >= 2 * (size_t)(TR + NQ) * (KC + 16), "two stages at the most queries");
+    static_assert((KC / 2 / KG) % 16 == 0 && TR <= 64, "whole k16 steps per warp; rows by two lanes");
+};
+
+struct UnionShared {
+    int sel[kUnionMaxB];    // the fallback sequences
+    int qtok[kUnionMaxB];   // their anchors' table rows
+    float qss[kUnionMaxB];  // |query|^2
+    int64_t scan[32];
+    int nsel;
+    int abort;
+};
+
+// NT: query tiles of 8 (the queries, rounded up, are NT * 8 <= 64).
+template <int NT>
+__global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args) {
+    using G = UGeom<NT>;
+    const UnionLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    extern __shared__ __align__(128) uint8_t smem[];
+    uint8_t *ring = smem;
+    float *red = (float *)(smem + G::RING);  // [KG-1][TR][REDW]
+    uint64_t *full = (uint64_t *)(smem + G::RING + G::RED);
+    uint64_t *empty = full + G::NSMAX;
+    UnionShared &sh = *(UnionShared *)(empty + G::NSMAX);
+
+    pdl_wait_then_release();
+    const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int d = a.d;
+    // ---- the fallback sequences and their query rows (every CTA alike)
+    {
+        int rows = 0;
+        const bool in = t < a.B && union_seq(a, ws, t, &rows) && rows > 0;
+        int64_t total;
+        const int64_t ex = block_exclusive_scan(in ? 1 : 0, &total, sh.scan);
+        if (in) {
+            const int raw = ws.rep_tok[(int64_t)t * a.ld + rows];  // the anchor, as stored
+            const int row = canon(raw, a.vocab);
+            if (row != raw && blockIdx.x == 0 && a.status)
+                atomicOr(a.status + t, ADAPLD_SEQ_BAD_TOKEN);
+            sh.sel[ex] = t;
+            sh.qtok[ex] = row;
+        }
+        if (t == 0) {
+            sh.nsel = (int)total;
+            sh.abort = 0;
+            for (int i = 0; i < G::NSMAX; ++i) {
+                mbar_init(&full[i], kUProducers);
+                mbar_init(&empty[i], kUConsumers);
+            }
+            fence_barrier_init();
+        }
+    }
+    __syncthreads();
+    const int nsel = sh.nsel;
+    const int U = *ws.ucount;
+    const int ntiles = (U + G::TR - 1) / G::TR;
+    if (nsel == 0 || (int)blockIdx.x >= ntiles) return;
+    // a stage: TR row slices and the live query tiles' slices, of KC
+    // elements, or KC / 2 where KC would leave room for one stage only
+    const int ntl = (nsel + 7) >> 3;
+    const int KC = (size_t)2 * (G::TR + 8 * ntl) * (G::KC * 2 + 16) <= G::RING ? G::KC
+                                                                              : G::KC / 2;
+    const int PITCH = KC * 2 + 16;  // bytes per staged slice (padded)
+    const int KW = KC / G::KG;      // K elements per MMA warp and stage
+    const int nk = (d + KC - 1) / KC;  // K chunks per tile
+    const int stage_bytes = (G::TR + 8 * ntl) * PITCH;
+    const int NS = min(G::NSMAX, (int)(G::RING / stage_bytes));
+    const int my_tiles = (ntiles - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x;
+    const int total_it = my_tiles * nk;
+
+    // ------------------------------------------------------------ producers
+    // A stage's copies (its rows, then its queries) are numbered c = 0 ..
+    // nrows + nsel - 1; producer warp pw issues c = pw + kUProducers (lane +
+    // 32 h), each warp announcing its own bytes on the stage's mbarrier.
+    if (warp >= kUConsumers) {
+        const int pw = warp - kUConsumers;
+        int it = 0;
+        bool failed = false;
+        for (int ti = 0; ti < my_tiles && !failed; ++ti) {
+            const int tile = (int)blockIdx.x + ti * (int)gridDim.x;
+            const int nrows = min(G::TR, U - tile * G::TR);
+            const int ncopies = nrows + nsel;
+            const int mine = ncopies > pw ? (ncopies - pw + kUProducers - 1) / kUProducers : 0;
+            int tk[2];  // the table row of each of this lane's copies
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int c = pw + kUProducers * (lane + 32 * h);
+                tk[h] = c < nrows ? ws.ulist[tile * G::TR + c] : (c < ncopies ? sh.qtok[c - nrows] : 0);
+            }
+            for (int kc = 0; kc < nk; ++kc, ++it) {
+                const int s = it % NS, r = it / NS;
+                int ok = 1;
+                if (lane == 0) {
+                    if (r > 0 && !mbar_wait_bounded(&empty[s], (r - 1) & 1)) ok = 0;
+                    if (*(volatile int *)&sh.abort) ok = 0;
+                }
+                ok = __shfl_sync(0xffffffffu, ok, 0);
+                if (!ok) {
+                    failed = true;
+                    break;
+                }
+                const int k0 = kc * KC, kl = min(KC, d - k0);
+                const uint32_t bytes = (uint32_t)kl * 2;
+                uint8_t *st = ring + (size_t)s * stage_bytes;
+                if (lane == 0) mbar_arrive_expect_tx(&full[s], bytes * (uint32_t)mine);
+                __syncwarp();
+                const uint64_t pol = l2_evict_normal_policy();
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int c = pw + kUProducers * (lane + 32 * h);
+                    if (c < ncopies)
+                        bulk_g2s(st + (size_t)(c < nrows ? c : G::TR + c - nrows) * PITCH,
+                                 a.table + (int64_t)tk[h] * d + k0, bytes, &full[s], pol);
+                }
+            }
+        }
+        if (failed && lane == 0) {
+            sh.abort = 1;
+            atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
+            for (int i = max(0, it - NS); i < it; ++i)  // copies still in flight
+                (void)mbar_wait_bounded(&full[i % NS], (uint32_t)(i / NS) & 1);
+        }
+        return;
+    }
+
+    // ------------------------------------------------------------ consumers
+    for (int q = warp; q < nsel; q += kUConsumers) {  // |query|^2, a warp per query
+        const uint16_t *qr = a.table + (int64_t)sh.qtok[q] * d;
+        float part = 0.f;
+        for (int ch = lane; ch < (d >> 3); ch += 32) {
+            const uint4 w = ldg_nc_v4(qr + (size_t)ch * 8);
+            const uint32_t w4[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                part = fmaf(bf16lo(w4[e]), bf16lo(w4[e]), part);
+                part = fmaf(bf16hi(w4[e]), bf16hi(w4[e]), part);
+            }
+        }
+        part = warp_sum(part);
+        if (lane == 0) sh.qss[q] = part;
+    }
+    named_bar_sync(1, kUConsumers * 32);  // qss visible
+
+    const int rg = warp % G::RG, kg = warp / G::RG;  // row group, K group
+    const int g = lane >> 2, cq = (lane & 3) * 2;    // accumulator row / query of this lane
+    // fragment addresses: A = rows 16 rg + lane % 16, k half lane / 16; B =
+    // queries (lane % 8) + 8 (lane / 16), k half (lane / 8) % 2
+    const uint32_t ring_s = smem_u32(ring);
+    const uint32_t a_off = (uint32_t)((rg * 16 + (lane & 15)) * PITCH + (lane >> 4) * 16 +
+                                      kg * KW * 2);
+    const uint32_t b_off = (uint32_t)((G::TR + (lane & 7) + ((lane >> 4) << 3)) * PITCH +
+                                      ((lane >> 3) & 1) * 16 + kg * KW * 2);
+    // the last, odd query tile: lanes 16..31 repeat its rows (the stage has
+    // no slices past the live tiles)
+    const uint32_t b_off_last = (uint32_t)((G::TR + (lane & 7)) * PITCH +
+                                           ((lane >> 3) & 1) * 16 + kg * KW * 2);
+    float acc[NT][4], self0[4], self1[4];
+    // the tile's (row, query) pairs of this thread: pair pi = r * nsel + q
+    // for pi = t + 256 m; the first kBatch have their row token (loaded at
+    // the tile's first chunk) and first hash probe (at its second) in flight
+    // while the tile streams, so the epilogue waits for no load of theirs
+    constexpr int kPer = (G::TR * G::NQ + kUConsumers * 32 - 1) / (kUConsumers * 32);
+    constexpr int kBatch = kPer < 8 ? kPer : 8;
+    const int npairs = G::TR * nsel;
+    int pu[kBatch];
+    uint32_t ph[kBatch];
+    unsigned long long pv[kBatch];
+    bool aborted = false;
+    for (int it = 0; it < total_it; ++it) {
+        const int ti = it / nk, kc = it - ti * nk;
+        const int s = it % NS;
+        const int tile = (int)blockIdx.x + ti * (int)gridDim.x;
+        if (kc == 0) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+#pragma unroll
+                for (int j = 0; j < NT; ++j) acc[j][e] = 0.f;
+                self0[e] = self1[e] = 0.f;
+            }
+#pragma unroll
+            for (int m = 0; m < kBatch; ++m) {
+                const int pi = t + m * kUConsumers * 32;
+                const int row = tile * G::TR + pi / nsel;
+                pu[m] = (pi < npairs && row < U) ? __ldcg(ws.ulist + row) : -1;
+            }
+        }
+        if (kc == min(1, nk - 1)) {
+#pragma unroll
+            for (int m = 0; m < kBatch; ++m) {
+                const int pi = t + m * kUConsumers * 32;
+                const int q = pi - (pi / nsel) * nsel;
+                ph[m] = pu[m] >= 0 ? (uint32_t)(hash32((uint32_t)pu[m]) & (uint64_t)(ws.H - 1)) : 0u;
+                pv[m] = pu[m] >= 0 ? __ldcg(ws.htab + (int64_t)sh.sel[q] * ws.H + ph[m]) : 0ull;
+            }
+        }
+        if (!aborted && *(volatile int *)&sh.abort) aborted = true;  // the producer gave up
+        if (!aborted && !mbar_wait_bounded(&full[s], (uint32_t)(it / NS) & 1)) {
+            aborted = true;
+            if (lane == 0) {
+                sh.abort = 1;
+                atomicOr(ws.dev_status, ADAPLD_DEV_TIMEOUT);
+            }
+        }
+        if (!aborted) {
+            const int kl = min(KC, d - kc * KC);
+            const int ks = max(0, min(KW, kl - kg * KW)) / 16;  // k16 steps of this warp
+            const uint32_t sb = ring_s + (uint32_t)(s * stage_bytes);
+#pragma unroll 2
+            for (int k16 = 0; k16 < ks; ++k16) {
+                uint32_t af[4];
+                ldsm_x4(sb + a_off + k16 * 32, af);
+                // an A fragment's rows 0..7 (af[0], af[2]) and 8..15 (af[1],
+                // af[3]) have the lane layout of a B fragment
+                mma_16816(self0, af, af[0], af[2]);
+                mma_16816(self1, af, af[1], af[3]);
+#pragma unroll
+                for (int j = 0; j < NT; j += 2) {
+                    if (j >= ntl) break;
+                    uint32_t bf[4];
+                    ldsm_x4(sb + (j + 1 < ntl ? b_off : b_off_last) + (uint32_t)(j * 8 * PITCH) +
+                                k16 * 32,
+                            bf);
+                    mma_16816(acc[j], af, bf[0], bf[1]);
+                    if (j + 1 < ntl) mma_16816(acc[j + 1], af, bf[2], bf[3]);
+                }
+            }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[s]);
+        if (kc != nk - 1) continue;
+
+        // ---- the tile's epilogue.  (g, g) of self0 and (g + 8, g) of self1
+        // sit in lane 4 g + g / 2.
+        const int src = (lane & ~3) | (g >> 1);
+        const float n0 = __shfl_sync(0xffffffffu, (g & 1) ? self0[1] : self0[0], src);
+        const float n1 = __shfl_sync(0xffffffffu, (g & 1) ? self1[3] : self1[2], src);
+        // K groups 1.. leave their partial sums in red[kg - 1]; K group 0
+        // adds them in order and leaves the totals in red[0]
+        const int r0 = rg * 16 + g;
+        if (kg > 0) {
+            float *rp = red + (size_t)(kg - 1) * G::TR * G::REDW;
+#pragma unroll
+            for (int j = 0; j < NT; ++j) {
+                if (j >= ntl) break;
+                rp[r0 * G::REDW + j * 8 + cq] = acc[j][0];
+                rp[r0 * G::REDW + j * 8 + cq + 1] = acc[j][1];
+                rp[(r0 + 8) * G::REDW + j * 8 + cq] = acc[j][2];
+                rp[(r0 + 8) * G::REDW + j * 8 + cq + 1] = acc[j][3];
+            }
+            if ((lane & 3) == 0) {
+                rp[r0 * G::REDW + G::NQ] = n0;
+                rp[(r0 + 8) * G::REDW + G::NQ] = n1;
+            }
+        }
+        named_bar_sync(1, kUConsumers * 32);
+        if (kg == 0 && G::KG > 1) {
+            float v[NT][4];
+            float m0 = n0, m1 = n1;
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) v[j][e] = acc[j][e];
+#pragma unroll
+            for (int p = 0; p < G::KG - 1; ++p) {
+                const float *rp = red + (size_t)p * G::TR * G::REDW;
+#pragma unroll
+                for (int j = 0; j < NT; ++j) {
+                    if (j >= ntl) break;
+                    v[j][0] += rp[r0 * G::REDW + j * 8 + cq];
+                    v[j][1] += rp[r0 * G::REDW + j * 8 + cq + 1];
+                    v[j][2] += rp[(r0 + 8) * G::REDW + j * 8 + cq];
+                    v[j][3] += rp[(r0 + 8) * G::REDW + j * 8 + cq + 1];
+                }
+                m0 += rp[r0 * G::REDW + G::NQ];
+                m1 += rp[(r0 + 8) * G::REDW + G::NQ];
+            }
+            // the totals replace slot 0 (each element read and written by
+            // the same lane)
+            __syncwarp();
+#pragma unroll
+            for (int j = 0; j < NT; ++j) {
+                if (j >= ntl) break;
+                red[r0 * G::REDW + j * 8 + cq] = v[j][0];
+                red[r0 * G::REDW + j * 8 + cq + 1] = v[j][1];
+                red[(r0 + 8) * G::REDW + j * 8 + cq] = v[j][2];
+                red[(r0 + 8) * G::REDW + j * 8 + cq + 1] = v[j][3];
+            }
+            if ((lane & 3) == 0) {
+                red[r0 * G::REDW + G::NQ] = m0;
+                red[(r0 + 8) * G::REDW + G::NQ] = m1;
+            }
+        }
+        named_bar_sync(1, kUConsumers * 32);
+        // every (row, query) pair of the tile: the row token's latest
+        // position in the query's sequence (-1: not held), then the cosine
+        // at that position; all first probes of a thread in flight together
+        if (!aborted) {
+#pragma unroll 1
+            for (int m0 = 0; m0 < kPer; m0 += kBatch) {
+                int uu[kBatch];
+                uint32_t hh[kBatch];
+                unsigned long long vv[kBatch];
+#pragma unroll
+                for (int m = 0; m < kBatch; ++m) {
+                    if (m0 == 0) {
+                        uu[m] = pu[m];
+                        hh[m] = ph[m];
+                        vv[m] = pv[m];
+                        continue;
+                    }
+                    const int pi = t + (m0 + m) * kUConsumers * 32;
+                    const int r = pi / nsel, q = pi - r * nsel;
+                    const int row = tile * G::TR + r;
+                    uu[m] = (pi < npairs && row < U) ? __ldcg(ws.ulist + row) : -1;
+                    hh[m] = uu[m] >= 0 ? (uint32_t)(hash32((uint32_t)uu[m]) & (uint64_t)(ws.H - 1))
+                                       : 0u;
+                    vv[m] = uu[m] >= 0 ? __ldcg(ws.htab + (int64_t)sh.sel[q] * ws.H + hh[m]) : 0ull;
+                }
+#pragma unroll
+                for (int m = 0; m < kBatch; ++m) {
+                    if (uu[m] < 0) continue;
+                    const int pi = t + (m0 + m) * kUConsumers * 32;
+                    const int r = pi / nsel, q = pi - r * nsel;
+                    const int b = sh.sel[q];
+                    const int pos =
+                        hash_latest(ws.htab + (int64_t)b * ws.H, ws.H, uu[m], hh[m], vv[m]);
+                    if (pos >= 0 && idx_ok(pos, 0, a.ld, ws.dev_status))
+                        ws.score_pos[(int64_t)b * a.ld + pos] = cosine_from(
+                            red[r * G::REDW + q], red[r * G::REDW + G::NQ], sh.qss[q]);
+                }
+            }
+        }
+        // every read of red is done before the next tile's partial sums
+        // may land there (a K group can finish a short tile early)
+        named_bar_sync(1, kUConsumers * 32);
+    }
+}
+
+
+// One CTA per sequence: the top-k of its list by the union pass's scores.
+__global__ void __launch_bounds__(kThreads4) seq_topk_kernel(UnionArgs args) {
+    const UnionLaunch &a = args.p;
+    const Workspace &ws = args.ws;
+    __shared__ float wl_s[kThreads4 / 32][32];
+    __shared__ int wl_j[kThreads4 / 32][32];
+    __shared__ int wl_n[kThreads4 / 32];
+    pdl_wait_then_release();
+    const int b = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    int n = 0;
+    if (!union_seq(a, ws, b, &n)) return;
+    const int k = a.k;
+    const float tau = a.tau;
+    const int32_t *pos = ws.rep_pos + (int64_t)b * a.ld;
+    const float *sc = ws.score_pos + (int64_t)b * a.ld;
+    WarpTopK tk;
+    tk.reset();
+    constexpr int U8 = 8;  // list entries per lane per step, loads in flight together
+    for (int base = warp * 32 * U8; base < n; base += kThreads4 * U8) {
+        int p[U8];
+#pragma unroll
+        for (int u = 0; u < U8; ++u) {
+            const int r = base + u * 32 + lane;
+            p[u] = r < n ? pos[r] : -1;
+        }
+        float s[U8];
+#pragma unroll
+        for (int u = 0; u < U8; ++u)
+            s[u] = (p[u] >= 0 && idx_ok(p[u], 0, a.ld, ws.dev_status)) ? sc[p[u]] : -INFINITY;
+#pragma unroll
+        for (int u = 0; u < U8; ++u) {
+            const int r = base + u * 32 + lane;
+            tk.insert(r < n && s[u] >= tau, s[u], r, k);
+        }
+    }
+    wl_s[warp][lane] = tk.s;
+    wl_j[warp][lane] = tk.j;
+    if (lane == 0) wl_n[warp] = tk.n;
+    __syncthreads();
+    if (warp == 0) {
+        WarpTopK f;
+        f.reset();
+        for (int w = 0; w < kThreads4 / 32; ++w)
+            f.insert(lane < wl_n[w], wl_s[w][lane], wl_j[w][lane], k);
+        if (lane < k) {
+            a.cand[(int64_t)b * k + lane] = lane < f.n ? f.j : -1;
+            a.score[(int64_t)b * k + lane] = lane < f.n ? f.s : 0.f;
+        }
+        if (lane == 0) {
+            a.n_cand[b] = f.n;
+            if (a.hit_kind) a.hit_kind[b] = f.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
+        }
+    }
+}
+
+template <int NT>
+cudaError_t launch_mma(const UnionArgs &args, int sms, cudaStream_t s) {
+    auto kern = union_mma_kernel<NT>;
+    const size_t smem = UGeom<NT>::SMEM + sizeof(UnionShared);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return launch_dependent(kern, dim3(sms), dim3(kUThreads), smem, s, args);
+}
+
+}  // namespace
+
+bool union_applies(int32_t B, int64_t ld, int32_t d) {
+    if (const char *e = std::getenv("ADAPLD_EMB_UNION"))  // A/B switch for measurements
+        if (e[0] == '0') return false;
+    return union_enabled(B, ld) && d % 16 == 0;
+}
+
+cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t s) {
+    const int sms = device_sms();
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    CompactArgs ca{ws, (int64_t)a.B * a.ld};
+    cudaError_t e = launch_dependent(union_compact_kernel, dim3(2 * sms), dim3(256), 0, s, ca);
+    if (e != cudaSuccess) return e;
+    UnionArgs ua{a, ws};
+    static_assert(kUnionMaxB <= 16, "two query tiles of 8");
+    e = launch_mma<2>(ua, sms, s);
+    if (e != cudaSuccess) return e;
+    return launch_dependent(seq_topk_kernel, dim3(a.B), dim3(kThreads4), 0, s, ua);
+}
+
+}  // namespace adapld

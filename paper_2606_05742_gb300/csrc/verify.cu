@@ -240,7 +240,7 @@ cudaError_t launch_verify(const VerifyLaunch &a, const Workspace &ws, cudaStream
     const int S = max(1, min(groups, kMaxNodes / a.N));
     VerifyArgs args{a, ws, S};
     verify_kernel<<<dim3(S, a.N, a.B), kThreadsV, 0, s>>>(args);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = counted(cudaGetLastError());
     if (e != cudaSuccess) return e;
     return launch_dependent(walk_kernel, dim3(a.B), dim3(kThreadsV), 0, s, args);
 }

@@ -36,7 +36,7 @@ EXPORTED = [
     "adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
     "adapld_step", "adapld_step_ex", "adapld_read_device_status",
     "adapld_semantic_topk_static", "adapld_embedding_topk", "adapld_accept_greedy",
-    "adapld_step_from_host", "adapld_semantic_topk_static_status",
+    "adapld_step_from_host", "adapld_semantic_topk_static_status", "adapld_kernel_launches",
 ]
 STATIC_MAX_B = 1024
 ERR_NULL = -1
@@ -119,6 +119,8 @@ def _configure(lib: ctypes.CDLL) -> ctypes.CDLL:
                                          i32, P, P, P, sz, P]
     lib.adapld_step_from_host.argtypes = [P, i64, P, P, i32, P, i32, P, P, P, P, P, P, P, P, sz,
                                           P]
+    lib.adapld_kernel_launches.argtypes = []
+    lib.adapld_kernel_launches.restype = ctypes.c_ulonglong
     for f in ("adapld_lexical_match", "adapld_semantic_topk", "adapld_build_draft_tree",
               "adapld_step", "adapld_step_ex", "adapld_read_device_status",
               "adapld_semantic_topk_static", "adapld_embedding_topk",
@@ -204,6 +206,11 @@ def semantic_topk_static(reps, query, lengths, k: int, tau: float, cand, score, 
                                             _ptr(active), B, k, tau, _ptr(cand), _ptr(score),
                                             _ptr(n_cand), _stream(stream))
     _check(rc, "adapld_semantic_topk_static")
+
+
+def kernel_launches() -> int:
+    """Kernels the library has enqueued in this process (adapld_kernel_launches)."""
+    return int(load().adapld_kernel_launches())
 
 
 def semantic_topk_static_status(stream=None) -> int:

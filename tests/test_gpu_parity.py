@@ -717,13 +717,19 @@ EMB_CASES = [  # (cfg, B, L, d, de, V, seed)
     (3, 6, 2000, 640, 136, 3000, 2), (4, 20, 500, 64, 8, 2048, 3),
     (5, 3, 1200, 64, 8192, 2048, 4),
     (5, 3, 20000, 64, 256, 4096, 5),    # several chunks and slices per history
+    (2, 16, 900, 64, 512, 3000, 6),     # 9-16 fallback queries: two query tiles
+    (3, 12, 1500, 64, 1040, 4000, 7),   # a table width that ends in a partial slice
 ]
 
 
+@pytest.mark.parametrize("union", ["1", "0"])
 @pytest.mark.parametrize("cfg,B,L,d,de,V,seed", EMB_CASES)
-def test_embedding_mode(cfg, B, L, d, de, V, seed):
+def test_embedding_mode(cfg, B, L, d, de, V, seed, union, monkeypatch):
     """Eq. 4 over token embeddings, Eq. 6 rerank of the semantic candidates,
-    and the successor backoff of Sec. 3.5, against the oracle."""
+    and the successor backoff of Sec. 3.5, against the oracle; through the
+    union pass (batches of up to 16: every table row of the batch read once,
+    tensor cores) and through the per-sequence lists (ADAPLD_EMB_UNION=0)."""
+    monkeypatch.setenv("ADAPLD_EMB_UNION", union)
     w = synth.make_workload(cfg, B=B, L=L, d=d, V=V, nohit=0.6, seed=seed)
     E = synth.make_embeddings(w, V, de, seed)
     backoff = 0
@@ -944,3 +950,26 @@ def test_full_size_embedding_config5():
     assert rep.tie_resolved == 0, rep
     for b in [int(x) for x in w.forced]:
         assert g["hit_kind"][b] == 2
+
+
+def test_kernel_launch_counter():
+    """adapld_kernel_launches() counts the kernels the library enqueues: the
+    same step adds the same count each time (its kernels: lexical, semantic,
+    tree stage at least), and a call refused by the argument checks adds
+    none."""
+    w = synth.make_workload(5, B=3, L=20000, d=64, nohit=0.5, seed=91)
+    P = P_of(w)
+    tok, ln, reps, q = to_dev(w)
+    eng = native.Engine(w.B, w.ld, w.d, params(P))
+    eng.run(tok, ln, reps, q)
+    torch.cuda.synchronize()
+    n0 = native.kernel_launches()
+    eng.run(tok, ln, reps, q)
+    n1 = native.kernel_launches()
+    eng.run(tok, ln, reps, q)
+    n2 = native.kernel_launches()
+    torch.cuda.synchronize()
+    assert n1 - n0 == n2 - n1 >= 3
+    with pytest.raises(native.AdapldError):
+        native.step(tok, ln, reps, q, params(P), eng.out, eng.ws[:64])  # workspace too small
+    assert native.kernel_launches() == n2
