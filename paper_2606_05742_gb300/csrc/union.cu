@@ -245,6 +245,8 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
             for (int h = 0; h < 2; ++h) {
                 const int c = pw + kUProducers * (lane + 32 * h);
                 tk[h] = c < nrows ? ws.ulist[tile * G::TR + c] : (c < ncopies ? sh.qtok[c - nrows] : 0);
+                // (checked build: a table row outside the table reads row 0)
+                if (c < ncopies && !idx_ok(tk[h], 0, a.vocab, ws.dev_status)) tk[h] = 0;
             }
             for (int kc = 0; kc < nk; ++kc, ++it) {
                 const int s = it % NS, r = it / NS;
