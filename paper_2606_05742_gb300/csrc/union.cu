@@ -37,10 +37,11 @@
 //      hold it; the first probes of a thread's pairs were loaded while the
 //      tile streamed) and the cosine written to score_pos[b][latest
 //      position].
-//  seq_topk_kernel  one CTA per fallback sequence: over its list (entry r:
-//      the token whose latest position is rep_pos[r]) the top-k by
-//      (score desc, r desc) at or above tau; r order is latest-position
-//      order, so this is the ranking the expansion expects.
+//  seq_topk_kernel  a cluster of 8 CTAs per fallback sequence: over its list
+//      (entry r: the token whose latest position is rep_pos[r]) the top-k by
+//      (score desc, r desc) at or above tau, a slice of the list per CTA,
+//      merged in CTA rank 0; r order is latest-position order, so this is the
+//      ranking the expansion expects.
 //
 // Every mbarrier wait is bounded: on expiry the CTA raises ADAPLD_DEV_TIMEOUT,
 // stops issuing copies, drains those in flight and finishes without scores.
@@ -498,30 +499,44 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
 }
 
 
-// One CTA per sequence: the top-k of its list by the union pass's scores.
+// The per-sequence top k over the union scores: a cluster of kTopkSlices
+// CTAs per fallback sequence, CTA x ranking slice x of the sequence's list
+// (entry r: the token whose latest position is rep_pos[r]; 8 entries per
+// lane in flight), by (score desc, r desc) at or above tau; r order is
+// latest-position order, so this is the ranking the expansion expects.
+// Each CTA pushes its best k into CTA rank 0's shared memory, which merges
+// them after one cluster barrier.
+constexpr int kTopkSlices = 8;
+
 __global__ void __launch_bounds__(kThreads4) seq_topk_kernel(UnionArgs args) {
     const UnionLaunch &a = args.p;
     const Workspace &ws = args.ws;
     __shared__ float wl_s[kThreads4 / 32][32];
     __shared__ int wl_j[kThreads4 / 32][32];
     __shared__ int wl_n[kThreads4 / 32];
+    __shared__ float m_s[kTopkSlices][32];  // rank 0: every slice's list
+    __shared__ int m_j[kTopkSlices][32];
+    __shared__ int m_n[kTopkSlices];
     pdl_wait_then_release();
-    const int b = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int b = blockIdx.y, x = blockIdx.x, t = threadIdx.x, lane = t & 31, warp = t >> 5;
     int n = 0;
-    if (!union_seq(a, ws, b, &n)) return;
+    if (!union_seq(a, ws, b, &n)) return;  // the whole cluster (b is its sequence)
+    cluster_arrive_relaxed();  // every CTA has started before the pushes (waited below)
     const int k = a.k;
     const float tau = a.tau;
     const int32_t *pos = ws.rep_pos + (int64_t)b * a.ld;
     const float *sc = ws.score_pos + (int64_t)b * a.ld;
+    const int per = (n + kTopkSlices - 1) / kTopkSlices;
+    const int lo = x * per, hi = min(n, lo + per);
     WarpTopK tk;
     tk.reset();
     constexpr int U8 = 8;  // list entries per lane per step, loads in flight together
-    for (int base = warp * 32 * U8; base < n; base += kThreads4 * U8) {
+    for (int base = lo + warp * 32 * U8; base < hi; base += kThreads4 * U8) {
         int p[U8];
 #pragma unroll
         for (int u = 0; u < U8; ++u) {
             const int r = base + u * 32 + lane;
-            p[u] = r < n ? pos[r] : -1;
+            p[u] = r < hi ? pos[r] : -1;
         }
         float s[U8];
 #pragma unroll
@@ -530,26 +545,35 @@ __global__ void __launch_bounds__(kThreads4) seq_topk_kernel(UnionArgs args) {
 #pragma unroll
         for (int u = 0; u < U8; ++u) {
             const int r = base + u * 32 + lane;
-            tk.insert(r < n && s[u] >= tau, s[u], r, k);
+            tk.insert(r < hi && s[u] >= tau, s[u], r, k);
         }
     }
     wl_s[warp][lane] = tk.s;
     wl_j[warp][lane] = tk.j;
     if (lane == 0) wl_n[warp] = tk.n;
     __syncthreads();
+    cluster_wait();
     if (warp == 0) {
         WarpTopK f;
         f.reset();
         for (int w = 0; w < kThreads4 / 32; ++w)
             f.insert(lane < wl_n[w], wl_s[w][lane], wl_j[w][lane], k);
-        if (lane < k) {
-            a.cand[(int64_t)b * k + lane] = lane < f.n ? f.j : -1;
-            a.score[(int64_t)b * k + lane] = lane < f.n ? f.s : 0.f;
-        }
-        if (lane == 0) {
-            a.n_cand[b] = f.n;
-            if (a.hit_kind) a.hit_kind[b] = f.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
-        }
+        st_cluster_f32(&m_s[x][lane], 0, f.s);
+        st_cluster_i32(&m_j[x][lane], 0, f.j);
+        if (lane == 0) st_cluster_i32(&m_n[x], 0, f.n);
+    }
+    cluster_sync_all();  // the slices' lists are in rank 0
+    if (x != 0 || warp != 0) return;
+    WarpTopK f;
+    f.reset();
+    for (int r = 0; r < kTopkSlices; ++r) f.insert(lane < m_n[r], m_s[r][lane], m_j[r][lane], k);
+    if (lane < k) {
+        a.cand[(int64_t)b * k + lane] = lane < f.n ? f.j : -1;
+        a.score[(int64_t)b * k + lane] = lane < f.n ? f.s : 0.f;
+    }
+    if (lane == 0) {
+        a.n_cand[b] = f.n;
+        if (a.hit_kind) a.hit_kind[b] = f.n > 0 ? ADAPLD_HIT_SEM : ADAPLD_HIT_NONE;
     }
 }
 
@@ -580,7 +604,20 @@ cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t
     static_assert(kUnionMaxB <= 16, "two query tiles of 8");
     e = launch_mma<2>(ua, sms, s);
     if (e != cudaSuccess) return e;
-    return launch_dependent(seq_topk_kernel, dim3(a.B), dim3(kThreads4), 0, s, ua);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kTopkSlices, a.B);
+    cfg.blockDim = dim3(kThreads4);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = kTopkSlices;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return counted(cudaLaunchKernelEx(&cfg, seq_topk_kernel, ua));
 }
 
 }  // namespace adapld
