@@ -28,11 +28,12 @@
 //      it multiplies the 16 rows by the queries (mma.sync m16n8k16, bf16 in,
 //      fp32 accumulate; fragments by ldmatrix from slices padded by 16
 //      bytes, so the 8 rows of a fragment hit different banks; query tiles
-//      past the last query are skipped) and by themselves (two more MMAs on
-//      the A fragment, which has a B fragment's lane layout; their diagonals
-//      are |row|^2).  At the end of a tile the K groups' partial sums are
-//      added in a fixed order through shared memory, and the 256 MMA threads
-//      take the tile's (row, query) pairs: the row token's latest position in
+//      past the last query are skipped) and sums the squares of its A
+//      fragments on the CUDA cores for |row|^2 (two more MMAs per step, of
+//      the fragment with itself, measured slower).  At the end of a tile every warp leaves its K group's
+//      partial sums in shared memory and, after one barrier, the thread of
+//      each of the tile's (row, query) pairs adds them in a fixed order and
+//      takes the pair: the row token's latest position in
 //      the query's sequence (the list kernels' hash; -1: the sequence does not
 //      hold it; the first probes of a thread's pairs were loaded while the
 //      tile streamed) and the cosine written to score_pos[b][latest
@@ -151,7 +152,7 @@ struct UGeom {
     static constexpr int TR = UCfg<NT>::TR, KC = UCfg<NT>::KC, NSMAX = 6;
     static constexpr int NQ = NT * 8, RG = TR / 16, KG = kUConsumers / RG;
     static constexpr int REDW = NQ + 1;             // partial dots + |row|^2 per row
-    static constexpr size_t RED = sizeof(float) * (size_t)(KG > 1 ? KG - 1 : 1) * TR * REDW;
+    static constexpr size_t RED = sizeof(float) * (size_t)2 * KG * TR * REDW;  // two tiles
     // the ring takes what the reduction buffer, the mbarriers and the shared
     // variables leave of 227 KB; its stage count follows the live queries
     static constexpr size_t RING = 227 * 1024 - RED - 2 * NSMAX * sizeof(uint64_t) - 2048;
@@ -178,7 +179,7 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
     const Workspace &ws = args.ws;
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t *ring = smem;
-    float *red = (float *)(smem + G::RING);  // [KG-1][TR][REDW]
+    float *red = (float *)(smem + G::RING);  // [2][KG][TR][REDW]
     uint64_t *full = (uint64_t *)(smem + G::RING + G::RED);
     uint64_t *empty = full + G::NSMAX;
     UnionShared &sh = *(UnionShared *)(empty + G::NSMAX);
@@ -316,7 +317,8 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
     // no slices past the live tiles)
     const uint32_t b_off_last = (uint32_t)((G::TR + (lane & 7)) * PITCH +
                                            ((lane >> 3) & 1) * 16 + kg * KW * 2);
-    float acc[NT][4], self0[4], self1[4];
+    float acc[NT][4];
+    float ss0 = 0.f, ss1 = 0.f;  // |row g|^2, |row g + 8|^2: this lane's share of its K group
     // the tile's (row, query) pairs of this thread: pair pi = r * nsel + q
     // for pi = t + 256 m; the first kBatch have their row token (loaded at
     // the tile's first chunk) and first hash probe (at its second) in flight
@@ -337,7 +339,7 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
             for (int e = 0; e < 4; ++e) {
 #pragma unroll
                 for (int j = 0; j < NT; ++j) acc[j][e] = 0.f;
-                self0[e] = self1[e] = 0.f;
+                ss0 = ss1 = 0.f;
             }
 #pragma unroll
             for (int m = 0; m < kBatch; ++m) {
@@ -371,10 +373,19 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
             for (int k16 = 0; k16 < ks; ++k16) {
                 uint32_t af[4];
                 ldsm_x4(sb + a_off + k16 * 32, af);
-                // an A fragment's rows 0..7 (af[0], af[2]) and 8..15 (af[1],
-                // af[3]) have the lane layout of a B fragment
-                mma_16816(self0, af, af[0], af[2]);
-                mma_16816(self1, af, af[1], af[3]);
+                // the squares of the fragment's elements (af[0], af[2]: row g;
+                // af[1], af[3]: row g + 8) on the CUDA cores, next to the MMAs
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const float lo = bf16lo(af[e]), hi = bf16hi(af[e]);
+                    if (e & 1) {
+                        ss1 = fmaf(lo, lo, ss1);
+                        ss1 = fmaf(hi, hi, ss1);
+                    } else {
+                        ss0 = fmaf(lo, lo, ss0);
+                        ss0 = fmaf(hi, hi, ss0);
+                    }
+                }
 #pragma unroll
                 for (int j = 0; j < NT; j += 2) {
                     if (j >= ntl) break;
@@ -391,16 +402,21 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
         if (lane == 0) mbar_arrive(&empty[s]);
         if (kc != nk - 1) continue;
 
-        // ---- the tile's epilogue.  (g, g) of self0 and (g + 8, g) of self1
-        // sit in lane 4 g + g / 2.
-        const int src = (lane & ~3) | (g >> 1);
-        const float n0 = __shfl_sync(0xffffffffu, (g & 1) ? self0[1] : self0[0], src);
-        const float n1 = __shfl_sync(0xffffffffu, (g & 1) ? self1[3] : self1[2], src);
-        // K groups 1.. leave their partial sums in red[kg - 1]; K group 0
-        // adds them in order and leaves the totals in red[0]
+        // ---- the tile's epilogue: the rows' |row|^2 over the quad of lanes
+        // holding them
+        float n0 = ss0, n1 = ss1;
+        n0 += __shfl_xor_sync(0xffffffffu, n0, 1);
+        n0 += __shfl_xor_sync(0xffffffffu, n0, 2);
+        n1 += __shfl_xor_sync(0xffffffffu, n1, 1);
+        n1 += __shfl_xor_sync(0xffffffffu, n1, 2);
+        // every MMA warp leaves its K group's partial sums in red[ti % 2][kg]
+        // (two buffers by tile parity: a warp that starts the next tile's
+        // epilogue early never meets this tile's reads, which end before the
+        // next barrier)
         const int r0 = rg * 16 + g;
-        if (kg > 0) {
-            float *rp = red + (size_t)(kg - 1) * G::TR * G::REDW;
+        float *const rbuf = red + (size_t)(ti & 1) * G::KG * G::TR * G::REDW;
+        {
+            float *rp = rbuf + (size_t)kg * G::TR * G::REDW;
 #pragma unroll
             for (int j = 0; j < NT; ++j) {
                 if (j >= ntl) break;
@@ -412,44 +428,6 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
             if ((lane & 3) == 0) {
                 rp[r0 * G::REDW + G::NQ] = n0;
                 rp[(r0 + 8) * G::REDW + G::NQ] = n1;
-            }
-        }
-        named_bar_sync(1, kUConsumers * 32);
-        if (kg == 0 && G::KG > 1) {
-            float v[NT][4];
-            float m0 = n0, m1 = n1;
-#pragma unroll
-            for (int j = 0; j < NT; ++j)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) v[j][e] = acc[j][e];
-#pragma unroll
-            for (int p = 0; p < G::KG - 1; ++p) {
-                const float *rp = red + (size_t)p * G::TR * G::REDW;
-#pragma unroll
-                for (int j = 0; j < NT; ++j) {
-                    if (j >= ntl) break;
-                    v[j][0] += rp[r0 * G::REDW + j * 8 + cq];
-                    v[j][1] += rp[r0 * G::REDW + j * 8 + cq + 1];
-                    v[j][2] += rp[(r0 + 8) * G::REDW + j * 8 + cq];
-                    v[j][3] += rp[(r0 + 8) * G::REDW + j * 8 + cq + 1];
-                }
-                m0 += rp[r0 * G::REDW + G::NQ];
-                m1 += rp[(r0 + 8) * G::REDW + G::NQ];
-            }
-            // the totals replace slot 0 (each element read and written by
-            // the same lane)
-            __syncwarp();
-#pragma unroll
-            for (int j = 0; j < NT; ++j) {
-                if (j >= ntl) break;
-                red[r0 * G::REDW + j * 8 + cq] = v[j][0];
-                red[r0 * G::REDW + j * 8 + cq + 1] = v[j][1];
-                red[(r0 + 8) * G::REDW + j * 8 + cq] = v[j][2];
-                red[(r0 + 8) * G::REDW + j * 8 + cq + 1] = v[j][3];
-            }
-            if ((lane & 3) == 0) {
-                red[r0 * G::REDW + G::NQ] = m0;
-                red[(r0 + 8) * G::REDW + G::NQ] = m1;
             }
         }
         named_bar_sync(1, kUConsumers * 32);
@@ -486,15 +464,19 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
                     const int b = sh.sel[q];
                     const int pos =
                         hash_latest(ws.htab + (int64_t)b * ws.H, ws.H, uu[m], hh[m], vv[m]);
-                    if (pos >= 0 && idx_ok(pos, 0, a.ld, ws.dev_status))
-                        ws.score_pos[(int64_t)b * a.ld + pos] = cosine_from(
-                            red[r * G::REDW + q], red[r * G::REDW + G::NQ], sh.qss[q]);
+                    if (pos >= 0 && idx_ok(pos, 0, a.ld, ws.dev_status)) {
+                        // the pair's dot and the row's |row|^2, K groups in order
+                        float dot = 0.f, ss = 0.f;
+#pragma unroll
+                        for (int p = 0; p < G::KG; ++p) {
+                            dot += rbuf[((size_t)p * G::TR + r) * G::REDW + q];
+                            ss += rbuf[((size_t)p * G::TR + r) * G::REDW + G::NQ];
+                        }
+                        ws.score_pos[(int64_t)b * a.ld + pos] = cosine_from(dot, ss, sh.qss[q]);
+                    }
                 }
             }
         }
-        // every read of red is done before the next tile's partial sums
-        // may land there (a K group can finish a short tile early)
-        named_bar_sync(1, kUConsumers * 32);
     }
 }
 
