@@ -14,27 +14,30 @@
 //      atomic add per 2048 slots (the list's order does not matter: every
 //      score is computed the same way wherever its row lands; a token-ordered
 //      list, tried, was slower).
-//  union_mma_kernel<NT>  persistent, one CTA per SM: 4 producer warps and
+//  union_mma_kernel<NT>  persistent, one CTA per SM: 2 producer warps and
 //      8 MMA warps.  A tile is 16 union rows; its K dimension (d) streams
 //      through a ring of stages of 2048-element slices (4 KB; 2 KB when more
 //      than 8 queries leave room for one such stage only), each stage the
 //      tile's row slices and the live queries' slices (8 per query tile
-//      holding one), as many stages as fit 227 KB (2 to 4): the producers'
+//      holding one), as many stages as fit 227 KB (2 or 3): the producers'
 //      lanes issue one bulk copy (cp.async.bulk) per slice, completing on the
-//      stage's mbarrier.  Long slices and about 100-200 KB in flight per SM
-//      read fastest (measured: 1 KB slices 2.6 TB/s, 2 KB 3.5, 4 KB 4.5 at
-//      the B = 2 config-5 shape; deeper rings of the same slices read
-//      slower).  Each MMA warp takes a K group of an eighth of the stage:
-//      it multiplies the 16 rows by the queries (mma.sync m16n8k16, bf16 in,
-//      fp32 accumulate; fragments by ldmatrix from slices padded by 16
-//      bytes, so the 8 rows of a fragment hit different banks; query tiles
-//      past the last query are skipped) and sums the squares of its A
-//      fragments on the CUDA cores for |row|^2 (two more MMAs per step, of
-//      the fragment with itself, measured slower).  At the end of a tile every warp leaves its K group's
-//      partial sums in shared memory and, after one barrier, the thread of
-//      each of the tile's (row, query) pairs adds them in a fixed order and
-//      takes the pair: the row token's latest position in
-//      the query's sequence (the list kernels' hash; -1: the sequence does not
+//      stage's mbarrier.  Long slices read fastest (a copy-only probe over
+//      random table rows: 1 KB slices 2.0 TB/s, 2 KB 3.7, 4 KB 5.9-6.5,
+//      whole 16 KB rows 6.7-6.9).  Each MMA warp takes a K group of an
+//      eighth of the stage, in two halves: it loads a half's fragments by
+//      ldmatrix (slices padded by 16 bytes, so the 8 rows of a fragment hit
+//      different banks), multiplies the 16 rows by the queries (mma.sync
+//      m16n8k16, bf16 in, fp32 accumulate; query tiles past the last query
+//      skipped) and sums the squares of its A fragments on the CUDA cores for
+//      |row|^2; the stage's slot is released once the second half's
+//      fragments are in registers, before their arithmetic, so the ring
+//      refills during it (release after all the arithmetic: 225 us at config
+//      5; norms by two more MMAs of the fragment with itself, which made the
+//      tensor pipe the pace: 245 us).  At the end of a tile every warp leaves
+//      its K group's partial sums in shared memory and, after one barrier,
+//      the thread of each of the tile's (row, query) pairs adds them in a
+//      fixed order and takes the pair: the row token's latest position in the
+//      query's sequence (the list kernels' hash; -1: the sequence does not
 //      hold it; the first probes of a thread's pairs were loaded while the
 //      tile streamed) and the cosine written to score_pos[b][latest
 //      position].
@@ -143,7 +146,7 @@ template <int NT> struct UCfg;
 template <> struct UCfg<2> { static constexpr int TR = 16, KC = 2048; };
 
 constexpr int kUConsumers = 8;  // MMA warps
-constexpr int kUProducers = 4;  // copy-issuing warps (a bulk copy costs its thread
+constexpr int kUProducers = 2;  // copy-issuing warps (a bulk copy costs its thread
                                 // about 100 cycles to issue)
 constexpr int kUThreads = (kUConsumers + kUProducers) * 32;
 
@@ -161,6 +164,85 @@ struct UGeom {
     static_assert(RING >= 2 * (size_t)(TR + NQ) * (KC + 16), "two stages at the most queries");
     static_assert((KC / 2 / KG) % 16 == 0 && TR <= 64, "whole k16 steps per warp; rows by two lanes");
 };
+
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t (&r)[2]) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];"
+                 : "=r"(r[0]), "=r"(r[1])
+                 : "r"(addr));
+}
+
+// One stage of an MMA warp, in two halves of its ks <= KMAX k16 steps: the
+// first half's fragments are loaded and multiplied, then the second half's
+// are loaded, the stage's slot is released (`empty`) and they are multiplied
+// -- the ring refills while the second half computes.  A fragments: 16 rows;
+// B fragments: NTL live query tiles of 8 (an x2 load for one tile, an x4 for
+// two).  The rows' squares go to ss0 (row g) and ss1 (row g + 8).
+template <int KH, int NTL, int NT>
+__device__ __forceinline__ void half_mma(uint32_t sb, uint32_t a_off, uint32_t b_off,
+                                         uint32_t b_off_last, int k0, int ks,
+                                         uint32_t (&af)[KH][4], uint32_t (&bf)[KH][2 * NTL]) {
+#pragma unroll
+    for (int i = 0; i < KH; ++i) {
+        const int k16 = k0 + i;
+        if (k16 < ks) {
+            ldsm_x4(sb + a_off + k16 * 32, af[i]);
+            if constexpr (NTL == 1) {
+                uint32_t b2[2];
+                ldsm_x2(sb + b_off_last + k16 * 32, b2);
+                bf[i][0] = b2[0];
+                bf[i][1] = b2[1];
+            } else {
+                uint32_t b4[4];
+                ldsm_x4(sb + b_off + k16 * 32, b4);
+#pragma unroll
+                for (int e = 0; e < 4; ++e) bf[i][e] = b4[e];
+            }
+        }
+    }
+}
+
+template <int KH, int NTL, int NT>
+__device__ __forceinline__ void half_math(int k0, int ks, const uint32_t (&af)[KH][4],
+                                          const uint32_t (&bf)[KH][2 * NTL],
+                                          float (&acc)[NT][4], float &ss0, float &ss1) {
+#pragma unroll
+    for (int i = 0; i < KH; ++i) {
+        if (k0 + i < ks) {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float lo = bf16lo(af[i][e]), hi = bf16hi(af[i][e]);
+                if (e & 1) {
+                    ss1 = fmaf(lo, lo, ss1);
+                    ss1 = fmaf(hi, hi, ss1);
+                } else {
+                    ss0 = fmaf(lo, lo, ss0);
+                    ss0 = fmaf(hi, hi, ss0);
+                }
+            }
+            mma_16816(acc[0], af[i], bf[i][0], bf[i][1]);
+            if constexpr (NTL == 2) mma_16816(acc[1], af[i], bf[i][2], bf[i][3]);
+        }
+    }
+}
+
+template <int KMAX, int NTL, int NT>
+__device__ __forceinline__ void stage_mma(uint32_t sb, uint32_t a_off, uint32_t b_off,
+                                          uint32_t b_off_last, int ks, uint64_t *empty,
+                                          int lane, float (&acc)[NT][4], float &ss0,
+                                          float &ss1) {
+    static_assert(NTL <= NT && NTL <= 2 && KMAX % 2 == 0, "one or two live query tiles");
+    constexpr int KH = KMAX / 2;
+    uint32_t af[KH][4];
+    uint32_t bf[KH][2 * NTL];
+    half_mma<KH, NTL, NT>(sb, a_off, b_off, b_off_last, 0, ks, af, bf);
+    half_math<KH, NTL, NT>(0, ks, af, bf, acc, ss0, ss1);
+    half_mma<KH, NTL, NT>(sb, a_off, b_off, b_off_last, KH, ks, af, bf);
+    // (the warp's shared-memory reads are ordered before lane 0's arrive by
+    // the warp barrier and the arrive's release semantics)
+    __syncwarp();
+    if (lane == 0) mbar_arrive(empty);
+    half_math<KH, NTL, NT>(KH, ks, af, bf, acc, ss0, ss1);
+}
 
 struct UnionShared {
     int sel[kUnionMaxB];    // the fallback sequences
@@ -369,37 +451,16 @@ __global__ void __launch_bounds__(kUThreads, 1) union_mma_kernel(UnionArgs args)
             const int kl = min(KC, d - kc * KC);
             const int ks = max(0, min(KW, kl - kg * KW)) / 16;  // k16 steps of this warp
             const uint32_t sb = ring_s + (uint32_t)(s * stage_bytes);
-#pragma unroll 2
-            for (int k16 = 0; k16 < ks; ++k16) {
-                uint32_t af[4];
-                ldsm_x4(sb + a_off + k16 * 32, af);
-                // the squares of the fragment's elements (af[0], af[2]: row g;
-                // af[1], af[3]: row g + 8) on the CUDA cores, next to the MMAs
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const float lo = bf16lo(af[e]), hi = bf16hi(af[e]);
-                    if (e & 1) {
-                        ss1 = fmaf(lo, lo, ss1);
-                        ss1 = fmaf(hi, hi, ss1);
-                    } else {
-                        ss0 = fmaf(lo, lo, ss0);
-                        ss0 = fmaf(hi, hi, ss0);
-                    }
-                }
-#pragma unroll
-                for (int j = 0; j < NT; j += 2) {
-                    if (j >= ntl) break;
-                    uint32_t bf[4];
-                    ldsm_x4(sb + (j + 1 < ntl ? b_off : b_off_last) + (uint32_t)(j * 8 * PITCH) +
-                                k16 * 32,
-                            bf);
-                    mma_16816(acc[j], af, bf[0], bf[1]);
-                    if (j + 1 < ntl) mma_16816(acc[j + 1], af, bf[2], bf[3]);
-                }
-            }
+            // the warp's fragments of the whole stage go to registers first,
+            // so the slot is released before the arithmetic
+            if (ntl == 1)
+                stage_mma<16, 1>(sb, a_off, b_off, b_off_last, ks, &empty[s], lane, acc, ss0, ss1);
+            else
+                stage_mma<8, 2>(sb, a_off, b_off, b_off_last, ks, &empty[s], lane, acc, ss0, ss1);
+        } else {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
         }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty[s]);
         if (kc != nk - 1) continue;
 
         // ---- the tile's epilogue: the rows' |row|^2 over the quad of lanes
