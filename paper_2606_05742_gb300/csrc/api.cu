@@ -135,7 +135,7 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
     // the distinct tokens of the selected histories and the plan over them,
     // the scores of the distinct tokens, then their positions
-    const bool uni = union_applies(B, ld, emb->dim);  // every table row read once
+    const bool uni = union_applies(B, ld, emb->dim, emb->vocab);  // every table row read once
     DedupeLaunch da{tokens, ld,   lengths, B,       emb->vocab, active, nullptr, status,
                     false,  true, nullptr, true,    k,          cand,   score,   n_cand};
     da.union_insert = uni;
@@ -223,7 +223,7 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
         // small batches: the fallback reads each table row of the batch's
         // union once, scored against every fallback query by the tensor
         // cores (csrc/union.cu), instead of once per sequence
-        const bool uni = emb && union_applies(B, ld, emb->dim);
+        const bool uni = emb && union_applies(B, ld, emb->dim, emb->vocab);
         if (emb) {  // Eq. 4 over token embeddings, scored once per distinct token
             // lists for the fallback sequences, and for lexical hits too when
             // those draft successors (their backoff needs them)

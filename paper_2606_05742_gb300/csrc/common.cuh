@@ -72,12 +72,12 @@ struct Workspace {
     // the union of the fallback sequences' distinct tokens (two-representation
     // mode, small batches: every table row is read once per step, not once per
     // sequence holding it); NULL where union_enabled() is false
-    uint32_t *uhash;         // [UH] token + 1 (0: empty), after htab (one memset clears both)
+    uint32_t *uhash;         // [UH] union bitmap (bit u: token u), after htab (one memset clears both)
     int32_t *ucount;         // [1]  union tokens (a counter)
     int32_t *ulist;          // [B * ld] the union's tokens, in no particular order
     int32_t *rep_pos;        // [B][ld] latest position of each listed token
     float *score_pos;        // [B][ld] Eq. 4 score of the token whose latest position it is
-    int64_t UH;              // union hash slots (a power of two >= 2 B (ld-1))
+    int64_t UH;              // union bitmap words (a power of two >= 2 B (ld-1))
     int64_t H;               // hash slots per sequence (a power of two >= 2 (ld-1))
     size_t htab_bytes;       // htab and uhash
     size_t counters_bytes;
@@ -743,7 +743,7 @@ struct UnionLaunch {
 };
 cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t s);
 // Whether the union pass serves a batch of this shape.
-bool union_applies(int32_t B, int64_t ld, int32_t d);
+bool union_applies(int32_t B, int64_t ld, int32_t d, int32_t vocab);
 
 struct VerifyLaunch {
     const uint16_t *logits;  // [B][N][V] bf16

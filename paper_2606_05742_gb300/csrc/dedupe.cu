@@ -176,27 +176,19 @@ __device__ int mark_chunk(const DedupeLaunch &a, const Workspace &ws, int b, int
     return mine;
 }
 
-// Inserts token u into the union hash (open addressing, token + 1 as the
-// key); a table that runs full raises ADAPLD_DEV_INTERNAL (it is sized for
-// twice the batch's positions, so it never does).
-__device__ __forceinline__ void union_insert(uint32_t *U, int64_t UH, int u, int32_t *dst) {
-    const uint32_t key = (uint32_t)u + 1u;
-    uint64_t h = hash32((uint32_t)u) & (uint64_t)(UH - 1);
-    for (int64_t probe = 0; probe < UH; ++probe) {
-        const uint32_t old = atomicCAS(U + h, 0u, key);
-        if (old == 0u || old == key) return;
-        h = (h + 1) & (uint64_t)(UH - 1);
-    }
-    atomicOr(dst, ADAPLD_DEV_INTERNAL);
+// Adds token u to the union: bit u of the union bitmap (a reduction, no
+// reply awaited).
+__device__ __forceinline__ void union_insert(uint32_t *U, int u) {
+    atomicOr(U + (u >> 5), 1u << (u & 31));
 }
 
 // Writes the marked positions' tokens of the chunk starting at j0 in
 // position order to out (s_word: the chunk's 128 words in shared memory),
-// and with pos_out their positions, inserting each token into the union hash
+// and with pos_out their positions, adding each token to the union bitmap
 // when uh is given.  One scan over the word counts gives every offset.
 __device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32_t *s_word,
                               int *s_off, int64_t *s_scan, int32_t *out, int64_t room,
-                              int32_t *dst, int32_t *pos_out, uint32_t *uh, int64_t UH) {
+                              int32_t *dst, int32_t *pos_out, uint32_t *uh) {
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     const uint32_t w = t < kWordsPerChunk ? s_word[t] : 0u;
     int64_t all;
@@ -215,7 +207,7 @@ __device__ void scatter_chunk(const DedupeLaunch &a, int b, int j0, const uint32
             const int u = canon(M[j], a.vocab);
             out[o] = u;
             if (pos_out) pos_out[o] = j;
-            if (uh) union_insert(uh, UH, u, dst);
+            if (uh) union_insert(uh, u);
         }
     }
 }
@@ -280,7 +272,7 @@ __global__ void __launch_bounds__(kThreads1) rep_count_kernel(DedupeArgs args) {
             const bool uni = joins_union(a, ws, b);
             scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld, a.ld,
                           ws.dev_status, uni ? ws.rep_pos + (int64_t)b * a.ld : nullptr,
-                          uni ? ws.uhash : nullptr, ws.UH);
+                          uni ? ws.uhash : nullptr);
             if (t == 0) {
                 ws.rep_len[b] = (int)total + 1;
                 ws.rep_tok[(int64_t)b * a.ld + total] = M[len - 1];  // the anchor (as stored)
@@ -346,8 +338,7 @@ __global__ void __launch_bounds__(kThreads1) rep_scatter_kernel(DedupeArgs args)
     const bool uni = joins_union(a, ws, b);
     scatter_chunk(a, b, j0, s_word, s_off, s_scan, ws.rep_tok + (int64_t)b * a.ld + off,
                   a.ld - off, ws.dev_status,
-                  uni ? ws.rep_pos + (int64_t)b * a.ld + off : nullptr, uni ? ws.uhash : nullptr,
-                  ws.UH);
+                  uni ? ws.rep_pos + (int64_t)b * a.ld + off : nullptr, uni ? ws.uhash : nullptr);
 }
 
 // ---------------------------------------------------------------- expansion

@@ -9,11 +9,10 @@
 // fallback sequences (the anchors' table rows) form one dense contraction,
 // union rows x queries over d, which runs on the tensor cores:
 //
-//  union_compact_kernel  the union hash (filled by the list scatter) into a
-//      list of tokens: each CTA compacts a slot range and appends it with one
-//      atomic add per 2048 slots (the list's order does not matter: every
-//      score is computed the same way wherever its row lands; a token-ordered
-//      list, tried, was slower).
+//  union_compact_kernel  the union bitmap over the vocabulary (a bit per
+//      token, set by the list scatter with one atomic OR) into a list of
+//      tokens in a scrambled order (every score is computed the same way
+//      wherever its row lands; a token-ordered list read slower).
 //  union_mma_kernel<NT>  persistent, one CTA per SM: 2 producer warps and
 //      8 MMA warps.  A tile is 16 union rows; its K dimension (d) streams
 //      through a ring of stages of 2048-element slices (4 KB; 2 KB when more
@@ -64,7 +63,9 @@ struct UnionArgs {
 
 struct CompactArgs {
     Workspace ws;
-    int64_t cap;  // ulist entries (B * ld)
+    int64_t cap;      // ulist entries (B * ld)
+    uint32_t nwords;  // bitmap words covering the vocabulary
+    uint32_t nsteps;  // the power of two >= nwords the visiting order runs over
 };
 
 // Whether sequence b is scored by the union pass and listed (the same test
@@ -78,23 +79,32 @@ __device__ __forceinline__ bool union_seq(const UnionLaunch &a, const Workspace 
     return a.active ? a.active[b] != 0 : true;
 }
 
+// The union bitmap's set bits into the union list.  Word w is visited at
+// step i with w = i * 0x9E3779B1 mod 2^n (odd multiplier: a bijection of the
+// 2^n >= nwords steps), so the list is in scrambled token order: tiles of
+// consecutive entries, which the MMA kernel's CTAs take in turn, read rows
+// from all over the table (a token-ordered list read slower).  Each CTA
+// takes a range of steps and appends its tokens with one atomic add per
+// 2048 steps.
 __global__ void __launch_bounds__(256) union_compact_kernel(CompactArgs args) {
     const Workspace &ws = args.ws;
     __shared__ int64_t s_scan[32];
     __shared__ int s_base;
     pdl_wait_then_release();
-    constexpr int kPer = 8;  // slots per thread and step
-    const int64_t per_cta = (ws.UH + gridDim.x - 1) / gridDim.x;
-    const int64_t lo = (int64_t)blockIdx.x * per_cta;
-    const int64_t hi = min(lo + per_cta, ws.UH);
-    for (int64_t base = lo; base < hi; base += 256 * kPer) {
-        uint32_t key[kPer];
+    constexpr int kPer = 8;  // steps per thread and round
+    const uint32_t nsteps = args.nsteps;  // a power of two >= nwords
+    const uint32_t per_cta = (nsteps + gridDim.x - 1) / gridDim.x;
+    const uint32_t lo = blockIdx.x * per_cta;
+    const uint32_t hi = min(lo + per_cta, nsteps);
+    for (uint32_t base = lo; base < hi; base += 256 * kPer) {
+        uint32_t word[kPer], widx[kPer];
         int mine = 0;
 #pragma unroll
         for (int e = 0; e < kPer; ++e) {
-            const int64_t i = base + (int64_t)e * 256 + threadIdx.x;
-            key[e] = i < hi ? __ldcg(ws.uhash + i) : 0u;
-            mine += key[e] != 0u;
+            const uint32_t i = base + (uint32_t)e * 256 + threadIdx.x;
+            widx[e] = (i * 0x9E3779B1u) & (nsteps - 1u);
+            word[e] = (i < hi && widx[e] < args.nwords) ? __ldcg(ws.uhash + widx[e]) : 0u;
+            mine += __popc(word[e]);
         }
         int64_t total;
         const int64_t ex = block_exclusive_scan(mine, &total, s_scan);
@@ -103,8 +113,9 @@ __global__ void __launch_bounds__(256) union_compact_kernel(CompactArgs args) {
         int o = s_base + (int)ex;
 #pragma unroll
         for (int e = 0; e < kPer; ++e)
-            if (key[e] != 0u && idx_ok(o, 0, args.cap, ws.dev_status))
-                ws.ulist[o++] = (int)(key[e] - 1u);
+            for (uint32_t m = word[e]; m; m &= m - 1)
+                if (idx_ok(o, 0, args.cap, ws.dev_status))
+                    ws.ulist[o++] = (int)(widx[e] * 32u + (uint32_t)(__ffs(m) - 1));
         __syncthreads();  // before s_base is rewritten
     }
 }
@@ -631,16 +642,21 @@ cudaError_t launch_mma(const UnionArgs &args, int sms, cudaStream_t s) {
 
 }  // namespace
 
-bool union_applies(int32_t B, int64_t ld, int32_t d) {
+bool union_applies(int32_t B, int64_t ld, int32_t d, int32_t vocab) {
     if (const char *e = std::getenv("ADAPLD_EMB_UNION"))  // A/B switch for measurements
         if (e[0] == '0') return false;
-    return union_enabled(B, ld) && d % 16 == 0;
+    // the bitmap (the workspace's UH words) must cover the vocabulary
+    return union_enabled(B, ld) && d % 16 == 0 &&
+           ((int64_t)vocab + 31) / 32 <= hash_slots((int64_t)B * (ld - 1) + 1);
 }
 
 cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t s) {
     const int sms = device_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
-    CompactArgs ca{ws, (int64_t)a.B * a.ld};
+    const uint32_t nwords = (uint32_t)(((int64_t)a.vocab + 31) / 32);
+    uint32_t nsteps = 1;
+    while (nsteps < nwords) nsteps <<= 1;
+    CompactArgs ca{ws, (int64_t)a.B * a.ld, nwords, nsteps};
     cudaError_t e = launch_dependent(union_compact_kernel, dim3(2 * sms), dim3(256), 0, s, ca);
     if (e != cudaSuccess) return e;
     UnionArgs ua{a, ws};
