@@ -915,6 +915,18 @@ def test_embedding_mode_extreme_histories(kind):
         check_all(w, run_step(w, P, emb=E), P, emb=E)
 
 
+def test_embedding_mode_vocabulary_beyond_the_union_bitmap():
+    """A batch whose table has more rows than the union pass's bitmap covers
+    (short histories, a large vocabulary) keeps the per-sequence lists; the
+    results match the oracle all the same, as does a batch just inside."""
+    for L, V in ((20, 50000), (200, 4000)):
+        w = synth.make_workload(2, B=3, L=L, d=32, V=V, nohit=1.0, seed=86)
+        E = synth.make_embeddings(w, V, 32, 86)
+        for tau in (0.1, NEG_INF):
+            P = P_of(w, tau=tau)
+            check_all(w, run_step(w, P, emb=E), P, emb=E)
+
+
 def test_embedding_mode_token_out_of_table():
     """A token id outside the table reads row 0 and is flagged, no fault."""
     w = synth.make_workload(2, B=3, L=400, d=32, V=1000, nohit=1.0, seed=73)
