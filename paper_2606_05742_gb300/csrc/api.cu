@@ -131,11 +131,12 @@ int adapld_embedding_topk(const int32_t *tokens, int64_t ld, const int32_t *leng
     ADAPLD_TRY(check_ws(ws, ws_bytes, B, ld, 1));
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, 1);
+    const bool uni = union_applies(B, ld, emb->dim, emb->vocab);  // every table row read once
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
-    ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
+    ADAPLD_TRY(cuda_status(
+        cudaMemsetAsync(w.htab, 0, union_clear_bytes(w, B, emb->vocab, uni), s)));
     // the distinct tokens of the selected histories and the plan over them,
     // the scores of the distinct tokens, then their positions
-    const bool uni = union_applies(B, ld, emb->dim, emb->vocab);  // every table row read once
     DedupeLaunch da{tokens, ld,   lengths, B,       emb->vocab, active, nullptr, status,
                     false,  true, nullptr, true,    k,          cand,   score,   n_cand};
     da.union_insert = uni;
@@ -179,7 +180,9 @@ int adapld_build_draft_tree(const int32_t *tokens, int64_t ld, const int32_t *le
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.dev_status, 0, w.counters_bytes, s)));
-    if (emb) ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
+    if (emb)
+        ADAPLD_TRY(cuda_status(
+            cudaMemsetAsync(w.htab, 0, union_clear_bytes(w, B, emb->vocab, false), s)));
     TreeLaunch a{tokens, ld, lengths, reps, d, query, B, hit_kind, cand, score, n_cand,
                  next_topk, next_topk ? Kn : 0, *p, *out, status};
     if (emb) a.emb = *emb;
@@ -198,8 +201,14 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
     cudaStream_t s = (cudaStream_t)stream;
     Workspace w = layout_workspace(ws, B, ld, p->branch_width);
     const bool semantic = !(p->flags & ADAPLD_NO_SEMANTIC);
+    // small batches: the fallback reads each table row of the batch's union
+    // once, scored against every fallback query by the tensor cores
+    // (csrc/union.cu), instead of once per sequence
+    const bool uni = emb && semantic && union_applies(B, ld, emb->dim, emb->vocab);
     // (the workspace counters are zeroed by the lexical kernel)
-    if (emb) ADAPLD_TRY(cuda_status(cudaMemsetAsync(w.htab, 0, w.htab_bytes, s)));
+    if (emb)
+        ADAPLD_TRY(cuda_status(
+            cudaMemsetAsync(w.htab, 0, union_clear_bytes(w, B, emb->vocab, uni), s)));
 
     ADAPLD_TRY(record(ev ? ev->lexical_begin : nullptr, s));
     LexLaunch la{tokens, ld, lengths, B, p->n_max, p->k, out->hit_kind, out->match_n, out->cand,
@@ -220,10 +229,6 @@ int adapld_step_ex(const int32_t *tokens, int64_t ld, const int32_t *lengths,
         SemLaunch sa{reps, ld, d, query, lengths, nullptr, B, p->k, p->tau, out->cand, out->score,
                      out->n_cand, out->hit_kind, true};
         sa.plan_from_outcome = !emb && small_plan;
-        // small batches: the fallback reads each table row of the batch's
-        // union once, scored against every fallback query by the tensor
-        // cores (csrc/union.cu), instead of once per sequence
-        const bool uni = emb && union_applies(B, ld, emb->dim, emb->vocab);
         if (emb) {  // Eq. 4 over token embeddings, scored once per distinct token
             // lists for the fallback sequences, and for lexical hits too when
             // those draft successors (their backoff needs them)

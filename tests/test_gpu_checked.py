@@ -80,7 +80,8 @@ def test_checked_build_single_cache(libs, monkeypatch, cfg, B, L, d, seed, over)
 
 @pytest.mark.parametrize("cfg,B,L,d,de,V,seed", [(2, 8, 1500, 128, 64, 4096, 0),
                                                  (4, 20, 500, 64, 8, 2048, 3),
-                                                 (5, 3, 20000, 64, 256, 4096, 5)])
+                                                 (5, 3, 20000, 64, 256, 4096, 5),
+                                                 (4, 150, 300, 32, 64, 2500, 12)])
 def test_checked_build_embeddings(libs, monkeypatch, cfg, B, L, d, de, V, seed):
     w = synth.make_workload(cfg, B=B, L=L, d=d, V=V, seed=seed, nohit=0.6)
     E = synth.make_embeddings(w, V, de, seed)

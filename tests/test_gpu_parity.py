@@ -719,6 +719,10 @@ EMB_CASES = [  # (cfg, B, L, d, de, V, seed)
     (5, 3, 20000, 64, 256, 4096, 5),    # several chunks and slices per history
     (2, 16, 900, 64, 512, 3000, 6),     # 9-16 fallback queries: two query tiles
     (3, 12, 1500, 64, 1040, 4000, 7),   # a table width that ends in a partial slice
+    # batches above 16 sequences (the per-sequence lists whatever the switch)
+    (4, 24, 700, 64, 144, 2048, 9),
+    (2, 40, 900, 64, 256, 3000, 8),
+    (4, 220, 400, 32, 64, 2500, 11),    # more than 128 fallback sequences
 ]
 
 
@@ -728,7 +732,8 @@ def test_embedding_mode(cfg, B, L, d, de, V, seed, union, monkeypatch):
     """Eq. 4 over token embeddings, Eq. 6 rerank of the semantic candidates,
     and the successor backoff of Sec. 3.5, against the oracle; through the
     union pass (batches of up to 16: every table row of the batch read once,
-    tensor cores) and through the per-sequence lists (ADAPLD_EMB_UNION=0)."""
+    tensor cores) and through the per-sequence lists (ADAPLD_EMB_UNION=0,
+    and every batch above 16)."""
     monkeypatch.setenv("ADAPLD_EMB_UNION", union)
     w = synth.make_workload(cfg, B=B, L=L, d=d, V=V, nohit=0.6, seed=seed)
     E = synth.make_embeddings(w, V, de, seed)
@@ -944,11 +949,14 @@ def test_embedding_mode_token_out_of_table():
     assert not st[0] & native.SEQ_BAD_TOKEN
 
 
-def test_full_size_embedding_config5():
-    """Config 5 with a 128256 x 8192 embedding table (2.1 GB), launched as the
-    benchmark's embedding mode does; every sequence against the oracle."""
-    w = synth.make_workload(5, device="cuda")
-    V, de = synth.CONFIGS[5]["V"], w.d
+@pytest.mark.parametrize("cfg", [2, 3, 4, 5])
+def test_full_size_embedding(cfg):
+    """A full-size workload with a vocabulary x d embedding table (config 5:
+    128256 x 8192, 2.1 GB), launched as the benchmark's embedding mode does;
+    every sequence against the oracle.  Config 5 (8 sequences) takes the
+    union pass, configs 2-4 (32-256 sequences) the per-sequence lists."""
+    w = synth.make_workload(cfg, device="cuda")
+    V, de = synth.CONFIGS[cfg]["V"], w.d
     Ed = synth.make_embeddings(w, V, de, 0)
     P = P_of(w)
     eng = native.Engine(w.B, w.ld, w.d, params(P))
@@ -958,7 +966,7 @@ def test_full_size_embedding_config5():
     g = eng.out.to_host()
     E = Ed.view(torch.int16).cpu().numpy().view(np.uint16)
     rep = compare_device_workload(w, g, P, emb=E)
-    print(f"config 5 with embeddings: {rep}")
+    print(f"config {cfg} with embeddings: {rep}")
     assert rep.tie_resolved == 0, rep
     for b in [int(x) for x in w.forced]:
         assert g["hit_kind"][b] == 2
