@@ -16,6 +16,14 @@ std::atomic<unsigned long long> g_launches{0};  // kernels enqueued by the libra
 
 int cuda_status(cudaError_t e) { return e == cudaSuccess ? ADAPLD_OK : ADAPLD_ERR_CUDA; }
 
+// Bytes from ws.htab that a two-representation call clears before the list
+// kernels: the per-sequence hashes and, with the union pass, the bitmap words
+// that cover the vocabulary (not the whole bitmap area the workspace holds).
+size_t union_clear_bytes(const Workspace &w, int32_t B, int32_t vocab, bool uni) {
+    const size_t hashes = sizeof(unsigned long long) * (size_t)B * (size_t)w.H;
+    return uni ? hashes + sizeof(uint32_t) * (size_t)(((int64_t)vocab + 31) / 32) : hashes;
+}
+
 int record(void *ev, cudaStream_t s) {
     if (!ev) return ADAPLD_OK;
     return cuda_status(cudaEventRecord((cudaEvent_t)ev, s));

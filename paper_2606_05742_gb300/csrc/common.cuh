@@ -744,10 +744,6 @@ struct UnionLaunch {
 cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t s);
 // Whether the union pass serves a batch of this shape.
 bool union_applies(int32_t B, int64_t ld, int32_t d, int32_t vocab);
-// Bytes from ws.htab that a two-representation call clears before the list
-// kernels: the per-sequence hashes and, with the union pass, the bitmap words
-// that cover the vocabulary (not the whole bitmap area).
-size_t union_clear_bytes(const Workspace &ws, int32_t B, int32_t vocab, bool uni);
 
 struct VerifyLaunch {
     const uint16_t *logits;  // [B][N][V] bf16

@@ -650,11 +650,6 @@ bool union_applies(int32_t B, int64_t ld, int32_t d, int32_t vocab) {
            ((int64_t)vocab + 31) / 32 <= hash_slots((int64_t)B * (ld - 1) + 1);
 }
 
-size_t union_clear_bytes(const Workspace &ws, int32_t B, int32_t vocab, bool uni) {
-    const size_t hashes = sizeof(unsigned long long) * (size_t)B * (size_t)ws.H;
-    return uni ? hashes + sizeof(uint32_t) * (size_t)(((int64_t)vocab + 31) / 32) : hashes;
-}
-
 cudaError_t launch_union(const UnionLaunch &a, const Workspace &ws, cudaStream_t s) {
     const int sms = device_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
