@@ -444,9 +444,23 @@ __device__ __forceinline__ void scan_branches(const int *s_tok, int64_t p0, int6
 // Publishes the successor-candidate count of branch w of sequence b.  A
 // branch token that never occurs earlier backs off (Sec. 3.5) to the
 // embedding fallback with the branch token as the anchor: with a table, the
-// (sequence, branch) pair is registered for the gathered pass.
+// (sequence, branch) pair is registered for the gathered pass.  On the step
+// path a semantic hit's own anchor never occurred earlier either, and its
+// backoff -- Eq. 4 with that anchor as the query over the same positions,
+// threshold and k -- is exactly the fallback this step already ran: its
+// candidate set (nc entries of s_cand, in any order; Eq. 14 takes a
+// maximum) is copied instead of being scored again.  reuse: the sequence is
+// such a hit, anchor its token.
 __device__ __forceinline__ void register_successors(const TreeLaunch &a, const Workspace &ws,
-                                                    int b, int w, int total, int token) {
+                                                    int b, int w, int total, int token,
+                                                    bool reuse, int anchor, int nc,
+                                                    const int *s_cand) {
+    if (total == 0 && reuse && token == anchor) {
+        int32_t *dst = ws.succ + ((int64_t)b * ws.W + w) * kMaxK;
+        for (int i = 0; i < nc; ++i) dst[i] = s_cand[i];
+        ws.succ_n[(int64_t)b * ws.W + w] = nc;
+        return;
+    }
     ws.succ_n[(int64_t)b * ws.W + w] = total;
     if (total == 0 && a.emb.table) {
         const int idx = atomicAdd(ws.npairs, 1);
@@ -626,6 +640,9 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
     const int nld = (int)min((int64_t)kSlice4 + 1, a.ld - p0);
     for (int i = t; i < nld; i += kThreads4) cp_async4(s_tok + i, M + p0 + i);
     const SeqView v = view_of(a, b);
+    // a semantic hit of this step reuses its fallback for its anchor's backoff
+    const bool reuse = a.lists_ready && v.sem && v.valid;
+    const int anchor = reuse ? __ldg(M + v.len - 1) : 0;
     cp_async_wait_all();  // (also before an exit: the copies target this CTA's memory)
     if (!v.need_succ && !(FUSED && sl == 0)) return;
     __syncthreads();
@@ -707,7 +724,8 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
         }
         if (lane == 0) {
             if (single)
-                register_successors(a, ws, b, w, min(cnt, k), s_br[w]);
+                register_successors(a, ws, b, w, min(cnt, k), s_br[w], reuse, anchor, v.nc,
+                                    s_cand);
             else
                 part[0] = min(cnt, k);
         }
@@ -727,7 +745,8 @@ __global__ void __launch_bounds__(kThreads4, U == 8 ? 2 : 1) succ_scan_kernel(Tr
                 (int)gridDim.x, k, [&](int s2) { return __ldcg(pw + s2 * stride); },
                 [&](int s2, int i) { return __ldcg(pw + s2 * stride + 1 + i); },
                 ws.succ + ((int64_t)b * ws.W + w) * kMaxK);
-            if (lane == 0) register_successors(a, ws, b, w, total, s_br[w]);
+            if (lane == 0)
+                register_successors(a, ws, b, w, total, s_br[w], reuse, anchor, v.nc, s_cand);
         }
     }
     if (!FUSED && (v.lex || v.rr) && t < v.nc) {
