@@ -578,6 +578,26 @@ def test_successor_backoff_bruteforce(seed):
     assert oracle.successor_candidates(M, L, R, d, js, V - 1, k) == ([], [])
 
 
+@pytest.mark.parametrize("seed", range(20))
+def test_anchor_backoff_is_the_fallback(seed):
+    """A semantic hit's anchor never occurred earlier (else the lexical match
+    holds at n = 1); when it is a branch token its backoff of Sec. 3.5 -- Eq. 4
+    with the anchor as the query -- returns the fallback's own candidate list,
+    which the GPU step takes over instead of scoring the rows again."""
+    rng = np.random.default_rng(950 + seed)
+    V, L, d, k = 9, int(rng.integers(3, 40)), 8, int(rng.integers(1, 6))
+    M = rng.integers(0, V - 1, size=L).astype(np.int32)
+    M[-1] = V - 1                                   # the anchor: no earlier occurrence
+    E = rows_to_bf16(rng.integers(-2, 3, size=(V, 3)).tolist(), d)
+    R = rows_to_bf16(rng.integers(-2, 3, size=(L, 3)).tolist(), d)
+    js = int(rng.integers(0, L - 1))
+    assert oracle.lexical(M, 3, k)[0] == 0          # no lexical hit
+    for tau in (0.1, NEG_INF):
+        c, _ = oracle.semantic_emb(M, L, E, k, tau)
+        t, _ = oracle.successor_candidates_emb(M, L, R, d, E, tau, js, int(M[-1]), k)
+        assert t == c
+
+
 # ---------------------------------------------------- greedy verification
 def _logits_rows(g, case, N, V):
     L = np.zeros((N, V), np.float32)
