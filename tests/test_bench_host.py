@@ -1,5 +1,7 @@
 """Host-side helpers of bench.py (no GPU): ablation flag parsing and the
 algorithmic byte count under each variant."""
+import os
+
 import numpy as np
 import pytest
 
@@ -117,3 +119,30 @@ def test_workload_config_is_shared_by_both_arms():
     assert a["B"] == 8 and a["L"] == 131072 and a["d"] == 8192
     r = bench.workload_config(2, batch=4, flags=native.NO_SUCC)
     assert r["B"] == r["global_batch"] == 4 and r["flags"] == native.NO_SUCC
+
+
+def test_profile_summaries_describe_the_current_sources():
+    """Every ncu summary under profiles/ records the sha256 of the sources it
+    was captured against; each must match the source as it stands, or the
+    summary must say how the current file (named by its current hash)
+    differs.  The semantic kernel's summary, which the benchmark scales into
+    roofline.traffic, must match exactly."""
+    import glob
+    import hashlib
+    import re
+
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    csrc = os.path.join(root, "paper_2606_05742_gb300", "csrc")
+    current = {os.path.basename(f): hashlib.sha256(open(f, "rb").read()).hexdigest()
+               for f in glob.glob(os.path.join(csrc, "*.cu*"))}
+    summaries = sorted(glob.glob(os.path.join(root, "profiles", "*.md")))
+    assert summaries
+    for path in summaries:
+        text = open(path).read()
+        recorded = re.findall(r"([a-z_]+\.cuh?) sha256 ([0-9a-f]{64})", text)
+        assert recorded, f"{os.path.basename(path)} records no source hashes"
+        for name, h in recorded:
+            assert name in current, (path, name)
+            assert h == current[name] or current[name] in text, (
+                f"{os.path.basename(path)}: {name} changed since the capture")
+    assert bench.semantic_traffic(10**9) is not None
